@@ -37,9 +37,11 @@ SUPPORTED_BITS = (1, 2, 4, 8)
 
 def _all_finite_f16_sorted():
     bits = np.arange(0x10000, dtype=np.uint32).astype(np.uint16)
-    vals = bits.view(np.float16).astype(np.float64)
-    vals = vals[np.isfinite(vals)]
-    return np.unique(vals)  # sorted, -0 and +0 merged into one 0
+    finite = (bits & 0x7C00) != 0x7C00  # exponent field not all ones
+    vals = bits[finite].view(np.float16).astype(np.float64)
+    vals = np.unique(vals + 0.0)  # sorted; x + 0.0 turns -0 into +0
+    assert not np.signbit(vals[vals == 0]).any()
+    return vals
 
 
 _F16_TABLE = _all_finite_f16_sorted()

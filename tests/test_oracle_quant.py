@@ -44,6 +44,9 @@ def test_round_up_f16_is_least_upper_fp16():
         assert Fraction(float(rv)) >= Fraction(float(xv))
         if rv > 0:
             assert Fraction(float(_prev16(rv))) < Fraction(float(xv))
+    # an exact zero rounds to +0, whatever order the table was built in
+    z = quant.round_up_f16(np.array([0.0, -0.0]))
+    assert z.view(np.uint16).tolist() == [0, 0]
     # fp16 values map to themselves
     h = rng.standard_normal(1000).astype(np.float16)
     h = np.abs(h)
@@ -124,7 +127,7 @@ def test_one_bit_random_groups_overshoot_at_most_one_ulp():
 def test_constant_group(bits):
     x = np.full((3, 32), [[1.5], [-7.25], [0.0]], dtype=np.float16)
     c, s, z = quant.quantize_groups(x, bits)
-    assert np.all(s == 0) and np.all(c == 0)
+    assert np.all(s.view(np.uint16) == 0) and np.all(c == 0)  # scale is +0
     assert np.array_equal(quant.dequantize_groups(c, s, z), x.astype(np.float64))
 
 
