@@ -1,0 +1,604 @@
+#!/usr/bin/env python3
+"""Decode-step benchmark of the packed low-bit KV cache + DGAP epilogue.
+
+A step is one pass of the whole hot path over one batch: for every layer,
+kvq_pack appends the step's token and kvq_decode_attn attends over the cache;
+then dgap_restore runs once on the step's logits.  Default workload:
+Llama-3.1-8B-shaped K1V1 decode (batch 1, 32 q / 8 kv heads, head_dim 128,
+context 32768, 32 layers with distinct seeded caches, logits [1, 128256],
+K = 32, hidden 256, tau 0.60).  The per-step packed KV (~552 MB) is larger
+than L2, so every step streams it from HBM.
+
+The step runs as three CUDA graphs (packs, attentions, epilogue) replayed
+back to back, with CUDA events between them on the launching stream; the
+attention events give the dominant kernel's average launch duration for the
+roofline.  One JSON line is printed by rank 0.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the CPU oracle on the same config
+"""
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+DEFAULT_WORKLOAD = "llama8b-k1v1-32k"
+METRIC = "packed-KV decode attn HBM GB/s (% of GB300 peak); DGAP epilogue µs/step"
+FALLBACK_HBM_GBS = 6800.0
+DGAP_K, DGAP_HIDDEN, DGAP_TAU = 32, 256, 0.60
+ATTN_PROFILE = ROOT / "profiles" / "attn_llama8b_k1v1_32k.md"
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=2000)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", default="kvq", choices=["kvq", "reference"])
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--bits", type=int, default=0, help="bit width for the sweep workload")
+    p.add_argument("--layers", type=int, default=0, help="override the layer count")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--cpu-worker", default="", help=argparse.SUPPRESS)
+    return p.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# Workload description and algorithmic bytes
+# ---------------------------------------------------------------------------
+
+
+def workload_spec(args):
+    from paper_2607_16248_gb300 import synth
+    if args.workload not in synth.WORKLOADS:
+        raise SystemExit(f"unknown workload {args.workload}; one of {sorted(synth.WORKLOADS)}")
+    spec = dict(synth.WORKLOADS[args.workload])
+    if isinstance(spec["bits"], tuple):
+        spec["bits"] = args.bits or spec["bits"][0]
+    elif args.bits:
+        spec["bits"] = args.bits
+    if args.layers:
+        spec["layers"] = args.layers
+    return spec
+
+
+def packed_len(L, R=128):
+    return 32 * (max(L - R, 0) // 32)
+
+
+def attn_bytes(L, hkv, hq, bk, bv, R=128):
+    """Algorithmic HBM bytes of one sequence's attention for one layer:
+    packed codes + scale/zero of Lq tokens, fp16 residual tokens, q and out."""
+    Lq = packed_len(L, R)
+    per_tok = 16 * (bk + bv) + 32
+    return hkv * (Lq * per_tok + (L - Lq) * 512) + 2 * hq * 128 * 2
+
+
+def source_digest(*names):
+    h = hashlib.sha256()
+    for n in names:
+        h.update((ROOT / "paper_2607_16248_gb300" / "csrc" / n).read_bytes())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic():
+    """DRAM bytes per attention launch from the committed ncu summary, if it
+    was taken on the current attention source."""
+    if not ATTN_PROFILE.exists():
+        return None
+    fields = {}
+    for line in ATTN_PROFILE.read_text().splitlines():
+        if ":" in line and line.strip().startswith("- "):
+            k, v = line.strip()[2:].split(":", 1)
+            fields[k.strip()] = v.strip().strip("`")
+    try:
+        if fields.get("attn_source_sha") != source_digest("attn.cu", "common.cuh"):
+            return None
+        return float(fields["dram_bytes_per_launch_full"])
+    except (KeyError, ValueError):
+        return None
+
+
+def measured_peak_hbm():
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        try:
+            return float(json.loads(p.read_text())["hbm_gbs"]), "measured"
+        except (KeyError, ValueError):
+            pass
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+
+class Clocks:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [r.split(",") for r in self.file.read().splitlines() if r.strip()]
+        self.file.close()
+        os.unlink(self.file.name)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, r[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline leg and --impl reference)
+# ---------------------------------------------------------------------------
+
+
+def cpu_worker(spec_json, budget_s, mode):
+    """Run the oracle on a bounded sample of the workload; print JSON."""
+    import numpy as np
+    from oracle import attention, dgap, quant
+    from paper_2607_16248_gb300 import synth
+
+    spec = json.loads(spec_json)
+    hkv, hq, b = spec["n_kv_heads"], spec["n_q_heads"], spec["bits"]
+    gq = hq // hkv
+    L = spec["context"] if isinstance(spec["context"], int) else spec["context"][1]
+    k, v = synth.kv_heads(spec["seed"], 1, L)
+    qh = quant.quantize_head(k[0].numpy(), v[0].numpy(), b, b, 128)
+    q = synth.queries(spec["seed"], 1, gq)[0].numpy()
+    w = synth.dgap_weights(spec["seed"], K=DGAP_K, hidden=DGAP_HIDDEN)
+    det, cor = synth.split_weights(w)
+    z = synth.logits(spec["seed"], 1, spec["vocab"])[0].numpy().astype(np.float64)
+    unit_bytes = attn_bytes(L, 1, gq, b, b)
+
+    def unit():
+        khat, vhat = quant.dequantize_head(qh)
+        attention.attend_head(q, khat, vhat, 1 / math.sqrt(128))
+
+    t0 = time.perf_counter()
+    unit()
+    t_unit = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    dgap.restore_row(z, DGAP_K, DGAP_TAU, det, cor)
+    t_epi = time.perf_counter() - t0
+    if mode == "baseline":
+        n = max(1, int(budget_s / max(t_unit, 1e-6)))
+        t0 = time.perf_counter()
+        for _ in range(n):
+            unit()
+        t = time.perf_counter() - t0
+        out = {"value": unit_bytes * n / t / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+               "epilogue_ms_per_row": t_epi * 1e3,
+               "sample": f"{n} x one (layer, kv-head) of {hkv * spec['layers']} per step, "
+                         f"context {L}, K{b}V{b}: float64 dequant + softmax attention "
+                         f"(numpy, 1 thread); DGAP restore of one [{spec['vocab']}] row "
+                         f"timed once"}
+    else:  # reference arm: W + K steps of one sampled unit each
+        steps, warmup = spec["_steps"], spec["_warmup"]
+        for _ in range(warmup):
+            unit()
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            unit()
+        t = time.perf_counter() - t0
+        out = {"value": unit_bytes * steps / t / 1e9, "unit": "GB/s", "cores": 1,
+               "ms_per_step": t / steps * 1e3, "kind": "oracle",
+               "sample": f"each step: one (layer, kv-head) of {hkv * spec['layers']}, "
+                         f"context {L}, K{b}V{b}, float64 numpy, 1 thread"}
+    print(json.dumps(out))
+
+
+def run_cpu_worker(spec, budget_s, mode):
+    env = dict(os.environ)
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[var] = "1"
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    cmd = [sys.executable, str(ROOT / "bench.py"), "--cpu-worker", mode,
+           "--workload", "x"]
+    res = subprocess.run(cmd + ["--", json.dumps(spec), str(budget_s)], env=env,
+                         stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True, timeout=900)
+    if res.returncode != 0:
+        raise RuntimeError(f"cpu worker failed: {res.stderr[-2000:]}")
+    return json.loads(res.stdout.strip().splitlines()[-1])
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+
+def dist_setup(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def reduce_max(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+class Step:
+    """Caches, inputs, workspaces and the three captured graphs of a step."""
+
+    def __init__(self, spec, steps_total, device, rank):
+        import torch
+        from paper_2607_16248_gb300 import kvq, synth
+
+        self.spec = spec
+        B, hq, hkv, b = spec["batch"], spec["n_q_heads"], spec["n_kv_heads"], spec["bits"]
+        layers, V, seed = spec["layers"], spec["vocab"], spec["seed"] + 7919 * rank
+        ctx = spec["context"]
+        if isinstance(ctx, (tuple, list)):
+            self.lengths0 = synth.ragged_lengths(seed, B, ctx[0], ctx[1])
+        else:
+            self.lengths0 = [ctx] * B
+        max_len = 32 * math.ceil((max(self.lengths0) + steps_total + 1) / 32)
+        self.cfg = kvq.CacheConfig(batch=B, n_q_heads=hq, n_kv_heads=hkv, bits_k=b, bits_v=b,
+                                   max_len=max_len)
+        self.caches = []
+        for l in range(layers):
+            cache = kvq.QuantKVCache(self.cfg, device)
+            for s, L in enumerate(self.lengths0):
+                k, v = synth.kv_heads(seed * 100003 + l * 1009 + s, hkv, L, device=device)
+                kvq.kvq_pack(cache, k[None], v[None], batch_begin=s)
+                del k, v
+            self.caches.append(cache)
+        torch.cuda.synchronize()
+        g = synth.generator(seed + 1, device)
+        self.q = torch.randn(layers, B, hq, 128, generator=g, device=device).half()
+        self.k_new = torch.randn(layers, B, hkv, 1, 128, generator=g, device=device).half()
+        self.v_new = torch.randn(layers, B, hkv, 1, 128, generator=g, device=device).half()
+        self.out = torch.empty(layers, B, hq, 128, dtype=torch.float16, device=device)
+        self.ws_attn = kvq.attn_workspace(self.cfg, 0, device)
+        self.n_splits = kvq.default_splits(self.cfg)
+        self.dgap = kvq.DGAP(synth.dgap_weights(seed, K=DGAP_K, hidden=DGAP_HIDDEN), K=DGAP_K,
+                             tau=DGAP_TAU, device=device)
+        self.logits0 = synth.logits(seed, B, V, device=device)
+        self.logits = self.logits0.clone()
+        self.ws_dgap = self.dgap.workspace(B, V, device)
+        self.dout = dict(
+            topk_idx=torch.empty(B, DGAP_K, dtype=torch.int32, device=device),
+            topk_val=torch.empty(B, DGAP_K, dtype=torch.float32, device=device),
+            risk=torch.empty(B, dtype=torch.float32, device=device),
+            gate=torch.empty(B, dtype=torch.uint8, device=device),
+            next_token=torch.empty(B, dtype=torch.int32, device=device),
+            features=None)
+        if spec.get("gated_fraction"):
+            self.dgap.tau = self._quantile_tau(spec["gated_fraction"])
+        self._capture(kvq)
+
+    def _quantile_tau(self, frac):
+        """tau at the widest gap of the sorted risks near the (1 - frac)
+        quantile, from an ungated dgap_restore on the step's logits."""
+        import torch
+        z = self.logits0.clone()
+        o = self.dgap.restore(z, tau=2.0, workspace=self.ws_dgap)
+        r = sorted(o["risk"].cpu().tolist())
+        n = len(r)
+        lo, hi = max(0, int((1 - frac - 0.08) * n)), min(n - 1, int((1 - frac + 0.08) * n))
+        if hi <= lo:
+            return r[int((1 - frac) * n)]
+        i = max(range(lo, hi), key=lambda j: r[j + 1] - r[j])
+        torch.cuda.synchronize()
+        return 0.5 * (r[i] + r[i + 1])
+
+    def _capture(self, kvq):
+        import torch
+        L = self.spec["layers"]
+        self.g_pack, self.g_attn, self.g_dgap = (torch.cuda.CUDAGraph() for _ in range(3))
+        with torch.cuda.graph(self.g_pack):
+            for l in range(L):
+                kvq.kvq_pack(self.caches[l], self.k_new[l], self.v_new[l])
+        with torch.cuda.graph(self.g_attn):
+            for l in range(L):
+                kvq.kvq_decode_attn(self.caches[l], self.q[l], out=self.out[l],
+                                    n_splits=self.n_splits, workspace=self.ws_attn)
+        with torch.cuda.graph(self.g_dgap):
+            self.dgap.restore(self.logits, outputs=self.dout, workspace=self.ws_dgap)
+        torch.cuda.synchronize()
+
+    def launches_per_step(self):
+        return 2 * self.spec["layers"] + 1
+
+    def bytes_for_step(self, step_index):
+        """Attention bytes of the step whose pack made sequences L0 + i + 1 long."""
+        s = self.spec
+        per_layer = sum(attn_bytes(L + step_index + 1, s["n_kv_heads"], s["n_q_heads"],
+                                   s["bits"], s["bits"]) for L in self.lengths0)
+        return per_layer * s["layers"]
+
+
+def run_gpu(args, spec):
+    import torch
+
+    world, rank, local = dist_setup(args)
+    device = torch.device("cuda", local if world > 1 else 0)
+    K, W = args.steps, args.warmup
+    e2e_on = not args.no_e2e
+    total_steps = (W + K) * (2 if e2e_on else 1)
+    st = Step(spec, total_steps, device, rank)
+    done = 0  # steps replayed so far (each appends one token per sequence and layer)
+
+    def replay(n, ev=None):
+        nonlocal done
+        for i in range(n):
+            if ev is not None:
+                ev[i][0].record()
+            st.g_pack.replay()
+            if ev is not None:
+                ev[i][1].record()
+            st.g_attn.replay()
+            if ev is not None:
+                ev[i][2].record()
+            st.logits.copy_(st.logits0)
+            if ev is not None:
+                ev[i][3].record()
+            st.g_dgap.replay()
+            if ev is not None:
+                ev[i][4].record()
+        done += n
+
+    replay(W)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    step0 = done
+    clocks = Clocks(torch.cuda.current_device())
+    torch.cuda.synchronize()
+    barrier(world)
+    clocks.start()
+    time.sleep(0.25)  # let the sampler come up before the timed region
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    t_start.record()
+    replay(K, ev)
+    t_end.record()
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    barrier(world)
+    clk = clocks.stop()
+
+    total_ms = reduce_max(t_start.elapsed_time(t_end), world)
+    attn_ms = sum(e[1].elapsed_time(e[2]) for e in ev)
+    pack_ms = sum(e[0].elapsed_time(e[1]) for e in ev)
+    epi_ms = sum(e[3].elapsed_time(e[4]) for e in ev)
+    step_bytes = [st.bytes_for_step(step0 + i) for i in range(K)]
+    bytes_total = sum(step_bytes)
+    value = world * bytes_total / (total_ms * 1e-3) / 1e9
+    launches = K * st.launches_per_step()
+    attn_launches = K * spec["layers"]
+    achieved = bytes_total / (attn_ms * 1e-3) / 1e9
+    peak, peak_kind = measured_peak_hbm()
+
+    e2e = None
+    if e2e_on:
+        e2e = run_e2e(st, W, K, world)
+        done += W + K
+
+    s = spec
+    ctx = s["context"]
+    cfg = {"workload": args.workload, "batch": s["batch"], "n_q_heads": s["n_q_heads"],
+           "n_kv_heads": s["n_kv_heads"], "head_dim": 128, "bits_k": s["bits"],
+           "bits_v": s["bits"], "context": list(ctx) if isinstance(ctx, tuple) else ctx,
+           "context_lengths": st.lengths0 if isinstance(ctx, tuple) else None,
+           "layers": s["layers"], "vocab": s["vocab"], "residual": 128, "group": 32,
+           "dgap_K": DGAP_K, "dgap_hidden": DGAP_HIDDEN, "tau": round(st.dgap.tau, 6),
+           "n_splits": st.n_splits,
+           "l2": f"inputs larger than L2: {step_bytes[0] / 1e6:.0f} MB of packed KV read per "
+                 f"step (distinct cache per layer), L2 129 MB",
+           "step": f"{s['layers']} x (kvq_pack + kvq_decode_attn) + dgap_restore, "
+                   f"3 CUDA graphs", "parallelism": f"replicas x{world}" if world > 1 else "1 GPU"}
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": round(total_ms / K, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded N(0,1) q/k/v with 4 x10 key outlier channels per head; "
+                "N(0,3^2) logits; random-init DGAP MLPs)",
+        "config": cfg,
+        "attn_gbs": round(achieved, 2),
+        "attn_frac_of_peak": round(achieved / peak, 4),
+        "attn_us_per_layer": round(attn_ms / attn_launches * 1e3, 3),
+        "pack_us_per_step": round(pack_ms / K * 1e3, 3),
+        "epilogue_us_per_step": round(epi_ms / K * 1e3, 3),
+        "epilogue_frac_of_step_attn": round(epi_ms / attn_ms, 5),
+        "gated_rows_fraction": float(st.dout["gate"].float().mean().item()),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
+                     "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "peak_source": f"{peak_kind} hbm_gbs (copy)",
+                     "traffic": profiled_traffic(),
+                     "algorithmic_bytes_per_launch": round(bytes_total / attn_launches)},
+        "gpu_launches": launches,
+        "wall_s_timed": round(wall, 4),
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        try:
+            line["cpu_baseline"] = run_cpu_worker(spec, 12.0, "baseline")
+        except Exception as exc:  # reported, not hidden
+            line["cpu_baseline"] = {"error": str(exc)[-300:]}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_e2e(st, W, K, world):
+    """The same metric through the public calls with host buffers: per step,
+    copy the step's inputs from pinned host memory, replay the step, read the
+    step's result (greedy token, window, risk, gate) back and synchronise."""
+    import torch
+    h_q = st.q.cpu().pin_memory()
+    h_k = st.k_new.cpu().pin_memory()
+    h_v = st.v_new.cpu().pin_memory()
+    h_z = st.logits0.cpu().pin_memory()
+    outs = [st.dout[k] for k in ("next_token", "topk_idx", "topk_val", "risk", "gate")]
+    h_out = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    bi = sum(t.numel() * t.element_size() for t in (h_q, h_k, h_v, h_z))
+    bo = sum(t.numel() * t.element_size() for t in h_out)
+
+    def one():
+        st.q.copy_(h_q, non_blocking=True)
+        st.k_new.copy_(h_k, non_blocking=True)
+        st.v_new.copy_(h_v, non_blocking=True)
+        st.g_pack.replay()
+        st.g_attn.replay()
+        st.logits.copy_(h_z, non_blocking=True)
+        st.g_dgap.replay()
+        for h, d in zip(h_out, outs):
+            h.copy_(d, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    for _ in range(W):
+        one()
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(K):
+        one()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = reduce_max(t0.elapsed_time(t1), world)
+    # The e2e steps continue the same decode: lengths kept growing.
+    s = st.spec
+    start = 2 * W + K  # steps replayed before the first timed e2e step
+    total = sum(st.bytes_for_step(start + i) for i in range(K))
+    return {"value": round(world * total / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+            "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo,
+            "ms_per_step": round(ms / K, 5), "n_layers": s["layers"]}
+
+
+# ---------------------------------------------------------------------------
+# Reference arm: the CPU oracle, timed on the host cores
+# ---------------------------------------------------------------------------
+
+
+def run_reference(args, spec):
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return
+    # Each step samples one (layer, kv-head) unit; keep the run to a few minutes.
+    ref_steps, ref_warm = args.steps, args.warmup
+    sp = dict(spec, _steps=ref_steps, _warmup=ref_warm)
+    probe = run_cpu_worker(dict(sp, _steps=1, _warmup=0), 0.0, "reference")
+    per_step_s = probe["ms_per_step"] * 1e-3
+    budget = 150.0
+    if per_step_s * (ref_steps + ref_warm) > budget:
+        ref_steps = max(1, int(budget / per_step_s) - ref_warm)
+        sp["_steps"] = ref_steps
+    res = run_cpu_worker(sp, 0.0, "reference")
+    ctx = spec["context"]
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(res["value"], 4), "unit": "GB/s",
+        "n_gpus": world, "steps": ref_steps, "warmup": ref_warm,
+        "ms_per_step": round(res["ms_per_step"], 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.workload, "batch": spec["batch"],
+                   "n_q_heads": spec["n_q_heads"], "n_kv_heads": spec["n_kv_heads"],
+                   "bits_k": spec["bits"], "bits_v": spec["bits"],
+                   "context": list(ctx) if isinstance(ctx, tuple) else ctx,
+                   "layers": spec["layers"], "vocab": spec["vocab"]},
+        "cpu_baseline": {"value": round(res["value"], 4), "unit": "GB/s", "cores": res["cores"],
+                         "kind": "oracle", "sample": res["sample"]},
+        "e2e": {"value": round(res["value"], 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    if ref_steps != args.steps:
+        line["steps_note"] = f"{args.steps} steps requested; {ref_steps} run to stay within " \
+                             f"{budget:.0f} s of CPU time"
+    print(json.dumps(line))
+
+
+def main():
+    if "--cpu-worker" in sys.argv:
+        i = sys.argv.index("--cpu-worker")
+        mode = sys.argv[i + 1]
+        j = sys.argv.index("--")
+        cpu_worker(sys.argv[j + 1], float(sys.argv[j + 2]), mode)
+        return
+    args = parse()
+    spec = workload_spec(args)
+    if args.impl == "reference":
+        run_reference(args, spec)
+        return
+    from paper_2607_16248_gb300 import build
+    build.build()
+    run_gpu(args, spec)
+
+
+if __name__ == "__main__":
+    main()

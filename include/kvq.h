@@ -1,0 +1,256 @@
+/*
+ * kvq.h — C ABI of the low-bit KV-cache decode step and the DGAP epilogue.
+ *
+ * One decode step of the method of arXiv 2607.16248 ("High-accuracy Low-Bit
+ * KV-Cache Quantization via Local Distribution Restoration"), built for one
+ * GB300 (sm_103a):
+ *
+ *   kvq_pack         append the step's new K/V to a KbVb cache (Sec. 3.1)
+ *   kvq_decode_attn  softmax(q K^T / sqrt(d)) V over that cache (Sec. 1)
+ *   dgap_restore     features, detector, gate, top-K corrector, sparse merge
+ *                    on the step's logits (Sec. 4.1-4.3, Eqs. 2, 6, 11-13)
+ *
+ * Conventions for every call
+ * --------------------------
+ * - Pointers named "device" point to GPU memory owned by the caller; the
+ *   library never allocates, frees or synchronises.  Work is enqueued on the
+ *   CUDA stream passed as `stream` (a cudaStream_t; NULL = legacy default).
+ * - fp16 data is IEEE binary16 passed as uint16_t bit patterns.
+ * - Every call validates its arguments on the host first and returns a
+ *   kvq_status; on failure nothing is enqueued and kvq_last_error() (a
+ *   thread-local string) says why.  KVQ_ERR_CUDA reports a launch error.
+ * - Errors that only the device can see (a sequence pushed past max_len)
+ *   never fault the GPU: the kernel skips the write and sets a bit in the
+ *   cache's flag word (see kvq_cache).
+ */
+#ifndef KVQ_H
+#define KVQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum kvq_status {
+  KVQ_OK = 0,
+  KVQ_ERR_ARG = 1,         /* null pointer, bad scalar argument           */
+  KVQ_ERR_SHAPE = 2,       /* inconsistent sizes                           */
+  KVQ_ERR_UNSUPPORTED = 3, /* bits not in {1,2,4,8}, head_dim != 128 ...   */
+  KVQ_ERR_CAPACITY = 4,    /* workspace or cache too small                 */
+  KVQ_ERR_ALIGN = 5,       /* pointer not 16-byte aligned                  */
+  KVQ_ERR_CUDA = 6         /* kernel launch failed                         */
+} kvq_status;
+
+/* Device-side flag bits (cache flag word). */
+#define KVQ_FLAG_OVERFLOW 1u /* a kvq_pack would have passed max_len */
+
+/*
+ * Cache configuration.  KbVb with b_k = bits_k and b_v = bits_v (Sec. 3.1
+ * names the symmetric settings K1V1..K8V8; Table "ablation_target" of Sec. 5.5
+ * also uses K2V1 and K1V2, so the two widths are independent here).
+ *   head_dim  must be 128;  group must be 32;
+ *   residual  R, fp16 recent-token window, a positive multiple of 32;
+ *   max_len   capacity in tokens per sequence, a positive multiple of 32.
+ * Grouped-query attention: query head i reads kv-head i / (n_q_heads /
+ * n_kv_heads); n_q_heads / n_kv_heads must be an integer in [1, 8].
+ */
+typedef struct kvq_config {
+  int32_t batch;
+  int32_t n_q_heads;
+  int32_t n_kv_heads;
+  int32_t head_dim;
+  int32_t bits_k;
+  int32_t bits_v;
+  int32_t group;
+  int32_t residual;
+  int32_t max_len;
+} kvq_config;
+
+/*
+ * Cache storage (all device pointers, caller-owned; kvq_cache_layout gives
+ * the sizes and kvq_cache_bind carves them out of one buffer).
+ *
+ * Token groups are aligned to absolute position 0.  With L tokens cached,
+ * Lq = 32 * floor(max(L - R, 0) / 32) tokens live in quantized 32-token
+ * blocks and the other L - Lq (R <= L - Lq <= R + 31 once L >= R) stay fp16.
+ *
+ * pages   [batch][n_kv_heads][max_len / 32][page_bytes], one page per 32-token
+ *         block, page_bytes = 512 * (bits_k + bits_v) + 1024:
+ *           K codes  [128 channel][bits_k] uint32   (group = 32 tokens of one channel)
+ *           K meta   [128 channel] {fp16 scale, fp16 zero}
+ *           V codes  [32 token][4 group][bits_v] uint32 (group = 32 channels of one token)
+ *           V meta   [32 token][4 group] {fp16 scale, fp16 zero}
+ *         Element i of a group occupies bits [(i*b) mod 32, +b) of word
+ *         floor(i*b / 32).  Quantizer (b bits, group x_1..x_32):
+ *           zero  = min x_i
+ *           scale = RU16(RU32(RU32(max x_i - min x_i) / (2^b - 1)))
+ *           code  = clamp(rint(RN32(RN32(x - zero) / scale)), 0, 2^b - 1)
+ *         (RU = IEEE round toward +inf, RN = to nearest even; scale 0 gives
+ *         code 0).  Dequantized value: zero + scale * code.
+ * k_resid, v_resid  [batch][n_kv_heads][R + 32][128] fp16 ring; token at
+ *         absolute position p sits in slot p mod (R + 32).
+ * seq_len [batch + 2] int32: [0, batch) token counts L, [batch] the flag word
+ *         (KVQ_FLAG_*), [batch + 1] reserved; followed by `batch` uint32
+ *         tickets used by kvq_pack.  kvq_cache_reset zeroes all of it.
+ */
+typedef struct kvq_cache {
+  void* pages;
+  uint16_t* k_resid;
+  uint16_t* v_resid;
+  int32_t* seq_len;
+} kvq_cache;
+
+/* Thread-local description of the last failure ("" after success). */
+const char* kvq_last_error(void);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int32_t kvq_version(void);
+
+/* Host-only: KVQ_OK when `cfg` is supported. */
+kvq_status kvq_validate_config(const kvq_config* cfg);
+
+/* Host-only: bytes of one 32-token page (0 on an invalid config). */
+size_t kvq_page_bytes(const kvq_config* cfg);
+
+/*
+ * Host-only layout query.  *total_bytes receives the size of one buffer that
+ * holds the whole cache; offsets[0..3] the byte offsets of pages, k_resid,
+ * v_resid and seq_len inside it (each 256-byte aligned).
+ */
+kvq_status kvq_cache_layout(const kvq_config* cfg, size_t* total_bytes,
+                            size_t offsets[4]);
+
+/* Host-only: fill *cache with pointers into `base` (device, >= total_bytes,
+ * 256-byte aligned) following kvq_cache_layout. */
+kvq_status kvq_cache_bind(const kvq_config* cfg, void* base, kvq_cache* cache);
+
+/* Empty every sequence: zero seq_len, the flag word and the tickets. */
+kvq_status kvq_cache_reset(const kvq_config* cfg, const kvq_cache* cache,
+                           void* stream);
+
+/*
+ * kvq_pack — append n_new tokens to sequences [batch_begin, batch_begin +
+ * batch_count) and quantize every 32-token group that leaves the residual
+ * window (Sec. 3.1, KbVb).
+ *   k_new, v_new  device fp16 [batch_count][n_kv_heads][n_new][128], 16-byte
+ *                 aligned; the new tokens of each sequence, oldest first.
+ *   n_new         1 for a decode step; larger for prefill.  Sequences of
+ *                 different lengths are prefilled by calls with
+ *                 batch_count = 1.
+ * Each sequence's current length is read on the device, so the call can be
+ * captured once in a CUDA graph and replayed every step.  A sequence that
+ * would pass max_len is left unchanged and KVQ_FLAG_OVERFLOW is set.
+ * Must be ordered before the kvq_decode_attn of the same step (the query
+ * attends to its own token).
+ */
+kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache,
+                    const uint16_t* k_new, const uint16_t* v_new,
+                    int32_t n_new, int32_t batch_begin, int32_t batch_count,
+                    void* stream);
+
+/*
+ * Split-K workspace for kvq_decode_attn: per (sequence, query head, split)
+ * partial max, sum and fp32 output row, plus one ticket per (sequence,
+ * kv-head).  n_splits = 0 means the library's choice for this config.
+ * Returns 0 on an invalid config.
+ */
+size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits);
+
+/* The split count kvq_decode_attn uses when passed n_splits = 0. */
+int32_t kvq_attn_default_splits(const kvq_config* cfg);
+
+/*
+ * Zero a workspace (attention or DGAP) once after allocating it.  Both
+ * kernels leave their tickets at zero when they finish, so one
+ * initialisation serves any number of calls.
+ */
+kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * kvq_decode_attn — one decode step of grouped-query attention
+ *   out[b, i] = softmax(q[b, i] . K_hat[b, g(i)]^T * softmax_scale) V_hat[b, g(i)]
+ * over all L = seq_len[b] cached tokens (Sec. 1 gives softmax(QK^T/sqrt(d_k))V;
+ * g(i) = i / (n_q_heads / n_kv_heads)).  K_hat, V_hat are the dequantized
+ * blocks plus the fp16 residual window.
+ *   q, out         device fp16 [batch][n_q_heads][128], 16-byte aligned.
+ *   softmax_scale  0 selects 1/sqrt(128).
+ *   n_splits       0 = kvq_attn_default_splits(cfg); else 1..1024.
+ *   workspace      device, >= kvq_attn_workspace_bytes(cfg, n_splits), zeroed
+ *                  once by kvq_workspace_init.
+ * A sequence with L = 0 gets a zero output.  Calls that share a workspace
+ * must not overlap on the GPU.
+ */
+kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache,
+                           const uint16_t* q, uint16_t* out,
+                           float softmax_scale, int32_t n_splits,
+                           void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * DGAP parameters (Sec. 4.2 detector, Sec. 4.3 corrector).  Weights are
+ * device fp32, row-major [out][in]; H = hidden.
+ *   detector  f = w2 . relu(W1 phi + b1) + b2, r = sigmoid(f)   (Eq. 6)
+ *             det_w1 [H][8], det_b1 [H], det_w2 [H], det_b2 [1]
+ *   corrector Delta = W2 relu(W1 [xi | phi] + b1) + b2          (Eq. 12)
+ *             cor_w1 [H][5K + 8], cor_b1 [H], cor_w2 [K][H], cor_b2 [K]
+ *   K    recovery window size K_b, 2 <= K <= 64, K < vocab (Eqs. 2, 11)
+ *   H    1 <= hidden <= 1024
+ *   tau  risk threshold; the corrector runs when r > tau (Eq. 13); the
+ *        paper's calibrated value is 0.60 (Sec. 5.5).
+ * phi (8 features, in order): entropy of softmax(z); top-K mass; top-1
+ * probability; z_(0) - z_(1); (z_(0) - z_(K-1)) / (K - 1); least adjacent gap
+ * in the window; population std of the window logits; entropy of the
+ * window's renormalised probabilities.  xi (5 per window rank k):
+ * z_(k) - z_(0); log p_(k); k / (K - 1); z_(k-1) - z_(k) (0 at k = 0);
+ * z_(k) - z_(k+1) (z_(K) is the (K+1)-th logit).
+ */
+typedef struct dgap_params {
+  int32_t K;
+  int32_t hidden;
+  float tau;
+  const float* det_w1;
+  const float* det_b1;
+  const float* det_w2;
+  const float* det_b2;
+  const float* cor_w1;
+  const float* cor_b1;
+  const float* cor_w2;
+  const float* cor_b2;
+} dgap_params;
+
+/* Workspace bytes for dgap_restore on [batch][vocab] logits (0 if invalid). */
+size_t dgap_workspace_bytes(int32_t batch, int32_t vocab, const dgap_params* p);
+
+/*
+ * dgap_restore — the DGAP epilogue on one decode step's logits (Sec. 4.1-4.3).
+ * For each row z (finite fp32):
+ *   S = TopK(z, K): value descending, lowest index first on ties (Eqs. 2, 11);
+ *   phi = Phi(z); r = sigmoid(f_theta(phi)) (Eq. 6);
+ *   if r > tau: Delta = g_psi(xi_S, phi) and z[S_k] += Delta_k in place
+ *   (Eq. 13); every other logit, and every logit of an ungated row, is left
+ *   bit-identical.
+ *   logits      device fp32 [batch][vocab], updated in place, 16-byte aligned.
+ *   topk_idx    device int32 [batch][K]: S in rank order.
+ *   topk_val    device fp32 [batch][K]: merged values z~ at S.
+ *   risk        device fp32 [batch]: r.
+ *   gate        device uint8 [batch]: 1 when the corrector ran.
+ *   next_token  device int32 [batch] or NULL: argmax of the merged row
+ *               (lowest index on ties), i.e. greedy token selection.
+ *   features    device fp32 [batch][8] or NULL: phi.
+ *   workspace   device, >= dgap_workspace_bytes(...), zeroed once by
+ *               kvq_workspace_init; calls sharing it must not overlap.
+ * The gate is decided as f > log(tau / (1 - tau)) (tau >= 1: never; tau <= 0:
+ * always), which equals r > tau.
+ */
+kvq_status dgap_restore(const dgap_params* params, float* logits,
+                        int32_t batch, int32_t vocab, int32_t* topk_idx,
+                        float* topk_val, float* risk, uint8_t* gate,
+                        int32_t* next_token, float* features, void* workspace,
+                        size_t ws_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVQ_H */

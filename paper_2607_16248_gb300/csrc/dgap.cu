@@ -1,0 +1,413 @@
+// dgap_restore: the DGAP local-distribution-restoration epilogue
+// (Sec. 4.1-4.3 of the paper) on one decode step's logits [batch][vocab].
+//
+// One launch, grid (n_chunks, batch), 256 threads.  Each CTA scans a 4096-logit
+// chunk of one row once: running max m, S1 = sum e^{z-m}, S2 = sum (z-m) e^{z-m}
+// and the chunk's K+1 best (value descending, index ascending) candidates.
+// The last CTA of a row to finish (atomic ticket, no waiting) merges the
+// chunks, forms the window S = TopK(z, K) and z_(K), the features phi,
+// runs the detector r = sigmoid(f) (Eq. 6), and when f > logit(tau) the
+// candidate features xi, the corrector Delta = g(xi, phi) (Eq. 12) and the
+// sparse merge z[S_k] += Delta_k in place (Eq. 13).  Non-selected logits and
+// ungated rows are never written.
+//
+// Candidates are ranked by an order-preserving uint32 key of the float
+// (-0 folded onto +0) and then by the lower index.
+
+#include <limits.h>
+
+#include "common.cuh"
+
+namespace kvq {
+namespace {
+
+constexpr int kT = 256;
+constexpr int kWarpsD = kT / 32;
+constexpr int kPer = 16;
+constexpr int kChunk = kT * kPer;
+constexpr int kMaxChunks = kT;  // one candidate list per finalize thread
+constexpr int kMaxIn = 5 * kMaxK + 8;  // corrector input width
+
+struct DWs {
+  float4* stats;   // [B][n_chunks] (m, S1, S2, -)
+  uint2* cand;     // [B][n_chunks][K+1] (key, index)
+  unsigned* tk;    // [B]
+};
+
+__host__ __device__ inline size_t a256(size_t x) { return (x + 255) / 256 * 256; }
+
+__host__ __device__ inline DWs carve(void* base, int batch, int n_chunks, int K) {
+  DWs w;
+  char* p = static_cast<char*>(base);
+  w.stats = reinterpret_cast<float4*>(p);
+  p += a256((size_t)batch * n_chunks * sizeof(float4));
+  w.cand = reinterpret_cast<uint2*>(p);
+  p += a256((size_t)batch * n_chunks * (K + 1) * sizeof(uint2));
+  w.tk = reinterpret_cast<unsigned*>(p);
+  return w;
+}
+
+__device__ __forceinline__ uint32_t order_key(float x) {
+  uint32_t u = __float_as_uint(x);
+  if ((u << 1) == 0u) u = 0u;  // -0 ranks with +0
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float key_value(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+// (ka, ia) ranks before (kb, ib)?
+__device__ __forceinline__ bool before(uint32_t ka, int ia, uint32_t kb, int ib) {
+  return ka > kb || (ka == kb && ia < ib);
+}
+
+__device__ __forceinline__ float wsum(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float wmax(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Block-wide reductions over 256 threads (all threads get the result).
+__device__ float block_sum(float v, float* red) {
+  v = wsum(v);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float r = l < kWarpsD ? red[l] : 0.0f;
+  return wsum(r);
+}
+__device__ float block_max(float v, float* red) {
+  v = wmax(v);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float r = l < kWarpsD ? red[l] : -INFINITY;
+  return wmax(r);
+}
+
+// Merge up to 32 sorted lists (one per lane, `len` entries read by get(h))
+// into the first n entries of their common order; lane 0 writes ok/oi.
+template <typename Get>
+__device__ void warp_merge(int len, const Get& get, int n, uint32_t* ok, int* oi) {
+  const int lane = threadIdx.x & 31;
+  int head = 0;
+  uint32_t hk = 0u;
+  int hi = INT_MAX;
+  if (len > 0) get(0, hk, hi);
+  for (int r = 0; r < n; ++r) {
+    const uint32_t mk = __reduce_max_sync(0xffffffffu, hk);
+    const uint32_t mi = __reduce_min_sync(0xffffffffu, hk == mk ? (uint32_t)hi : 0xffffffffu);
+    if (lane == 0) {
+      ok[r] = mk;
+      oi[r] = (int)mi;
+    }
+    if (hk == mk && (uint32_t)hi == mi) {
+      ++head;
+      if (head < len) {
+        get(head, hk, hi);
+      } else {
+        hk = 0u;
+        hi = INT_MAX;
+      }
+    }
+  }
+  __syncwarp();
+}
+
+// Sort kPer (key, index) pairs held in registers, best first (bitonic).
+__device__ __forceinline__ void sort_desc(uint32_t (&k)[kPer], int (&ix)[kPer]) {
+#pragma unroll
+  for (int size = 2; size <= kPer; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        const int j = i ^ stride;
+        if (j > i) {
+          const bool first_best = (i & size) == 0;
+          const bool swap = first_best ? before(k[j], ix[j], k[i], ix[i])
+                                       : before(k[i], ix[i], k[j], ix[j]);
+          if (swap) {
+            const uint32_t tk = k[i];
+            k[i] = k[j];
+            k[j] = tk;
+            const int ti = ix[i];
+            ix[i] = ix[j];
+            ix[j] = ti;
+          }
+        }
+      }
+    }
+  }
+}
+
+struct Smem {
+  uint32_t sk[kPer][kT];
+  int si[kPer][kT];
+  uint32_t wk[kWarpsD][kMaxK + 1];
+  int wi[kWarpsD][kMaxK + 1];
+  uint32_t fk[kMaxK + 1];
+  int fi[kMaxK + 1];
+  float zt[kMaxK];
+  float x[kMaxIn];
+  float hb[kMaxHidden];
+  float phi[8];
+  float red[32];
+  float f;
+  int last;
+};
+
+__device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* logits, int row,
+                             int32_t* topk_idx, float* topk_val, float* risk, uint8_t* gate,
+                             int32_t* next_token, float* features, const DWs& ws, Smem& sm) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int K = d.K, K1 = d.K + 1, nc = d.n_chunks;
+  const float4* st = ws.stats + (size_t)row * nc;
+
+  // Merge the chunk statistics.
+  float mloc = -INFINITY;
+  for (int c = tid; c < nc; c += kT) mloc = fmaxf(mloc, __ldcg(&st[c].x));
+  const float M = block_max(mloc, sm.red);
+  float s1 = 0.0f, s2 = 0.0f;
+  for (int c = tid; c < nc; c += kT) {
+    const float4 v = __ldcg(&st[c]);
+    if (v.y > 0.0f) {
+      const float e = expf(v.x - M);
+      s1 += v.y * e;
+      s2 += (v.z + (v.x - M) * v.y) * e;
+    }
+  }
+  const float S1 = block_sum(s1, sm.red);
+  const float S2 = block_sum(s2, sm.red);
+
+  // Merge the chunk candidate lists: warp w takes lists w*32 + lane, then
+  // warp 0 merges the eight warp results (n_chunks <= 256).
+  const uint2* cand = ws.cand + (size_t)row * nc * K1;
+  const int li = warp * 32 + lane;
+  warp_merge(li < nc ? K1 : 0, [&](int h, uint32_t& k, int& i) {
+    const uint2 v = __ldcg(&cand[(size_t)li * K1 + h]);
+    k = v.x;
+    i = (int)v.y;
+  }, K1, sm.wk[warp], sm.wi[warp]);
+  __syncthreads();
+  if (warp == 0)
+    warp_merge(lane < kWarpsD ? K1 : 0, [&](int h, uint32_t& k, int& i) {
+      k = sm.wk[lane][h];
+      i = sm.wi[lane][h];
+    }, K1, sm.fk, sm.fi);
+  __syncthreads();
+
+  // Features phi (Sec. 4.2).
+  if (tid == 0) {
+    const float z0 = key_value(sm.fk[0]);
+    float mass_e = 0.0f, wsum_e = 0.0f, mean = 0.0f, min_gap = INFINITY;
+    for (int k = 0; k < K; ++k) {
+      const float zk = key_value(sm.fk[k]);
+      const float e = expf(zk - M);
+      mass_e += e;
+      wsum_e += e * (zk - M);
+      mean += zk;
+      if (k + 1 < K) min_gap = fminf(min_gap, zk - key_value(sm.fk[k + 1]));
+    }
+    mean /= (float)K;
+    float var = 0.0f;
+    for (int k = 0; k < K; ++k) {
+      const float dz = key_value(sm.fk[k]) - mean;
+      var += dz * dz;
+    }
+    var /= (float)K;
+    sm.phi[0] = logf(S1) - S2 / S1;
+    sm.phi[1] = mass_e / S1;
+    sm.phi[2] = expf(z0 - M) / S1;
+    sm.phi[3] = z0 - key_value(sm.fk[1]);
+    sm.phi[4] = (z0 - key_value(sm.fk[K - 1])) / (float)(K - 1);
+    sm.phi[5] = min_gap;
+    sm.phi[6] = sqrtf(var);
+    sm.phi[7] = logf(mass_e) - wsum_e / mass_e;
+  }
+  __syncthreads();
+
+  // Detector f = w2 . relu(W1 phi + b1) + b2 (Eq. 6).
+  float part = 0.0f;
+  for (int j = tid; j < d.hidden; j += kT) {
+    float a = p.det_b1[j];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a = fmaf(p.det_w1[j * 8 + i], sm.phi[i], a);
+    part = fmaf(p.det_w2[j], fmaxf(a, 0.0f), part);
+  }
+  const float f = block_sum(part, sm.red) + p.det_b2[0];
+  const bool gated = f > d.logit_tau;
+
+  // Window values before the merge.
+  for (int k = tid; k < K; k += kT) sm.zt[k] = key_value(sm.fk[k]);
+  __syncthreads();
+
+  if (gated) {
+    // Candidate features xi (Sec. 4.3), rank-major, then phi.
+    const int nin = 5 * K + 8;
+    const float lse = M + logf(S1);
+    const float z0 = sm.zt[0];
+    for (int k = tid; k < K; k += kT) {
+      const float zk = sm.zt[k];
+      const float znext = k + 1 < K ? sm.zt[k + 1] : key_value(sm.fk[K]);
+      sm.x[5 * k + 0] = zk - z0;
+      sm.x[5 * k + 1] = zk - lse;
+      sm.x[5 * k + 2] = (float)k / (float)(K - 1);
+      sm.x[5 * k + 3] = k == 0 ? 0.0f : sm.zt[k - 1] - zk;
+      sm.x[5 * k + 4] = zk - znext;
+    }
+    if (tid < 8) sm.x[5 * K + tid] = sm.phi[tid];
+    __syncthreads();
+    // Hidden layer: one warp per hidden unit, lanes over the inputs.
+    for (int j = warp; j < d.hidden; j += kWarpsD) {
+      const float* wrow = p.cor_w1 + (size_t)j * nin;
+      float a = 0.0f;
+      for (int i = lane; i < nin; i += 32) a = fmaf(wrow[i], sm.x[i], a);
+      a = wsum(a);
+      if (lane == 0) sm.hb[j] = fmaxf(a + p.cor_b1[j], 0.0f);
+    }
+    __syncthreads();
+    // Output layer Delta_k, then the sparse merge (Eq. 13).
+    for (int k = warp; k < K; k += kWarpsD) {
+      const float* wrow = p.cor_w2 + (size_t)k * d.hidden;
+      float a = 0.0f;
+      for (int j = lane; j < d.hidden; j += 32) a = fmaf(wrow[j], sm.hb[j], a);
+      a = wsum(a);
+      if (lane == 0) {
+        const float zt = sm.zt[k] + (a + p.cor_b2[k]);
+        sm.zt[k] = zt;
+        logits[(size_t)row * d.vocab + sm.fi[k]] = zt;
+      }
+    }
+    __syncthreads();
+  }
+
+  for (int k = tid; k < K; k += kT) {
+    topk_idx[(size_t)row * K + k] = sm.fi[k];
+    topk_val[(size_t)row * K + k] = sm.zt[k];
+  }
+  if (features && tid < 8) features[(size_t)row * 8 + tid] = sm.phi[tid];
+  if (tid == 0) {
+    risk[row] = 1.0f / (1.0f + expf(-f));
+    gate[row] = gated ? 1 : 0;
+    if (next_token) {
+      float bv = key_value(sm.fk[K]);
+      int bi = sm.fi[K];
+      for (int k = 0; k < K; ++k)
+        if (sm.zt[k] > bv || (sm.zt[k] == bv && sm.fi[k] < bi)) {
+          bv = sm.zt[k];
+          bi = sm.fi[k];
+        }
+      next_token[row] = bi;
+    }
+    ws.tk[row] = 0u;
+  }
+}
+
+__global__ void __launch_bounds__(kT)
+    dgap_kernel(DgapDims d, dgap_params p, float* __restrict__ logits, int32_t* topk_idx,
+                float* topk_val, float* risk, uint8_t* gate, int32_t* next_token,
+                float* features, DWs ws) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int chunk = blockIdx.x, row = blockIdx.y, K1 = d.K + 1;
+  const float* z = logits + (size_t)row * d.vocab;
+  const int base = chunk * kChunk;
+
+  float v[kPer];
+  uint32_t k[kPer];
+  int ix[kPer];
+  float lm = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    const int e = base + i * kT + tid;
+    if (e < d.vocab) {
+      v[i] = z[e];
+      k[i] = order_key(v[i]);
+      ix[i] = e;
+      lm = fmaxf(lm, v[i]);
+    } else {
+      v[i] = -INFINITY;
+      k[i] = 0u;
+      ix[i] = INT_MAX;
+    }
+  }
+  const float m = block_max(lm, sm.red);
+  float s1 = 0.0f, s2 = 0.0f;
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    if (ix[i] != INT_MAX) {
+      const float dz = v[i] - m;
+      const float e = expf(dz);
+      s1 += e;
+      s2 = fmaf(dz, e, s2);
+    }
+  }
+  s1 = block_sum(s1, sm.red);
+  s2 = block_sum(s2, sm.red);
+
+  sort_desc(k, ix);
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    sm.sk[i][tid] = k[i];
+    sm.si[i][tid] = ix[i];
+  }
+  __syncwarp();
+  warp_merge(kPer, [&](int h, uint32_t& kk, int& ii) {
+    kk = sm.sk[h][tid];
+    ii = sm.si[h][tid];
+  }, K1, sm.wk[warp], sm.wi[warp]);
+  __syncthreads();
+  uint2* out = ws.cand + ((size_t)row * d.n_chunks + chunk) * K1;
+  if (warp == 0) {
+    warp_merge(lane < kWarpsD ? K1 : 0, [&](int h, uint32_t& kk, int& ii) {
+      kk = sm.wk[lane][h];
+      ii = sm.wi[lane][h];
+    }, K1, sm.fk, sm.fi);
+    for (int r = lane; r < K1; r += 32) out[r] = make_uint2(sm.fk[r], (uint32_t)sm.fi[r]);
+    if (lane == 0) ws.stats[(size_t)row * d.n_chunks + chunk] = make_float4(m, s1, s2, 0.0f);
+  }
+
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    const unsigned t = atomicAdd(&ws.tk[row], 1u);
+    sm.last = (t == (unsigned)d.n_chunks - 1);
+  }
+  __syncthreads();
+  if (!sm.last) return;
+  __threadfence();
+  finalize_row(d, p, logits, row, topk_idx, topk_val, risk, gate, next_token, features, ws, sm);
+}
+
+}  // namespace
+
+int dgap_chunks(int vocab) { return (vocab + kChunk - 1) / kChunk; }
+int dgap_max_chunks() { return kMaxChunks; }
+
+size_t dgap_workspace_bytes_impl(int batch, int vocab, int K) {
+  const int nc = dgap_chunks(vocab);
+  return a256((size_t)batch * nc * sizeof(float4)) +
+         a256((size_t)batch * nc * (K + 1) * sizeof(uint2)) + a256((size_t)batch * 4);
+}
+
+cudaError_t launch_dgap(const DgapDims& d, const dgap_params& p, float* logits, int32_t* topk_idx,
+                        float* topk_val, float* risk, uint8_t* gate, int32_t* next_token,
+                        float* features, void* workspace, cudaStream_t stream) {
+  const DWs ws = carve(workspace, d.batch, d.n_chunks, d.K);
+  const size_t smem = sizeof(Smem);
+  static_assert(sizeof(Smem) <= 48 * 1024, "DGAP shared memory must fit the default limit");
+  dim3 grid(d.n_chunks, d.batch);
+  dgap_kernel<<<grid, kT, smem, stream>>>(d, p, logits, topk_idx, topk_val, risk, gate, next_token,
+                                          features, ws);
+  return cudaGetLastError();
+}
+
+}  // namespace kvq

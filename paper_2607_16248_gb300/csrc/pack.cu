@@ -1,0 +1,242 @@
+// kvq_pack: append new K/V tokens to the fp16 residual window and quantize
+// every 32-token group that leaves it (KbVb, Sec. 3.1 of the paper).
+//
+// Quantizer of one 32-element group x (b bits, levels = 2^b - 1), each step a
+// single IEEE float32 operation with the stated rounding:
+//   zero  = min x                                   (exact, fp16)
+//   scale = RU16(RU32(RU32(max x - min x) / levels)) (stored fp16)
+//   code  = clamp(rint(RN32(RN32(x - zero) / scale)), 0, levels); 0 if scale == 0
+// Codes of a group fill b little-endian uint32 words, element i at bits
+// [(i*b) % 32, +b) of word (i*b) / 32.  Keys group 32 tokens of one channel,
+// values 32 channels of one token.
+
+#include "common.cuh"
+
+namespace kvq {
+namespace {
+
+constexpr int kPackThreads = 256;
+constexpr int kRowPad = 136;  // halves per smem row (128 + 8) to spread banks
+
+struct Tile {
+  __half k[kGroup][kRowPad];
+  __half v[kGroup][kRowPad];
+};
+
+// Quantize the 32 values x[] and return the packed words + (scale, zero).
+template <int B>
+__device__ __forceinline__ void quantize_group(const float (&x)[kGroup], uint32_t (&w)[B],
+                                               __half2& meta) {
+  constexpr float kLevels = float((1 << B) - 1);
+  float lo = x[0], hi = x[0];
+#pragma unroll
+  for (int i = 1; i < kGroup; ++i) {
+    lo = fminf(lo, x[i]);
+    hi = fmaxf(hi, x[i]);
+  }
+  const __half s_h = __float2half_ru(__fdiv_ru(__fsub_ru(hi, lo), kLevels));
+  const float s = __half2float(s_h);
+#pragma unroll
+  for (int j = 0; j < B; ++j) w[j] = 0u;
+#pragma unroll
+  for (int i = 0; i < kGroup; ++i) {
+    uint32_t c = 0u;
+    if (s > 0.0f) {
+      float t = rintf(__fdiv_rn(__fsub_rn(x[i], lo), s));
+      t = fminf(fmaxf(t, 0.0f), kLevels);
+      c = (uint32_t)t;
+    }
+    w[(i * B) / 32] |= c << ((i * B) % 32);
+  }
+  meta = __halves2half2(s_h, __float2half_rn(lo));  // lo is an fp16 value: exact
+}
+
+template <int B>
+__device__ __forceinline__ void store_words(uint32_t* dst, const uint32_t (&w)[B]) {
+#pragma unroll
+  for (int j = 0; j < B; ++j) dst[j] = w[j];
+}
+
+template <int B>
+__device__ __forceinline__ void quantize_key_channel(const Tile& t, int c, char* page, int bits_k) {
+  float x[kGroup];
+#pragma unroll
+  for (int i = 0; i < kGroup; ++i) x[i] = __half2float(t.k[i][c]);
+  uint32_t w[B];
+  __half2 meta;
+  quantize_group<B>(x, w, meta);
+  store_words<B>(reinterpret_cast<uint32_t*>(page) + c * B, w);
+  reinterpret_cast<__half2*>(page + page_off_kmeta(bits_k))[c] = meta;
+}
+
+template <int B>
+__device__ __forceinline__ void quantize_value_group(const Tile& t, int pair, char* page,
+                                                     int bits_k, int bits_v) {
+  const int tok = pair >> 2, grp = pair & 3;
+  float x[kGroup];
+#pragma unroll
+  for (int i = 0; i < kGroup; ++i) x[i] = __half2float(t.v[tok][grp * kGroup + i]);
+  uint32_t w[B];
+  __half2 meta;
+  quantize_group<B>(x, w, meta);
+  store_words<B>(reinterpret_cast<uint32_t*>(page + page_off_vcodes(bits_k)) + pair * B, w);
+  reinterpret_cast<__half2*>(page + page_off_vmeta(bits_k, bits_v))[pair] = meta;
+}
+
+// 256 threads: 0..127 quantize one key channel each, 128..255 one
+// (token, 32-channel group) value group each.
+__device__ void quantize_tile(const Tile& t, char* page, int bits_k, int bits_v) {
+  const int tid = threadIdx.x;
+  if (tid < kHeadDim) {
+    switch (bits_k) {
+      case 1: quantize_key_channel<1>(t, tid, page, bits_k); break;
+      case 2: quantize_key_channel<2>(t, tid, page, bits_k); break;
+      case 4: quantize_key_channel<4>(t, tid, page, bits_k); break;
+      default: quantize_key_channel<8>(t, tid, page, bits_k); break;
+    }
+  } else {
+    const int pair = tid - kHeadDim;
+    switch (bits_v) {
+      case 1: quantize_value_group<1>(t, pair, page, bits_k, bits_v); break;
+      case 2: quantize_value_group<2>(t, pair, page, bits_k, bits_v); break;
+      case 4: quantize_value_group<4>(t, pair, page, bits_k, bits_v); break;
+      default: quantize_value_group<8>(t, pair, page, bits_k, bits_v); break;
+    }
+  }
+}
+
+__device__ __forceinline__ char* page_ptr(const Dims& d, void* pages, int b, int h, int j) {
+  return static_cast<char*>(pages) + (((long long)b * d.hkv + h) * d.max_blocks + j) * d.page_bytes;
+}
+
+// Source row (128 fp16) of absolute token p of (b, h): the ring for p < L0,
+// the caller's new tokens otherwise.
+struct RowSrc {
+  const __half* ring_k;
+  const __half* ring_v;
+  const __half* new_k;
+  const __half* new_v;
+  int L0, ring;
+  __device__ __forceinline__ const uint4* k(int p) const {
+    const __half* r = p < L0 ? ring_k + (long long)(p % ring) * kHeadDim
+                             : new_k + (long long)(p - L0) * kHeadDim;
+    return reinterpret_cast<const uint4*>(r);
+  }
+  __device__ __forceinline__ const uint4* v(int p) const {
+    const __half* r = p < L0 ? ring_v + (long long)(p % ring) * kHeadDim
+                             : new_v + (long long)(p - L0) * kHeadDim;
+    return reinterpret_cast<const uint4*>(r);
+  }
+};
+
+// Stage block j's 32 tokens into the smem tile (16 x 16-byte pieces per row).
+__device__ void load_tile(Tile& t, const RowSrc& src, int j) {
+  for (int e = threadIdx.x; e < kGroup * 16; e += kPackThreads) {
+    const int row = e >> 4, piece = e & 15;
+    const int p = j * kGroup + row;
+    *reinterpret_cast<uint4*>(&t.k[row][piece * 8]) = src.k(p)[piece];
+    *reinterpret_cast<uint4*>(&t.v[row][piece * 8]) = src.v(p)[piece];
+  }
+}
+
+__device__ __forceinline__ RowSrc make_src(const Dims& d, const kvq_cache& c, const __half* k_new,
+                                           const __half* v_new, int n_new, int b, int bi, int h,
+                                           int L0) {
+  RowSrc s;
+  const long long bh = (long long)b * d.hkv + h;
+  s.ring_k = reinterpret_cast<const __half*>(c.k_resid) + bh * d.ring * kHeadDim;
+  s.ring_v = reinterpret_cast<const __half*>(c.v_resid) + bh * d.ring * kHeadDim;
+  const long long nh = ((long long)bi * d.hkv + h) * n_new;
+  s.new_k = k_new + nh * kHeadDim;
+  s.new_v = v_new + nh * kHeadDim;
+  s.L0 = L0;
+  s.ring = d.ring;
+  return s;
+}
+
+// Blocks made only of new tokens (prefill).  grid (x, hkv, batch_count).
+__global__ void __launch_bounds__(kPackThreads)
+    pack_input_blocks_kernel(Dims d, kvq_cache c, const __half* __restrict__ k_new,
+                             const __half* __restrict__ v_new, int n_new, int batch_begin) {
+  __shared__ Tile tile;
+  const int bi = blockIdx.z, b = batch_begin + bi, h = blockIdx.y;
+  const int L0 = c.seq_len[b];
+  const int L1 = L0 + n_new;
+  if (L1 > d.max_len) return;  // the append kernel reports the overflow
+  const int first = max(packed_len(L0, d.residual), ((L0 + kGroup - 1) / kGroup) * kGroup) / kGroup;
+  const int j = first + blockIdx.x;
+  if (j >= packed_len(L1, d.residual) / kGroup) return;
+  const RowSrc src = make_src(d, c, k_new, v_new, n_new, b, bi, h, L0);
+  load_tile(tile, src, j);
+  __syncthreads();
+  quantize_tile(tile, page_ptr(d, c.pages, b, h, j), d.bits_k, d.bits_v);
+}
+
+// Blocks that touch the ring, the ring append, and the length update.
+// grid (hkv, batch_count); the last CTA of a sequence (ticket) publishes L1.
+__global__ void __launch_bounds__(kPackThreads)
+    pack_append_kernel(Dims d, kvq_cache c, const __half* __restrict__ k_new,
+                       const __half* __restrict__ v_new, int n_new, int batch_begin) {
+  __shared__ Tile tile;
+  const int bi = blockIdx.y, b = batch_begin + bi, h = blockIdx.x;
+  const int L0 = c.seq_len[b];
+  const int L1 = L0 + n_new;
+  if (L1 > d.max_len) {
+    if (threadIdx.x == 0 && h == 0) atomicOr(reinterpret_cast<unsigned*>(c.seq_len) + d.batch,
+                                             KVQ_FLAG_OVERFLOW);
+    return;
+  }
+  const int Lq0 = packed_len(L0, d.residual), Lq1 = packed_len(L1, d.residual);
+  const RowSrc src = make_src(d, c, k_new, v_new, n_new, b, bi, h, L0);
+
+  // 1. Groups leaving the window that start below L0 (they read the ring).
+  const int j_end = min(Lq1, ((L0 + kGroup - 1) / kGroup) * kGroup) / kGroup;
+  for (int j = Lq0 / kGroup; j < j_end; ++j) {
+    load_tile(tile, src, j);
+    __syncthreads();
+    quantize_tile(tile, page_ptr(d, c.pages, b, h, j), d.bits_k, d.bits_v);
+    __syncthreads();
+  }
+
+  // 2. New tokens that stay fp16 go to their ring slots (after every ring read).
+  const long long bh = (long long)b * d.hkv + h;
+  __half* ring_k = reinterpret_cast<__half*>(c.k_resid) + bh * d.ring * kHeadDim;
+  __half* ring_v = reinterpret_cast<__half*>(c.v_resid) + bh * d.ring * kHeadDim;
+  const int p0 = max(Lq1, L0);
+  for (int e = threadIdx.x; e < (L1 - p0) * 16; e += kPackThreads) {
+    const int p = p0 + (e >> 4), piece = e & 15;
+    reinterpret_cast<uint4*>(ring_k + (long long)(p % d.ring) * kHeadDim)[piece] = src.k(p)[piece];
+    reinterpret_cast<uint4*>(ring_v + (long long)(p % d.ring) * kHeadDim)[piece] = src.v(p)[piece];
+  }
+
+  // 3. Publish the new length once every kv-head of the sequence has read L0.
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned* tickets = reinterpret_cast<unsigned*>(c.seq_len) + d.batch + 2;
+    __threadfence();
+    const unsigned t = atomicAdd(&tickets[b], 1u);
+    if (t == (unsigned)d.hkv - 1) {
+      c.seq_len[b] = L1;
+      tickets[b] = 0u;
+      __threadfence();
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_pack(const Dims& d, const kvq_cache& cache, const __half* k_new,
+                        const __half* v_new, int n_new, int batch_begin, int batch_count,
+                        cudaStream_t stream) {
+  if (n_new > kGroup) {
+    dim3 grid(n_new / kGroup + 1, d.hkv, batch_count);
+    pack_input_blocks_kernel<<<grid, kPackThreads, 0, stream>>>(d, cache, k_new, v_new, n_new,
+                                                                 batch_begin);
+  }
+  dim3 grid2(d.hkv, batch_count);
+  pack_append_kernel<<<grid2, kPackThreads, 0, stream>>>(d, cache, k_new, v_new, n_new,
+                                                         batch_begin);
+  return cudaGetLastError();
+}
+
+}  // namespace kvq

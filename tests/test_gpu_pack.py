@@ -1,0 +1,109 @@
+"""kvq_pack (CUDA, through the C ABI) against the oracle quantizer: packed
+codes, scales, zeros and the fp16 residual window must be bit-identical."""
+
+import numpy as np
+import pytest
+import torch
+
+import _util
+from oracle import quant
+from paper_2607_16248_gb300 import kvq, synth
+
+pytestmark = pytest.mark.gpu
+
+BIT_PAIRS = [(1, 1), (2, 2), (4, 4), (8, 8), (2, 1), (1, 2), (8, 1)]
+
+
+@pytest.mark.parametrize("bk,bv", BIT_PAIRS)
+def test_prefill_ragged_batch(kvq_lib, bk, bv):
+    lengths = [1, 31, 128, 159, 160, 161, 193, 1000, 4096, 0]
+    cfg = kvq.CacheConfig(batch=len(lengths), n_q_heads=8, n_kv_heads=2, bits_k=bk, bits_v=bv,
+                          max_len=4352)
+    cache, kv = _util.make_cache(cfg, lengths, seed=bk * 10 + bv)
+    assert cache.seq_lens().cpu().tolist() == lengths
+    assert cache.flags() == 0
+    for b, L in enumerate(lengths):
+        k, v = kv[b]
+        for h in range(cfg.n_kv_heads):
+            want = quant.quantize_head(k[h].numpy(), v[h].numpy(), bk, bv, cfg.residual)
+            _util.assert_head_equal(_util.head_arrays(cache, b, h, L), want)
+
+
+@pytest.mark.parametrize("bk,bv", [(1, 1), (2, 2), (4, 8)])
+def test_decode_appends_cross_flush_boundaries(kvq_lib, bk, bv):
+    cfg = kvq.CacheConfig(batch=3, n_q_heads=4, n_kv_heads=1, bits_k=bk, bits_v=bv,
+                          max_len=512, residual=64)
+    L0 = [0, 90, 95]
+    total = 200
+    cache = kvq.QuantKVCache(cfg)
+    ks, vs = synth.kv_heads(7, 3, total + 10)  # [3 sequences as heads, T, 128]
+    for b, L in enumerate(L0):
+        if L:
+            kvq.kvq_pack(cache, ks[b:b + 1, :L][None].cuda(), vs[b:b + 1, :L][None].cuda(),
+                         batch_begin=b)
+    lens = list(L0)
+    for step in range(total - 95):
+        kn = torch.stack([ks[b, lens[b]] for b in range(3)])[:, None, None].cuda()
+        vn = torch.stack([vs[b, lens[b]] for b in range(3)])[:, None, None].cuda()
+        kvq.kvq_pack(cache, kn.contiguous(), vn.contiguous())
+        lens = [x + 1 for x in lens]
+        if step % 9 == 0 or step > total - 100:
+            torch.cuda.synchronize()
+            assert cache.seq_lens().cpu().tolist() == lens
+            for b in range(3):
+                L = lens[b]
+                want = quant.quantize_head(ks[b, :L].numpy(), vs[b, :L].numpy(), bk, bv, 64)
+                _util.assert_head_equal(_util.head_arrays(cache, b, 0, L), want)
+
+
+def test_multi_token_appends_match_one_shot_prefill(kvq_lib):
+    cfg = kvq.CacheConfig(batch=1, n_q_heads=4, n_kv_heads=2, bits_k=2, bits_v=4, max_len=1024)
+    k, v = synth.kv_heads(11, 2, 700)
+    cache = kvq.QuantKVCache(cfg)
+    pos = 0
+    for n in (5, 33, 1, 64, 200, 31, 32, 100, 234):
+        kvq.kvq_pack(cache, k[:, pos:pos + n][None].contiguous().cuda(),
+                     v[:, pos:pos + n][None].contiguous().cuda())
+        pos += n
+    assert pos == 700
+    torch.cuda.synchronize()
+    for h in range(2):
+        want = quant.quantize_head(k[h].numpy(), v[h].numpy(), 2, 4, 128)
+        _util.assert_head_equal(_util.head_arrays(cache, 0, h, 700), want)
+
+
+def test_overflow_sets_flag_and_leaves_cache(kvq_lib):
+    cfg = kvq.CacheConfig(batch=2, n_q_heads=4, n_kv_heads=1, bits_k=1, bits_v=1, max_len=256)
+    k, v = synth.kv_heads(3, 1, 300)
+    cache = kvq.QuantKVCache(cfg)
+    kvq.kvq_pack(cache, k[:, :250][None].cuda(), v[:, :250][None].cuda(), batch_begin=0)
+    before = cache.buffer.clone()
+    kvq.kvq_pack(cache, k[:, 250:260][None].cuda(), v[:, 250:260][None].cuda(), batch_begin=0)
+    torch.cuda.synchronize()
+    assert cache.flags() & kvq.FLAG_OVERFLOW
+    assert cache.seq_lens().cpu().tolist() == [250, 0]
+    diff = (cache.buffer != before).nonzero().flatten().cpu()
+    flag_byte = cache.offsets[3] + 4 * cfg.batch
+    assert all(flag_byte <= int(i) < flag_byte + 4 for i in diff)
+    cache.reset()
+    torch.cuda.synchronize()
+    assert cache.flags() == 0 and cache.seq_lens().cpu().tolist() == [0, 0]
+
+
+def test_constant_and_grid_groups_reach_exact_codes(kvq_lib):
+    cfg = kvq.CacheConfig(batch=1, n_q_heads=1, n_kv_heads=1, bits_k=8, bits_v=2, max_len=256)
+    L = 192
+    k = torch.zeros(1, L, 128, dtype=torch.float16)
+    k[0, :, :64] = 3.5  # constant key groups -> scale 0, code 0
+    k[0, :, 64:] = torch.arange(L, dtype=torch.float16)[:, None] % 32 * 8  # grid 0, 8, .. 240
+    k[0, 31::32, 64:] = 255.0  # with 255 on top: range 255, scale 1, codes = values
+    v = (torch.arange(128) % 4).to(torch.float16).repeat(1, L, 1) * 0.25 - 1.0  # grid on 0.25
+    cache = kvq.QuantKVCache(cfg)
+    kvq.kvq_pack(cache, k[None].cuda(), v[None].cuda())
+    torch.cuda.synchronize()
+    got = _util.head_arrays(cache, 0, 0, L)
+    want = quant.quantize_head(k[0].numpy(), v[0].numpy(), 8, 2, 128)
+    _util.assert_head_equal(got, want)
+    assert np.all(got["k_scale"][:, :64] == 0)
+    assert np.all(got["k_scale"][:, 64:] == 1)
+    assert np.all(got["v_scale"].astype(np.float64) == 0.25)
