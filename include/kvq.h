@@ -188,6 +188,31 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache,
                            void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * kvq_decode_attn_noalloc — kvq_decode_attn without a caller workspace.
+ * The paper has no counterpart; this serves callers that cannot allocate
+ * device memory where they run a decode step: code inside a framework whose
+ * memory pool owns the whole GPU (a raw allocation would fail or fragment
+ * it), or a serving loop that must not allocate per step.  The split
+ * partials and tickets live in one built-in device array of
+ * KVQ_NOALLOC_SCRATCH_BYTES, which every GPU that loads this library holds
+ * until the process exits.
+ *   Arguments and results: those of kvq_decode_attn, without workspace.
+ *   Returns KVQ_ERR_CAPACITY, with nothing enqueued, when
+ *   kvq_attn_workspace_bytes(cfg, n_splits) > KVQ_NOALLOC_SCRATCH_BYTES.
+ *   The first call on a device looks up the array's device address (once
+ *   per device, with that device current): make that first call before any
+ *   stream capture.  Every call shares the one array and it keeps the last
+ *   call's contents; each call zeroes the tickets it uses before its kernel.
+ *   Calls that overlap on the GPU (different streams, or unordered work)
+ *   race and give wrong results.  Allocates and frees nothing.
+ */
+#define KVQ_NOALLOC_SCRATCH_BYTES (4u << 20)
+kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache,
+                                   const uint16_t* q, uint16_t* out,
+                                   float softmax_scale, int32_t n_splits,
+                                   void* stream);
+
+/*
  * DGAP parameters (Sec. 4.2 detector, Sec. 4.3 corrector).  Weights are
  * device fp32, row-major [out][in]; H = hidden.
  *   detector  f = w2 . relu(W1 phi + b1) + b2, r = sigmoid(f)   (Eq. 6)

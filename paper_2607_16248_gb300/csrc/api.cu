@@ -249,6 +249,34 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const 
                      "kvq_decode_attn launch");
 }
 
+kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache,
+                                   const uint16_t* q, uint16_t* out, float softmax_scale,
+                                   int32_t n_splits, void* stream) {
+  kvq_status s = check_config(cfg);
+  if (s != KVQ_OK) return s;
+  if ((s = check_cache(*cfg, cache)) != KVQ_OK) return s;
+  if (!q || !out) return fail(KVQ_ERR_ARG, "q / out is NULL");
+  if (!aligned16(q) || !aligned16(out)) return fail(KVQ_ERR_ALIGN, "q / out must be 16-byte aligned");
+  if (!(softmax_scale >= 0.0f) || isinf(softmax_scale))
+    return fail(KVQ_ERR_ARG, "softmax_scale must be finite and >= 0");
+  if (n_splits == 0) n_splits = default_splits(*cfg);
+  if (n_splits < 1 || n_splits > kMaxSplits)
+    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits, n_splits);
+  Dims d = make_dims(*cfg);
+  const size_t need = attn_workspace_bytes(d, n_splits);
+  if (need > attn_static_scratch_bytes())
+    return fail(KVQ_ERR_CAPACITY,
+                "this config needs %zu bytes of scratch but the built-in array holds %zu; "
+                "use kvq_decode_attn with a workspace, or fewer splits",
+                need, attn_static_scratch_bytes());
+  const float scale = softmax_scale == 0.0f ? 1.0f / sqrtf((float)kHeadDim) : softmax_scale;
+  return cuda_status(launch_decode_attn_static(d, *cache, reinterpret_cast<const __half*>(q),
+                                               reinterpret_cast<__half*>(out),
+                                               scale * 1.4426950408889634f, n_splits,
+                                               static_cast<cudaStream_t>(stream)),
+                     "kvq_decode_attn_noalloc launch");
+}
+
 static kvq_status check_dgap(const dgap_params* p, int32_t batch, int32_t vocab) {
   if (!p) return fail(KVQ_ERR_ARG, "params is NULL");
   if (batch < 1 || vocab < 1) return fail(KVQ_ERR_SHAPE, "batch and vocab must be >= 1");

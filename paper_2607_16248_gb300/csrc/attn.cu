@@ -13,6 +13,8 @@
 
 #include <float.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace kvq {
@@ -297,6 +299,60 @@ cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& c, const __half* 
     case 4: return launch_bv<4>(d, c, q, out, scale_log2, S, ws, st);
     default: return launch_bv<8>(d, c, q, out, scale_log2, S, ws, st);
   }
+}
+
+// ---------------------------------------------------------------------------
+// Decode attention without caller-supplied scratch (kvq_decode_attn_noalloc).
+//
+// Some callers cannot allocate device memory where they run a decode step: a
+// host framework whose pool owns every byte of the GPU (a raw allocation would
+// fail or fragment it), or a serving loop that must not allocate per step.
+// For them the split partials and tickets live in this one file-scope device
+// array of fixed size, which every GPU that loads the library holds until the
+// process exits.  All calls share it, so calls that overlap on the GPU race.
+// ---------------------------------------------------------------------------
+
+namespace {
+constexpr size_t kStaticScratchBytes = size_t(4) << 20;  // 4 MiB
+constexpr int kMaxDevices = 64;
+__device__ __align__(256) unsigned char g_attn_scratch[kStaticScratchBytes];
+
+// Device address of g_attn_scratch on the current device, looked up once per
+// device with that device current.  In host code the symbol is only a
+// host-side stand-in: passing it to a kernel would fault or silently use the
+// wrong memory, so only the looked-up address is ever used.
+cudaError_t static_scratch(void** out) {
+  static std::mutex mu;
+  static void* addr[kMaxDevices] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_attn_scratch);
+    if (e != cudaSuccess) return e;
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return cudaSuccess;
+}
+}  // namespace
+
+size_t attn_static_scratch_bytes() { return kStaticScratchBytes; }
+
+cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& c, const __half* q,
+                                      __half* out, float scale_log2, int S, cudaStream_t st) {
+  void* ws = nullptr;
+  cudaError_t e = static_scratch(&ws);
+  if (e != cudaSuccess) return e;
+  // The array keeps the previous call's contents: the tickets must start at
+  // zero, the partials are always written before they are read.
+  const Ws w = carve(ws, d.batch, d.hq, d.hkv, S);
+  e = cudaMemsetAsync(w.tk, 0, (size_t)d.batch * d.hkv * sizeof(unsigned), st);
+  if (e != cudaSuccess) return e;
+  return launch_decode_attn(d, c, q, out, scale_log2, S, ws, st);
 }
 
 }  // namespace kvq

@@ -68,6 +68,10 @@ cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& cache, const __ha
                                __half* out, float scale_log2, int n_splits,
                                void* workspace, cudaStream_t stream);
 size_t attn_workspace_bytes(const Dims& d, int n_splits);
+size_t attn_static_scratch_bytes();
+cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& cache, const __half* q,
+                                      __half* out, float scale_log2, int n_splits,
+                                      cudaStream_t stream);
 
 struct DgapDims {
   int batch, vocab, K, hidden, n_chunks;

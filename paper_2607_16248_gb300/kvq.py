@@ -25,8 +25,9 @@ EXPORTS = (
     "kvq_last_error", "kvq_version", "kvq_validate_config", "kvq_page_bytes",
     "kvq_cache_layout", "kvq_cache_bind", "kvq_cache_reset", "kvq_pack",
     "kvq_attn_workspace_bytes", "kvq_attn_default_splits", "kvq_workspace_init",
-    "kvq_decode_attn", "dgap_workspace_bytes", "dgap_restore",
+    "kvq_decode_attn", "kvq_decode_attn_noalloc", "dgap_workspace_bytes", "dgap_restore",
 )
+NOALLOC_SCRATCH_BYTES = 4 << 20
 
 
 class KvqError(RuntimeError):
@@ -77,6 +78,7 @@ def lib():
             "kvq_attn_default_splits": (I32, [cfg_p]),
             "kvq_workspace_init": (I32, [P, SZ, P]),
             "kvq_decode_attn": (I32, [cfg_p, cache_p, P, P, F32, I32, P, SZ, P]),
+            "kvq_decode_attn_noalloc": (I32, [cfg_p, cache_p, P, P, F32, I32, P]),
             "dgap_workspace_bytes": (SZ, [I32, I32, par_p]),
             "dgap_restore": (I32, [par_p, P, I32, I32, P, P, P, P, P, P, P, SZ, P]),
         }
@@ -251,6 +253,24 @@ def kvq_decode_attn(cache: QuantKVCache, q, out=None, softmax_scale=0.0, n_split
                                  float(softmax_scale), n_splits,
                                  _dev(workspace, torch.uint8, "workspace"), workspace.numel(),
                                  _stream(stream)))
+    return out
+
+
+def kvq_decode_attn_noalloc(cache: QuantKVCache, q, out=None, softmax_scale=0.0, n_splits=0,
+                            stream=None):
+    """kvq_decode_attn with the library's built-in scratch array instead of a
+    workspace, for callers that cannot allocate device memory per step.  Calls
+    share the array: do not let two of them overlap on the GPU."""
+    cfg = cache.cfg
+    if q.shape != (cfg.batch, cfg.n_q_heads, cfg.head_dim):
+        raise ValueError(f"q must be [{cfg.batch}, {cfg.n_q_heads}, {cfg.head_dim}]")
+    if out is None:
+        out = torch.empty_like(q)
+    c = cfg.c()
+    _check(lib().kvq_decode_attn_noalloc(ctypes.byref(c), ctypes.byref(cache._c),
+                                         _dev(q, torch.float16, "q"),
+                                         _dev(out, torch.float16, "out"), float(softmax_scale),
+                                         n_splits, _stream(stream)))
     return out
 
 
