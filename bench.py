@@ -80,10 +80,11 @@ def packed_len(L, R=128):
 
 def attn_bytes(L, hkv, hq, bk, bv, R=128):
     """Algorithmic HBM bytes of one sequence's attention for one layer:
-    packed codes + scale/zero of Lq tokens, fp16 residual tokens, q and out."""
+    packed codes + scale/zero of Lq tokens, fp16 residual tokens, q (fp16 in)
+    and out (fp32)."""
     Lq = packed_len(L, R)
     per_tok = 16 * (bk + bv) + 32
-    return hkv * (Lq * per_tok + (L - Lq) * 512) + 2 * hq * 128 * 2
+    return hkv * (Lq * per_tok + (L - Lq) * 512) + hq * 128 * (2 + 4)
 
 
 def source_digest(*names):
@@ -319,7 +320,7 @@ class Step:
         self.q = torch.randn(layers, B, hq, 128, generator=g, device=device).half()
         self.k_new = torch.randn(layers, B, hkv, 1, 128, generator=g, device=device).half()
         self.v_new = torch.randn(layers, B, hkv, 1, 128, generator=g, device=device).half()
-        self.out = torch.empty(layers, B, hq, 128, dtype=torch.float16, device=device)
+        self.out = torch.empty(layers, B, hq, 128, dtype=torch.float32, device=device)
         self.ws_attn = kvq.attn_workspace(self.cfg, 0, device)
         self.n_splits = kvq.default_splits(self.cfg)
         self.dgap = kvq.DGAP(synth.dgap_weights(seed, K=DGAP_K, hidden=DGAP_HIDDEN), K=DGAP_K,

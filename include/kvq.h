@@ -79,9 +79,9 @@ typedef struct kvq_config {
  * pages   [batch][n_kv_heads][max_len / 32][page_bytes], one page per 32-token
  *         block, page_bytes = 512 * (bits_k + bits_v) + 1024:
  *           K codes  [128 channel][bits_k] uint32   (group = 32 tokens of one channel)
- *           K meta   [128 channel] {fp16 scale, fp16 zero}
- *           V codes  [32 token][4 group][bits_v] uint32 (group = 32 channels of one token)
- *           V meta   [32 token][4 group] {fp16 scale, fp16 zero}
+ *           K meta   fp16 scale[128 channel], then fp16 zero[128 channel]
+ *           V codes  [4 group][32 token][bits_v] uint32 (group = 32 channels of one token)
+ *           V meta   fp16 scale[4 group][32 token], then fp16 zero[4 group][32 token]
  *         Element i of a group occupies bits [(i*b) mod 32, +b) of word
  *         floor(i*b / 32).  Quantizer (b bits, group x_1..x_32):
  *           zero  = min x_i
@@ -152,8 +152,8 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache,
 
 /*
  * Split-K workspace for kvq_decode_attn: per (sequence, query head, split)
- * partial max, sum and fp32 output row, plus one ticket per (sequence,
- * kv-head).  n_splits = 0 means the library's choice for this config.
+ * partial max, sum and fp32 output row for n_splits + 1 splits, plus one
+ * ticket per (sequence, kv-head).  n_splits = 0 means the library's choice.
  * Returns 0 on an invalid config.
  */
 size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits);
@@ -174,16 +174,20 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream);
  * over all L = seq_len[b] cached tokens (Sec. 1 gives softmax(QK^T/sqrt(d_k))V;
  * g(i) = i / (n_q_heads / n_kv_heads)).  K_hat, V_hat are the dequantized
  * blocks plus the fp16 residual window.
- *   q, out         device fp16 [batch][n_q_heads][128], 16-byte aligned.
+ *   q              device fp16 [batch][n_q_heads][128], 16-byte aligned.
+ *   out            device fp32 [batch][n_q_heads][128], 16-byte aligned (the
+ *                  fp32 accumulation result; rounding it to fp16 is left to
+ *                  the caller).
  *   softmax_scale  0 selects 1/sqrt(128).
- *   n_splits       0 = kvq_attn_default_splits(cfg); else 1..1024.
+ *   n_splits       splits of the packed blocks (the fp16 window always gets
+ *                  one more); 0 = kvq_attn_default_splits(cfg); else 1..255.
  *   workspace      device, >= kvq_attn_workspace_bytes(cfg, n_splits), zeroed
  *                  once by kvq_workspace_init.
  * A sequence with L = 0 gets a zero output.  Calls that share a workspace
  * must not overlap on the GPU.
  */
 kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache,
-                           const uint16_t* q, uint16_t* out,
+                           const uint16_t* q, float* out,
                            float softmax_scale, int32_t n_splits,
                            void* workspace, size_t ws_bytes, void* stream);
 
@@ -208,7 +212,7 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache,
  */
 #define KVQ_NOALLOC_SCRATCH_BYTES (4u << 20)
 kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache,
-                                   const uint16_t* q, uint16_t* out,
+                                   const uint16_t* q, float* out,
                                    float softmax_scale, int32_t n_splits,
                                    void* stream);
 

@@ -115,14 +115,7 @@ static int sm_count() {
 }
 
 static int default_splits(const kvq_config& c) {
-  const int bh = c.batch * c.n_kv_heads;
-  const int max_blocks = c.max_len / kGroup;
-  int s = (2 * sm_count() + bh - 1) / bh;
-  const int cap = (max_blocks + 7) / 8;  // keep >= ~8 blocks per split
-  if (s > cap) s = cap;
-  if (s < 1) s = 1;
-  if (s > kMaxSplits) s = kMaxSplits;
-  return s;
+  return attn_default_splits(make_dims(c), sm_count());
 }
 
 }  // namespace kvq
@@ -209,8 +202,8 @@ int32_t kvq_attn_default_splits(const kvq_config* cfg) {
 size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits) {
   if (check_config(cfg) != KVQ_OK) return 0;
   if (n_splits == 0) n_splits = default_splits(*cfg);
-  if (n_splits < 1 || n_splits > kMaxSplits) {
-    set_error("n_splits must be in [1, %d] (got %d)", kMaxSplits, n_splits);
+  if (n_splits < 1 || n_splits > kMaxSplits - 1) {
+    set_error("n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, n_splits);
     return 0;
   }
   return attn_workspace_bytes(make_dims(*cfg), n_splits);
@@ -223,7 +216,7 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream) {
 }
 
 kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const uint16_t* q,
-                           uint16_t* out, float softmax_scale, int32_t n_splits,
+                           float* out, float softmax_scale, int32_t n_splits,
                            void* workspace, size_t ws_bytes, void* stream) {
   kvq_status s = check_config(cfg);
   if (s != KVQ_OK) return s;
@@ -233,8 +226,8 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const 
   if (!(softmax_scale >= 0.0f) || isinf(softmax_scale))
     return fail(KVQ_ERR_ARG, "softmax_scale must be finite and >= 0");
   if (n_splits == 0) n_splits = default_splits(*cfg);
-  if (n_splits < 1 || n_splits > kMaxSplits)
-    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits, n_splits);
+  if (n_splits < 1 || n_splits > kMaxSplits - 1)
+    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, n_splits);
   Dims d = make_dims(*cfg);
   const size_t need = attn_workspace_bytes(d, n_splits);
   if (!workspace) return fail(KVQ_ERR_ARG, "workspace is NULL");
@@ -244,13 +237,13 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const 
   const float scale = softmax_scale == 0.0f ? 1.0f / sqrtf((float)kHeadDim) : softmax_scale;
   const float scale_log2 = scale * 1.4426950408889634f;
   return cuda_status(launch_decode_attn(d, *cache, reinterpret_cast<const __half*>(q),
-                                        reinterpret_cast<__half*>(out), scale_log2, n_splits,
+                                        out, scale_log2, n_splits,
                                         workspace, static_cast<cudaStream_t>(stream)),
                      "kvq_decode_attn launch");
 }
 
 kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache,
-                                   const uint16_t* q, uint16_t* out, float softmax_scale,
+                                   const uint16_t* q, float* out, float softmax_scale,
                                    int32_t n_splits, void* stream) {
   kvq_status s = check_config(cfg);
   if (s != KVQ_OK) return s;
@@ -260,8 +253,8 @@ kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache
   if (!(softmax_scale >= 0.0f) || isinf(softmax_scale))
     return fail(KVQ_ERR_ARG, "softmax_scale must be finite and >= 0");
   if (n_splits == 0) n_splits = default_splits(*cfg);
-  if (n_splits < 1 || n_splits > kMaxSplits)
-    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits, n_splits);
+  if (n_splits < 1 || n_splits > kMaxSplits - 1)
+    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, n_splits);
   Dims d = make_dims(*cfg);
   const size_t need = attn_workspace_bytes(d, n_splits);
   if (need > attn_static_scratch_bytes())
@@ -271,7 +264,7 @@ kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache
                 need, attn_static_scratch_bytes());
   const float scale = softmax_scale == 0.0f ? 1.0f / sqrtf((float)kHeadDim) : softmax_scale;
   return cuda_status(launch_decode_attn_static(d, *cache, reinterpret_cast<const __half*>(q),
-                                               reinterpret_cast<__half*>(out),
+                                               out,
                                                scale * 1.4426950408889634f, n_splits,
                                                static_cast<cudaStream_t>(stream)),
                      "kvq_decode_attn_noalloc launch");

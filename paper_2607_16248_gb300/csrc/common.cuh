@@ -12,7 +12,7 @@ namespace kvq {
 constexpr int kHeadDim = 128;
 constexpr int kGroup = 32;
 constexpr int kMaxGq = 8;        // largest n_q_heads / n_kv_heads supported
-constexpr int kMaxSplits = 1024;
+constexpr int kMaxSplits = 256;    // splits per (sequence, kv-head), window split included
 constexpr int kMaxK = 64;        // largest DGAP recovery window
 constexpr int kMaxHidden = 1024; // largest DGAP hidden width
 
@@ -22,6 +22,7 @@ __host__ __device__ inline int v_codes_bytes(int bits_v) { return 512 * bits_v; 
 __host__ __device__ inline int page_bytes(int bits_k, int bits_v) {
   return 512 * (bits_k + bits_v) + 1024;
 }
+constexpr int page_bytes_c(int bits_k, int bits_v) { return 512 * (bits_k + bits_v) + 1024; }
 // Offsets of the four regions of a page.
 __host__ __device__ inline int page_off_kmeta(int bits_k) { return 512 * bits_k; }
 __host__ __device__ inline int page_off_vcodes(int bits_k) { return 512 * bits_k + 512; }
@@ -65,12 +66,13 @@ cudaError_t launch_pack(const Dims& d, const kvq_cache& cache, const __half* k_n
                         const __half* v_new, int n_new, int batch_begin,
                         int batch_count, cudaStream_t stream);
 cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& cache, const __half* q,
-                               __half* out, float scale_log2, int n_splits,
+                               float* out, float scale_log2, int n_splits,
                                void* workspace, cudaStream_t stream);
 size_t attn_workspace_bytes(const Dims& d, int n_splits);
+int attn_default_splits(const Dims& d, int sm_count);
 size_t attn_static_scratch_bytes();
 cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& cache, const __half* q,
-                                      __half* out, float scale_log2, int n_splits,
+                                      float* out, float scale_log2, int n_splits,
                                       cudaStream_t stream);
 
 struct DgapDims {

@@ -23,10 +23,10 @@ struct Tile {
   __half v[kGroup][kRowPad];
 };
 
-// Quantize the 32 values x[] and return the packed words + (scale, zero).
+// Quantize the 32 values x[] and return the packed words, scale and zero.
 template <int B>
 __device__ __forceinline__ void quantize_group(const float (&x)[kGroup], uint32_t (&w)[B],
-                                               __half2& meta) {
+                                               __half& scale, __half& zero) {
   constexpr float kLevels = float((1 << B) - 1);
   float lo = x[0], hi = x[0];
 #pragma unroll
@@ -48,7 +48,8 @@ __device__ __forceinline__ void quantize_group(const float (&x)[kGroup], uint32_
     }
     w[(i * B) / 32] |= c << ((i * B) % 32);
   }
-  meta = __halves2half2(s_h, __float2half_rn(lo));  // lo is an fp16 value: exact
+  scale = s_h;
+  zero = __float2half_rn(lo);  // lo is an fp16 value: exact
 }
 
 template <int B>
@@ -63,28 +64,34 @@ __device__ __forceinline__ void quantize_key_channel(const Tile& t, int c, char*
 #pragma unroll
   for (int i = 0; i < kGroup; ++i) x[i] = __half2float(t.k[i][c]);
   uint32_t w[B];
-  __half2 meta;
-  quantize_group<B>(x, w, meta);
+  __half sc, z;
+  quantize_group<B>(x, w, sc, z);
   store_words<B>(reinterpret_cast<uint32_t*>(page) + c * B, w);
-  reinterpret_cast<__half2*>(page + page_off_kmeta(bits_k))[c] = meta;
+  __half* meta = reinterpret_cast<__half*>(page + page_off_kmeta(bits_k));
+  meta[c] = sc;
+  meta[kHeadDim + c] = z;
 }
 
+// Value groups are stored group-major: index = grp * 32 + tok; the 128
+// scales precede the 128 zeros.
 template <int B>
 __device__ __forceinline__ void quantize_value_group(const Tile& t, int pair, char* page,
                                                      int bits_k, int bits_v) {
-  const int tok = pair >> 2, grp = pair & 3;
+  const int grp = pair >> 5, tok = pair & 31;
   float x[kGroup];
 #pragma unroll
   for (int i = 0; i < kGroup; ++i) x[i] = __half2float(t.v[tok][grp * kGroup + i]);
   uint32_t w[B];
-  __half2 meta;
-  quantize_group<B>(x, w, meta);
+  __half sc, z;
+  quantize_group<B>(x, w, sc, z);
   store_words<B>(reinterpret_cast<uint32_t*>(page + page_off_vcodes(bits_k)) + pair * B, w);
-  reinterpret_cast<__half2*>(page + page_off_vmeta(bits_k, bits_v))[pair] = meta;
+  __half* meta = reinterpret_cast<__half*>(page + page_off_vmeta(bits_k, bits_v));
+  meta[pair] = sc;
+  meta[kHeadDim + pair] = z;
 }
 
 // 256 threads: 0..127 quantize one key channel each, 128..255 one
-// (token, 32-channel group) value group each.
+// (32-channel group, token) value group each.
 __device__ void quantize_tile(const Tile& t, char* page, int bits_k, int bits_v) {
   const int tid = threadIdx.x;
   if (tid < kHeadDim) {

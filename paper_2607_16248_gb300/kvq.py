@@ -239,17 +239,18 @@ def default_splits(cfg: CacheConfig):
 
 def kvq_decode_attn(cache: QuantKVCache, q, out=None, softmax_scale=0.0, n_splits=0,
                     workspace=None, stream=None):
-    """out = softmax(q K^T * scale) V over the cache; q fp16 [batch, n_q_heads, 128]."""
+    """out = softmax(q K^T * scale) V over the cache; q fp16 [batch, n_q_heads, 128],
+    out fp32 of the same shape."""
     cfg = cache.cfg
     if q.shape != (cfg.batch, cfg.n_q_heads, cfg.head_dim):
         raise ValueError(f"q must be [{cfg.batch}, {cfg.n_q_heads}, {cfg.head_dim}]")
     if out is None:
-        out = torch.empty_like(q)
+        out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
     if workspace is None:
         workspace = attn_workspace(cfg, n_splits, q.device)
     c = cfg.c()
     _check(lib().kvq_decode_attn(ctypes.byref(c), ctypes.byref(cache._c),
-                                 _dev(q, torch.float16, "q"), _dev(out, torch.float16, "out"),
+                                 _dev(q, torch.float16, "q"), _dev(out, torch.float32, "out"),
                                  float(softmax_scale), n_splits,
                                  _dev(workspace, torch.uint8, "workspace"), workspace.numel(),
                                  _stream(stream)))
@@ -265,11 +266,11 @@ def kvq_decode_attn_noalloc(cache: QuantKVCache, q, out=None, softmax_scale=0.0,
     if q.shape != (cfg.batch, cfg.n_q_heads, cfg.head_dim):
         raise ValueError(f"q must be [{cfg.batch}, {cfg.n_q_heads}, {cfg.head_dim}]")
     if out is None:
-        out = torch.empty_like(q)
+        out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
     c = cfg.c()
     _check(lib().kvq_decode_attn_noalloc(ctypes.byref(c), ctypes.byref(cache._c),
                                          _dev(q, torch.float16, "q"),
-                                         _dev(out, torch.float16, "out"), float(softmax_scale),
+                                         _dev(out, torch.float32, "out"), float(softmax_scale),
                                          n_splits, _stream(stream)))
     return out
 

@@ -26,15 +26,20 @@ def head_arrays(cache, b, h, L):
         return np.ascontiguousarray(pages[:, a:c])
 
     kw = sl(0, 512 * bk).view(np.uint32).reshape(nb, 128, bk)
-    km = sl(512 * bk, 512 * bk + 512).view(np.float16).reshape(nb, 128, 2)
-    vw = sl(512 * bk + 512, 512 * (bk + bv) + 512).view(np.uint32).reshape(nb, 32, 4, bv)
-    vm = sl(512 * (bk + bv) + 512, 512 * (bk + bv) + 1024).view(np.float16).reshape(nb, 32, 4, 2)
+    # key metadata: 128 scales, then 128 zeros (one per channel)
+    km = sl(512 * bk, 512 * bk + 512).view(np.float16).reshape(nb, 2, 128)
+    # value groups are stored group-major: [nb][4 group][32 token]; the 128
+    # scales precede the 128 zeros
+    vw = sl(512 * bk + 512, 512 * (bk + bv) + 512).view(np.uint32).reshape(nb, 4, 32, bv)
+    vw = np.ascontiguousarray(vw.transpose(0, 2, 1, 3))
+    vm = sl(512 * (bk + bv) + 512, 512 * (bk + bv) + 1024).view(np.float16).reshape(nb, 2, 4, 32)
+    vm = np.ascontiguousarray(vm.transpose(0, 1, 3, 2))
     kr, vr = cache.resid()
     slots = torch.tensor([p % cfg.ring for p in range(Lq, L)], dtype=torch.long)
     k_res = kr[b, h].cpu()[slots].numpy()
     v_res = vr[b, h].cpu()[slots].numpy()
-    return dict(k_words=kw, k_scale=km[..., 0], k_zero=km[..., 1], v_words=vw,
-                v_scale=vm[..., 0], v_zero=vm[..., 1], k_res=k_res, v_res=v_res,
+    return dict(k_words=kw, k_scale=km[:, 0], k_zero=km[:, 1], v_words=vw,
+                v_scale=vm[:, 0], v_zero=vm[:, 1], k_res=k_res, v_res=v_res,
                 bits_k=bk, bits_v=bv, L=L, Lq=Lq)
 
 

@@ -35,7 +35,7 @@ def test_noalloc_matches_workspace_path_on_two_calls(kvq_lib):
     for call in range(2):  # the second call finds the previous call's scratch contents
         q = synth.queries(500 + call, cfg.batch, cfg.n_q_heads).cuda()
         ref = kvq.kvq_decode_attn(cache, q)
-        out = torch.full_like(q, float("nan"))
+        out = torch.full(q.shape, float("nan"), dtype=torch.float32, device=q.device)
         status = lib.kvq_decode_attn_noalloc(ctypes.byref(c), ctypes.byref(cache._c),
                                              ctypes.c_void_p(q.data_ptr()),
                                              ctypes.c_void_p(out.data_ptr()), 0.0, 0, stream)
@@ -49,10 +49,10 @@ def test_noalloc_rejects_configs_beyond_its_array(kvq_lib):
     cfg = kvq.CacheConfig(batch=64, n_q_heads=64, n_kv_heads=8, bits_k=1, bits_v=1,
                           max_len=1 << 20)
     c = cfg.c()
-    need = kvq.lib().kvq_attn_workspace_bytes(ctypes.byref(c), 512)
+    need = kvq.lib().kvq_attn_workspace_bytes(ctypes.byref(c), 255)
     assert need > kvq.NOALLOC_SCRATCH_BYTES
     fake = ctypes.c_void_p(0x1000)  # never used: the size check fails first
     cache = kvq._Cache(fake, fake, fake, fake)
     status = kvq.lib().kvq_decode_attn_noalloc(ctypes.byref(c), ctypes.byref(cache), fake, fake,
-                                               0.0, 512, ctypes.c_void_p(None))
+                                               0.0, 255, ctypes.c_void_p(None))
     assert status == 4 and "scratch" in kvq.last_error()
