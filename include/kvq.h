@@ -81,9 +81,19 @@ typedef struct kvq_config {
  *           K codes  [128 channel][bits_k] uint32   (group = 32 tokens of one channel)
  *           K meta   fp16 scale[128 channel], then fp16 zero[128 channel]
  *           V codes  [4 group][32 token][bits_v] uint32 (group = 32 channels of one token)
- *           V meta   fp16 scale[4 group][32 token], then fp16 zero[4 group][32 token]
- *         Element i of a group occupies bits [(i*b) mod 32, +b) of word
- *         floor(i*b / 32).  Quantizer (b bits, group x_1..x_32):
+ *           V meta   fp16 scale[128], then fp16 zero[128]; (group g, token t)
+ *                    at 32 g + 8 (t / 8) + 2 (t mod 4) + (t / 4) mod 2, i.e. the
+ *                    tokens of each 8-token run in the order 0 4 1 5 2 6 3 7
+ *         For b >= 2, element i of a group occupies bits [(i*b) mod 32, +b)
+ *         of word floor(i*b / 32).  1-bit codes (512 bytes per tensor) are
+ *         stored in the order the attention kernel's MMA fragments read
+ *         them: with gid = t / 4, j = t mod 4 (keys: token t, channel
+ *         c = 16 ks + 4 tig + 2 h + e) the key code sits in word
+ *         16 gid + 4 tig + ks / 2 at bit (10 + 16 e + j - 4 (2 (ks mod 2) + h))
+ *         mod 32; with gid = (c mod 32) / 4, j = c mod 4, tig = t / 8,
+ *         r = t mod 4, e = (t / 4) mod 2 (values: token t, channel c) the
+ *         value code sits in word 16 gid + 4 tig + c / 32 at bit
+ *         (10 + 16 e + j - 4 r) mod 32.  Quantizer (b bits, group x_1..x_32):
  *           zero  = min x_i
  *           scale = RU16(RU32(RU32(max x_i - min x_i) / (2^b - 1)))
  *           code  = clamp(rint(RN32(RN32(x - zero) / scale)), 0, 2^b - 1)
@@ -152,13 +162,17 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache,
 
 /*
  * Split-K workspace for kvq_decode_attn: per (sequence, query head, split)
- * partial max, sum and fp32 output row for n_splits + 1 splits, plus one
- * ticket per (sequence, kv-head).  n_splits = 0 means the library's choice.
- * Returns 0 on an invalid config.
+ * partial max, sum and fp32 output row for up to n_splits + 1 splits, plus
+ * one ticket per (sequence, kv-head).  n_splits = 0 means the library's
+ * choice.  Returns 0 on an invalid config.
  */
 size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits);
 
-/* The split count kvq_decode_attn uses when passed n_splits = 0. */
+/*
+ * The split count kvq_decode_attn uses when passed n_splits = 0: one
+ * 512-thread CTA per SM over all (sequence, kv-head) pairs,
+ * SMs / (batch * n_kv_heads), between 1 and 255.
+ */
 int32_t kvq_attn_default_splits(const kvq_config* cfg);
 
 /*
@@ -179,8 +193,11 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream);
  *                  fp32 accumulation result; rounding it to fp16 is left to
  *                  the caller).
  *   softmax_scale  0 selects 1/sqrt(128).
- *   n_splits       splits of the packed blocks (the fp16 window always gets
- *                  one more); 0 = kvq_attn_default_splits(cfg); else 1..255.
+ *   n_splits       CTAs per (sequence, kv-head) that share its 32-token
+ *                  blocks and window chunks; 0 = kvq_attn_default_splits(cfg);
+ *                  else 1..255.  With more than one, each CTA writes a partial
+ *                  (max, sum, output row) to the workspace and the last to
+ *                  finish merges them.
  *   workspace      device, >= kvq_attn_workspace_bytes(cfg, n_splits), zeroed
  *                  once by kvq_workspace_init.
  * A sequence with L = 0 gets a zero output.  Calls that share a workspace

@@ -1,19 +1,22 @@
 // kvq_decode_attn: one decode step of grouped-query attention
 // softmax(q K^T * scale) V (Sec. 1 of the paper) over the packed KbVb cache.
 //
-// Split-K ("flash-decoding"): grid (n_splits + 1, n_kv_heads, batch).  Splits
-// 0 .. n_splits-1 share the packed 32-token blocks of one (sequence, kv-head);
-// the last split takes the fp16 residual window.  Each CTA writes one partial
-// (max, sum, unnormalised row) per query head; the last CTA of a
-// (sequence, kv-head) to finish (atomic ticket, no waiting) merges them:
+// Grid (S, n_kv_heads, batch) of 512-thread CTAs, one per SM.  The S CTAs
+// of one (sequence, kv-head) share its work: the packed 32-token blocks and
+// the 32-token chunks of the fp16 residual window are cut into contiguous
+// ranges, one per warp (a warp takes only blocks or only window chunks).
+// Each warp streams its own pages into a private ring of shared-memory slots
+// with bulk asynchronous copies (cp.async.bulk + one mbarrier per slot) and
+// keeps a running softmax state.  The warps of a CTA merge in shared memory
+// into one partial (max, sum, unnormalised row) per query head; with S > 1
+// the last CTA of a (sequence, kv-head) to finish (atomic ticket, no
+// waiting) merges the S partials:
 //   out = sum_s 2^{m_s - M} o_s / sum_s 2^{m_s - M} l_s.
 // Scores are kept in the log2 domain (scaled by softmax_scale * log2 e).
 //
 // Packed blocks run on the tensor cores (mma.sync m16n8k16, f16 in, f32
 // accumulate) with operands built in registers straight from the packed
-// codes.  A producer warp streams each split's contiguous pages into shared
-// memory with bulk asynchronous copies (cp.async.bulk + mbarrier); four
-// consumer warps each take one 32-token block per stage:
+// codes:
 //
 //   keys    S[t][h] = sum_c code[t][c] * (q_h[c] s_c) + sum_c q_h[c] z_c
 //           A = codes (M = tokens, K = channels), B = q*s split into an fp16
@@ -25,11 +28,10 @@
 //           high / low fp16 parts in columns 0..3 / 4..7; P moves from the
 //           score (accumulator) layout to the B layout with movmatrix.
 //
-// Codes become fp16 values without a table: for 1-bit codes a shifted bit
-// lands on an exponent bit (value 2^e), for wider codes the code is OR-ed into
-// the mantissa of 1024 and 1024 is subtracted.  The four tokens (keys) or
-// channels (values) a lane owns are chosen to sit in one nibble / byte of a
-// packed word; the resulting per-row power-of-two factors are undone on the
+// Codes become fp16 values without a table: for 1-bit codes (stored in
+// fragment order) a rotated bit lands on an exponent bit (value 2^e), for
+// wider codes the code is OR-ed into the mantissa of 1024 and 1024 is
+// subtracted.  The resulting per-row power-of-two factors are undone on the
 // fp32 results.  The fp16 residual window takes the same MMAs with operands
 // loaded by ldmatrix from rows staged in shared memory.  Query-head groups
 // wider than 4 use the SIMT path for every unit.
@@ -43,19 +45,15 @@
 namespace kvq {
 namespace {
 
-constexpr int kConsumers = 5;                 // computing warps; the last one also streams
-constexpr int kThreads = 32 * kConsumers;
-constexpr int kResWarps = kConsumers;         // warps that stage the fp16 window
-#ifndef KVQ_ATTN_CTAS_PER_SM
-#define KVQ_ATTN_CTAS_PER_SM 2
+#ifndef KVQ_ATTN_WARPS
+#define KVQ_ATTN_WARPS 16
 #endif
-#ifndef KVQ_ATTN_UNIT_BLOCKS
-#define KVQ_ATTN_UNIT_BLOCKS 2
-#endif
-constexpr int kCtasPerSm = KVQ_ATTN_CTAS_PER_SM;   // resident CTAs per SM
-constexpr int kUnitBlocks = KVQ_ATTN_UNIT_BLOCKS;  // blocks per consumer warp per stage
-constexpr int kStageBudget = (kCtasPerSm >= 3 ? 60 : 80) * 1024;  // staged page bytes per CTA
+constexpr int kWarps = KVQ_ATTN_WARPS;            // warps per CTA
+constexpr int kThreads = 32 * kWarps;
+constexpr int kCtasPerSm = kWarps <= 8 ? 2 : 1;   // resident CTAs per SM
+constexpr int kRingBudget = (kCtasPerSm == 2 ? 96 : 192) * 1024;  // staged page bytes per CTA
 constexpr long long kWaitCycles = 4000000000LL;  // bounded mbarrier waits (~2 s)
+constexpr int kZeroBytes = 512;                   // all-zero metadata rows
 
 struct Ws {
   float* m;       // [B][Hq][S]
@@ -80,13 +78,19 @@ __host__ __device__ inline Ws carve(void* base, int batch, int hq, int hkv, int 
   return w;
 }
 
-// Shared-memory areas of one CTA.  The merge area overlaps the stage
-// buffers: it is written only after every stage has been consumed.
-struct MergeArea {
-  float qs[kMaxGq][kHeadDim];           // SIMT path: q * scale * log2 e
-  float wm[kConsumers][kMaxGq];
-  float wl[kConsumers][kMaxGq];
-  float wo[kConsumers][kMaxGq][kHeadDim];
+// A warp's final state (row maximum, row sum, unnormalised output row per
+// query head).  A tensor-core warp writes it at the start of its own ring as
+// soon as it is done; SIMT warps have a region each at the start of shared
+// memory.
+struct WarpState {
+  float m[kMaxGq];
+  float l[kMaxGq];
+  float o[kMaxGq][kHeadDim];
+};
+// Small shared arrays of the merges (static shared memory).
+struct MergeSmall {
+  float ww[kWarps][kMaxGq];             // warp merge weights 2^(m_w - M)
+  float cta_m[kMaxGq];
   int last;
 };
 
@@ -116,9 +120,6 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
                "r"(bytes)
                : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
@@ -163,7 +164,7 @@ __device__ __forceinline__ int read_len(const int* p) {
 
 __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {
-  asm volatile(
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
       "{%8,%9}, {%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
@@ -171,7 +172,7 @@ __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1
 }
 __device__ __forceinline__ uint32_t movmatrix_t(uint32_t a) {
   uint32_t d;
-  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  asm("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
   return d;
 }
 
@@ -234,14 +235,20 @@ __device__ void simt_packed_unit(State& st, const float (*qs)[kHeadDim], int gq,
   const uint32_t* kc = reinterpret_cast<const uint32_t*>(page);
   const __half* ksc = reinterpret_cast<const __half*>(page + page_off_kmeta(BK));  // [128] then zeros
   const uint32_t* vc = reinterpret_cast<const uint32_t*>(page + page_off_vcodes(BK));
-  const __half* vsc = reinterpret_cast<const __half*>(page + page_off_vmeta(BK, BV));  // [4][32] then zeros
+  const __half* vsc = reinterpret_cast<const __half*>(page + page_off_vmeta(BK, BV));  // scales, zeros
   constexpr uint32_t kMaskK = (1u << BK) - 1u, kMaskV = (1u << BV) - 1u;
   float sc[kMaxGq];
 #pragma unroll
   for (int g = 0; g < kMaxGq; ++g) sc[g] = 0.0f;
   const int kword = (lane * BK) / 32, kshift = (lane * BK) % 32;
   for (int c = 0; c < kHeadDim; ++c) {
-    const uint32_t code = (kc[c * BK + kword] >> kshift) & kMaskK;
+    uint32_t code;
+    if (BK == 1) {
+      const int bit = key1_bit(lane, c);
+      code = (kc[bit >> 5] >> (bit & 31)) & 1u;
+    } else {
+      code = (kc[c * BK + kword] >> kshift) & kMaskK;
+    }
     const float kh = fmaf(__half2float(ksc[c]), (float)code, __half2float(ksc[kHeadDim + c]));
 #pragma unroll
     for (int g = 0; g < kMaxGq; ++g) {
@@ -251,12 +258,19 @@ __device__ void simt_packed_unit(State& st, const float (*qs)[kHeadDim], int gq,
   }
   const int grp = lane >> 3;
   online_update(st, sc, gq, kGroup, [&](int t, float (&v)[4]) {
-    const float sv = __half2float(vsc[grp * 32 + t]), zv = __half2float(vsc[kHeadDim + grp * 32 + t]);
+    const int mi = vmeta_index(grp, t);
+    const float sv = __half2float(vsc[mi]), zv = __half2float(vsc[kHeadDim + mi]);
     const uint32_t* w = vc + (grp * 32 + t) * BV;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      const int cc = (4 * lane + i) & 31;
-      const uint32_t code = (w[(cc * BV) / 32] >> ((cc * BV) % 32)) & kMaskV;
+      uint32_t code;
+      if (BV == 1) {
+        const int bit = val1_bit(t, 4 * lane + i);
+        code = (vc[bit >> 5] >> (bit & 31)) & 1u;
+      } else {
+        const int cc = (4 * lane + i) & 31;
+        code = (w[(cc * BV) / 32] >> ((cc * BV) % 32)) & kMaskV;
+      }
       v[i] = fmaf(sv, (float)code, zv);
     }
   });
@@ -311,27 +325,36 @@ __device__ void simt_resid_unit(State& st, const float (*qs)[kHeadDim], int gq, 
 template <int B>
 struct Codes;
 
+// 1-bit codes are stored in fragment order (key1_bit / val1_bit): the word
+// w of a lane rotated left by 4 r holds, at bit 10 + 16 e + j, the code of
+// row j and half e of one fragment register, so each register is one AND
+// (an fp16 with a single exponent bit set: 2^-14, 2^-13, 2^-11, 2^-7).
 template <>
 struct Codes<1> {
   __device__ static constexpr float inv(int j) {
     return j == 0 ? 16384.0f : j == 1 ? 8192.0f : j == 2 ? 2048.0f : 128.0f;
   }
   __device__ static int word(int gid) { return 0; }
-  __device__ static void get(uint32_t a, uint32_t b, uint32_t sel, int sh, uint32_t (&v)[4]) {
-    const uint32_t y = __byte_perm(a, b, sel) << sh;  // nibble -> bits 10..13 of each half
-    v[0] = y & 0x04000400u;  // exponent bit 0: 2^-14
-    v[1] = y & 0x08000800u;  // exponent bit 1: 2^-13
-    v[2] = y & 0x10001000u;  // exponent bit 2: 2^-11
-    v[3] = y & 0x20002000u;  // exponent bit 3: 2^-7
+  __device__ static void rot(uint32_t w, int r, uint32_t (&v)[4]) {
+    // r = 1, 2 only read bits that a plain shift keeps; r = 3 wraps around.
+    const uint32_t y = r == 0 ? w : r == 1 ? w << 4 : r == 2 ? w << 8 : __funnelshift_l(w, w, 12);
+    v[0] = y & 0x04000400u;
+    v[1] = y & 0x08000800u;
+    v[2] = y & 0x10001000u;
+    v[3] = y & 0x20002000u;
   }
 };
+
+__device__ __forceinline__ uint32_t comp(const uint4& u, int i) {
+  return i == 0 ? u.x : i == 1 ? u.y : i == 2 ? u.z : u.w;
+}
 template <>
 struct Codes<2> {
   __device__ static constexpr float inv(int j) {
     return j == 0 ? 1.0f : j == 1 ? 0.25f : j == 2 ? 0.0625f : 0.015625f;
   }
   __device__ static int word(int gid) { return gid >> 2; }
-  __device__ static void get(uint32_t a, uint32_t b, uint32_t sel, int, uint32_t (&v)[4]) {
+  __device__ static void get(uint32_t a, uint32_t b, uint32_t sel, uint32_t (&v)[4]) {
     const uint32_t x = __byte_perm(a, b, sel);  // the lane's byte -> bits 0..7 of each half
 #pragma unroll
     for (int j = 0; j < 4; ++j) v[j] = hsub1024((x & (0x00030003u << (2 * j))) | 0x64006400u);
@@ -341,7 +364,7 @@ template <>
 struct Codes<4> {
   __device__ static constexpr float inv(int j) { return (j & 1) ? 0.0625f : 1.0f; }
   __device__ static int word(int gid) { return gid >> 1; }
-  __device__ static void get(uint32_t a, uint32_t b, uint32_t sel, int, uint32_t (&v)[4]) {
+  __device__ static void get(uint32_t a, uint32_t b, uint32_t sel, uint32_t (&v)[4]) {
     const uint32_t x = __byte_perm(a, b, sel);  // the lane's 16 bits -> each half
     const uint32_t y = x >> 8;
     v[0] = hsub1024((x & 0x000F000Fu) | 0x64006400u);
@@ -354,7 +377,7 @@ template <>
 struct Codes<8> {
   __device__ static constexpr float inv(int) { return 1.0f; }
   __device__ static int word(int gid) { return gid; }
-  __device__ static void get(uint32_t a, uint32_t b, uint32_t, int, uint32_t (&v)[4]) {
+  __device__ static void get(uint32_t a, uint32_t b, uint32_t, uint32_t (&v)[4]) {
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const uint32_t x = __byte_perm(a, b, j | (j << 4) | ((4 + j) << 8) | ((4 + j) << 12));
@@ -378,10 +401,8 @@ __device__ __forceinline__ uint32_t code_selector(int gid) {
 struct Lane {
   int gid, tig;
   uint32_t sel_k, sel_v;   // byte-permute selectors for key / value words
-  int sh;                   // 1-bit codes: nibble shift to the exponent bits
   int wk, wv;               // word of a group that holds the lane's 4 codes
-  uint32_t lo_cols;         // all ones for lanes holding B columns 4..7
-  uint32_t row0, row1, rows4;  // all ones for A rows 0 / 1 / 0..3
+  uint32_t neg_lo;          // fp16x2 -1 for lanes holding B columns 4..7, else 0
   float p_lo;               // 1 for lanes holding score columns 4..7
 };
 
@@ -452,9 +473,19 @@ __device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, c
 // NB packed 32-token blocks (pages in shared memory) for one warp: scores of
 // all blocks, one softmax update, then the value MMAs.
 template <int BK, int BV, int NB>
-__device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const uint32_t (&qb)[16],
-                                        const Lane& ln, float scale_log2, TcState& st) {
-  const int gid = ln.gid, tig = ln.tig;
+__device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char* zero,
+                                        const uint32_t (&qb)[16], const Lane& ln,
+                                        float scale_log2, TcState& st) {
+  const int gid = ln.gid, tig = ln.tig, lane = 4 * gid + tig;
+  // Zero-point MMA rows: row bi (lane group gid = bi) reads block bi's key
+  // metadata, the other rows the all-zero area (same 512-byte extent).
+  const char* zrow = gid == 0 ? pg[0] + page_off_kmeta(BK)
+                     : (NB == 2 && gid == 1) ? pg[NB - 1] + page_off_kmeta(BK) : zero;
+  uint4 kw1[NB];
+  if constexpr (BK == 1) {
+#pragma unroll
+    for (int bi = 0; bi < NB; ++bi) kw1[bi] = *reinterpret_cast<const uint4*>(pg[bi] + 16 * lane);
+  }
 
   // ---- keys: S[t][h] ----
   // K slots of k-step ks: lane tig's slots (2tig, 2tig+1) and (2tig+8, 2tig+9)
@@ -465,31 +496,23 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const uint3
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int c = 16 * ks + 4 * tig;
-    uint32_t azk[NB][2];
 #pragma unroll
     for (int bi = 0; bi < NB; ++bi) {
       const char* kc = pg[bi];
       const char* kmeta = pg[bi] + page_off_kmeta(BK);
-      uint32_t w[4];
-      if (BK == 1) {
-        const uint4 w4 = *reinterpret_cast<const uint4*>(kc + 4 * c);
-        w[0] = w4.x;
-        w[1] = w4.y;
-        w[2] = w4.z;
-        w[3] = w4.w;
-      } else {
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          w[i] = *reinterpret_cast<const uint32_t*>(kc + 4 * ((c + i) * BK + ln.wk));
-      }
-      // scales of channels c..c+3, then their zeros (two fp16 per word)
+      // scales of channels c..c+3 (two fp16 per word)
       const uint2 sw = *reinterpret_cast<const uint2*>(kmeta + 2 * c);
-      const uint2 zw = *reinterpret_cast<const uint2*>(kmeta + 2 * (kHeadDim + c));
       uint32_t a0[4], a1[4], b[2];
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         uint32_t v[4];
-        Codes<BK>::get(w[2 * half], w[2 * half + 1], ln.sel_k, ln.sh, v);
+        if constexpr (BK == 1) {
+          Codes<1>::rot(comp(kw1[bi], ks >> 1), 2 * (ks & 1) + half, v);
+        } else {
+          const uint32_t wa = *reinterpret_cast<const uint32_t*>(kc + 4 * ((c + 2 * half) * BK + ln.wk));
+          const uint32_t wb = *reinterpret_cast<const uint32_t*>(kc + 4 * ((c + 2 * half + 1) * BK + ln.wk));
+          Codes<BK>::get(wa, wb, ln.sel_k, v);
+        }
         a0[2 * half] = v[0];
         a0[2 * half + 1] = v[1];
         a1[2 * half] = v[2];
@@ -497,19 +520,13 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const uint3
         const uint32_t s2 = half ? sw.y : sw.x;
         // q*s as fp16 high part (columns 0..3) or its exact residual (4..7)
         const __half2 hi = __hmul2(u2h(qb[2 * ks + half]), u2h(s2));
-        const uint32_t c_in = (h2u(hi) ^ 0x80008000u) & ln.lo_cols;
-        b[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), u2h(c_in)));
-        azk[bi][half] = half ? zw.y : zw.x;
+        b[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hmul2(hi, u2h(ln.neg_lo))));
       }
       mma16816(dk[bi][0], a0[0], a0[1], a0[2], a0[3], b[0], b[1]);
       mma16816(dk[bi][1], a1[0], a1[1], a1[2], a1[3], b[0], b[1]);
     }
-    uint32_t az[2];
-#pragma unroll
-    for (int half = 0; half < 2; ++half)
-      az[half] = NB == 2 ? (azk[0][half] & ln.row0) | (azk[NB - 1][half] & ln.row1)
-                         : azk[0][half] & ln.row0;
-    mma16816(dz, az[0], 0u, az[1], 0u, qb[2 * ks], qb[2 * ks + 1]);
+    const uint2 zw = *reinterpret_cast<const uint2*>(zrow + 2 * (kHeadDim + c));
+    mma16816(dz, zw.x, 0u, zw.y, 0u, qb[2 * ks], qb[2 * ks + 1]);
   }
   // Scores in the log2 domain.  Lanes tig and tig^2 hold the two parts.
   float sc[NB][4][2];
@@ -534,35 +551,25 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const uint3
   tc_softmax<NB>(sc, st, ln, pt);
 
   // ---- values: o^T[c][h] ----
-  // Group-major value pages: group g's (scale, zero) and 1-bit code words of
-  // the lane's tokens 8tig .. 8tig+7 are two 16-byte loads each.
+  // Value scales and zeros are stored in token pairs (t, t + 4), so the
+  // B-operand scale of (k-step ks, dl) is word 2ks + dl of the lane's 8-token
+  // run; zero-point MMA rows 0..3 = groups (lane groups gid >= 4 read zeros).
 #pragma unroll
   for (int bi = 0; bi < NB; ++bi) {
     const char* vc = pg[bi] + page_off_vcodes(BK);
     const char* vmeta = pg[bi] + page_off_vmeta(BK, BV);
-    // zeros of group gid & 3 (zero-point MMA rows) for the lane's 8 tokens,
-    // two fp16 per word: token 8tig + i is half (i & 1) of word i / 2
-    const uint4 z8 = *reinterpret_cast<const uint4*>(vmeta + 2 * (kHeadDim + 32 * (gid & 3) + 8 * tig));
-    const uint32_t zw[4] = {z8.x, z8.y, z8.z, z8.w};
-#pragma unroll
-    for (int ks = 0; ks < 2; ++ks) {
-      uint32_t azv[2];
-#pragma unroll
-      for (int dl = 0; dl < 2; ++dl)  // tokens 8tig + (2ks + dl) and + 4
-        azv[dl] = __byte_perm(zw[ks], zw[ks + 2], dl ? 0x7632 : 0x5410) & ln.rows4;
-      mma16816(st.zv, azv[0], 0u, azv[1], 0u, pt[bi][ks][0], pt[bi][ks][1]);
-    }
+    const char* vzrow = gid < 4 ? vmeta : zero;
+    const uint4 z8 = *reinterpret_cast<const uint4*>(vzrow + 2 * (kHeadDim + 32 * (gid & 3) + 8 * tig));
+    mma16816(st.zv, z8.x, 0u, z8.y, 0u, pt[bi][0][0], pt[bi][0][1]);
+    mma16816(st.zv, z8.z, 0u, z8.w, 0u, pt[bi][1][0], pt[bi][1][1]);
+    uint4 vw1;
+    if constexpr (BV == 1) vw1 = *reinterpret_cast<const uint4*>(vc + 16 * lane);
 #pragma unroll
     for (int g = 0; g < 4; ++g) {
       const uint4 s8 = *reinterpret_cast<const uint4*>(vmeta + 2 * (32 * g + 8 * tig));
-      const uint32_t mw[4] = {s8.x, s8.y, s8.z, s8.w};  // scales of tokens 8tig .. 8tig+7
+      const uint32_t mw[4] = {s8.x, s8.y, s8.z, s8.w};  // scale pairs of tokens (8tig + i, + 4)
       uint32_t cw[8];
-      if (BV == 1) {
-        const uint4 cl = *reinterpret_cast<const uint4*>(vc + 4 * (32 * g + 8 * tig));
-        const uint4 chh = *reinterpret_cast<const uint4*>(vc + 4 * (32 * g + 8 * tig + 4));
-        cw[0] = cl.x; cw[1] = cl.y; cw[2] = cl.z; cw[3] = cl.w;
-        cw[4] = chh.x; cw[5] = chh.y; cw[6] = chh.z; cw[7] = chh.w;
-      } else {
+      if constexpr (BV != 1) {
 #pragma unroll
         for (int i = 0; i < 8; ++i)
           cw[i] = *reinterpret_cast<const uint32_t*>(vc + 4 * ((32 * g + 8 * tig + i) * BV + ln.wv));
@@ -574,13 +581,13 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const uint3
         for (int dl = 0; dl < 2; ++dl) {
           const int ia = 2 * ks + dl, ib = ia + 4;  // tokens 8tig + ia, 8tig + ib
           uint32_t v[4];
-          Codes<BV>::get(cw[ia], cw[ib], ln.sel_v, ln.sh, v);
+          if constexpr (BV == 1) Codes<1>::rot(comp(vw1, g), ia, v);
+          else Codes<BV>::get(cw[ia], cw[ib], ln.sel_v, v);
           am0[2 * dl] = v[0];
           am0[2 * dl + 1] = v[1];
           am1[2 * dl] = v[2];
           am1[2 * dl + 1] = v[3];
-          const uint32_t s2 = __byte_perm(mw[ia >> 1], mw[ib >> 1], (ia & 1) ? 0x7632 : 0x5410);
-          bv[dl] = h2u(__hmul2(u2h(pt[bi][ks][dl]), u2h(s2)));
+          bv[dl] = h2u(__hmul2(u2h(pt[bi][ks][dl]), u2h(mw[ia])));
         }
         mma16816(st.acc[2 * g], am0[0], am0[1], am0[2], am0[3], bv[0], bv[1]);
         mma16816(st.acc[2 * g + 1], am1[0], am1[1], am1[2], am1[3], bv[0], bv[1]);
@@ -596,13 +603,9 @@ __device__ __forceinline__ Lane make_lane(int lane) {
   ln.tig = lane & 3;
   ln.sel_k = code_selector<BK>(ln.gid);
   ln.sel_v = code_selector<BV>(ln.gid);
-  ln.sh = 10 - 4 * (ln.gid & 1);
   ln.wk = Codes<BK>::word(ln.gid);
   ln.wv = Codes<BV>::word(ln.gid);
-  ln.lo_cols = ln.gid >= 4 ? 0xffffffffu : 0u;
-  ln.row0 = ln.gid == 0 ? 0xffffffffu : 0u;
-  ln.row1 = ln.gid == 1 ? 0xffffffffu : 0u;
-  ln.rows4 = ln.gid < 4 ? 0xffffffffu : 0u;
+  ln.neg_lo = ln.gid >= 4 ? 0xBC00BC00u : 0u;
   ln.p_lo = ln.tig >= 2 ? 1.0f : 0.0f;
   return ln;
 }
@@ -640,7 +643,7 @@ __device__ __forceinline__ void init_state(TcState& st) {
 // packed layout (nibble of a group, power-of-two factors, zero-point term);
 // otherwise channel = 16 * m-tile + row.
 template <bool kPacked, int BV>
-__device__ __forceinline__ void tc_write_state(const TcState& st, MergeArea& ma, int warp, int lane) {
+__device__ __forceinline__ void tc_write_state(const TcState& st, WarpState& ws, int lane) {
   const int gid = lane >> 2, tig = lane & 3;
   float l0 = st.l[0], l1 = st.l[1];
 #pragma unroll
@@ -652,10 +655,10 @@ __device__ __forceinline__ void tc_write_state(const TcState& st, MergeArea& ma,
   zsum[0] = st.zv[0] + __shfl_xor_sync(0xffffffffu, st.zv[0], 2);
   zsum[1] = st.zv[1] + __shfl_xor_sync(0xffffffffu, st.zv[1], 2);
   if (gid == 0 && tig < 2) {
-    ma.wm[warp][2 * tig] = st.m[0];
-    ma.wm[warp][2 * tig + 1] = st.m[1];
-    ma.wl[warp][2 * tig] = l0;
-    ma.wl[warp][2 * tig + 1] = l1;
+    ws.m[2 * tig] = st.m[0];
+    ws.m[2 * tig + 1] = st.m[1];
+    ws.l[2 * tig] = l0;
+    ws.l[2 * tig + 1] = l1;
   }
 #pragma unroll
   for (int g = 0; g < 4; ++g) {
@@ -673,166 +676,65 @@ __device__ __forceinline__ void tc_write_state(const TcState& st, MergeArea& ma,
         for (int hh = 0; hh < 2; ++hh) {
           const float a = st.acc[mtp][2 * rh + hh];
           const float full_v = a + __shfl_xor_sync(0xffffffffu, a, 2);
-          if (tig < 2) ma.wo[warp][2 * tig + hh][cch] = fmaf(full_v, inv, hh ? zg1 : zg0);
+          if (tig < 2) ws.o[2 * tig + hh][cch] = fmaf(full_v, inv, hh ? zg1 : zg0);
         }
       }
     }
   }
 }
 
-// Blocks per consumer warp and stage: two when pages are small enough that
-// two stages of them fit in shared memory.
-template <int BK, int BV>
-struct Unit {
-  static constexpr int kBlocks = (kUnitBlocks > 1 && page_bytes_c(BK, BV) <= 6144) ? kUnitBlocks : 1;
-};
-
-// Packed split `split` of one (sequence, kv-head) on the tensor cores: the
-// packed blocks nb of the sequence are cut into n_split ranges of
-// ceil(nb / n_split) blocks.  A page is written once, when its group leaves
-// the window, and never changes afterwards, so before waiting for the
-// previous kernel (programmatic dependent launch) the producer already
-// streams the full stages of the range given by a length read before the
-// wait.  If the length after the wait gives another range start (the
-// previous kernel flushed a group of this cache) those stages are discarded.
-template <int BK, int BV>
-__device__ void tc_split(const Dims& d, const char* pages_bh, int split, int n_split,
-                         const int* len_b, int n_bufs, unsigned char* smem, const __half* qh,
-                         int gq, float scale_log2, unsigned* flag, MergeArea& ma) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int page = page_bytes(BK, BV);
-  constexpr int NB = Unit<BK, BV>::kBlocks;
-  constexpr int per_stage = kConsumers * NB;  // blocks per stage
-  const int stage = per_stage * page;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)n_bufs * stage);
-  uint64_t* empty = full + n_bufs;
-  __shared__ int issued;
-  __shared__ int timed_out;
-  __shared__ int hint_len;
-
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < n_bufs; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&empty[i], kConsumers);
-    }
-    issued = 0;
-    timed_out = 0;
-    hint_len = read_len(len_b);
-    fence_mbar_init();
-  }
-  __syncthreads();
-
-  auto range = [&](int len, int& lo, int& end) {
-    const int nb = packed_len(len, d.residual) / kGroup;
-    const int per = (nb + n_split - 1) / n_split;
-    lo = min(nb, split * per);
-    end = min(nb, lo + per);
-  };
-  int lo_h, end_h;
-  range(hint_len, lo_h, end_h);
-  const int pre = min((end_h - lo_h) / per_stage, n_bufs);  // full stages streamed early
-
-  TcState st;
-  int consumed = 0;
-  const bool streamer = warp == kConsumers - 1 && lane == 0;
-  auto issue = [&](int s, int first_blk, int nblk) {
-    const int slot = s % n_bufs;
-    const uint32_t bytes = (uint32_t)(nblk * page);
-    mbar_expect_tx(&full[slot], bytes);
-    bulk_g2s(smem + (size_t)slot * stage, pages_bh + (long long)first_blk * page, bytes,
-             &full[slot]);
-    issued = s + 1;
-  };
-  if (streamer)
-    for (int s = 0; s < pre; ++s) issue(s, lo_h + s * per_stage, per_stage);
-  pdl_wait();
-  int lo, end;
-  range(read_len(len_b), lo, end);
-  const int skip = lo == lo_h ? 0 : pre;  // pre-streamed stages of a stale range
-  const int nblk = end - lo;
-  const int total = skip + (nblk + per_stage - 1) / per_stage;
-  auto real_issue = [&](int s) {  // pipeline stage s >= skip
-    const int r = s - skip;
-    issue(s, lo + r * per_stage, min(per_stage, nblk - r * per_stage));
-  };
-  if (streamer)
-    for (int s = pre; s < min(total, n_bufs); ++s) real_issue(s);
-
-  const Lane ln = make_lane<BK, BV>(lane);
-  uint32_t qb[16];
-  load_qb<true>(qb, qh, gq, ln);
-  init_state(st);
-  for (int s = 0; s < total; ++s) {
-    const int slot = s % n_bufs;
-    if (!mbar_wait(&full[slot], (s / n_bufs) & 1)) {
-      if (lane == 0) atomicOr(flag, 2u);
-      timed_out = 1;
-      break;
-    }
-    consumed = s + 1;
-    if (s >= skip) {
-      const int r = s - skip;
-      const int blk = r * per_stage + warp * NB;  // first of the warp's blocks
-      const char* base = reinterpret_cast<const char*>(smem) + (size_t)slot * stage;
-      if (blk + NB <= nblk) {
-        const char* pg[NB];
-#pragma unroll
-        for (int i = 0; i < NB; ++i) pg[i] = base + (warp * NB + i) * page;
-        tc_unit<BK, BV, NB>(pg, qb, ln, scale_log2, st);
-      } else if (NB > 1 && blk < nblk) {
-        const char* pg[1] = {base + warp * NB * page};
-        tc_unit<BK, BV, 1>(pg, qb, ln, scale_log2, st);
-      }
-    }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[slot]);
-    // The streaming lane refills this slot once every warp has released it.
-    if (streamer && s + n_bufs < total) {
-      if (!mbar_wait(&empty[slot], (s / n_bufs) & 1)) {
-        atomicOr(flag, 2u);
-        timed_out = 1;
-      } else {
-        real_issue(s + n_bufs);
-      }
-    }
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    // Copies issued past what the consumers took (the length shrank, or a
-    // wait gave up) land before the stage area is reused (bounded waits).
-    for (int s = max(consumed, issued - n_bufs); s < issued; ++s)
-      mbar_wait(&full[s % n_bufs], (s / n_bufs) & 1);
-  }
-  __syncthreads();
-
-  tc_write_state<true, BV>(st, ma, warp, lane);
-}
-
 // ---------------------------------------------------------------------------
-// Tensor-core path for the fp16 residual window: each consumer warp stages a
-// 32-token chunk of K and V rows in shared memory and feeds the MMAs with
-// ldmatrix (keys as A with tokens as rows; values transposed, channels as
-// rows).  Rows past the window are zero and their scores -inf.
+// Tensor-core path for the fp16 residual window: a warp stages the K rows of
+// a 32-token chunk in shared memory, scores them with ldmatrix-fed MMAs
+// (keys as A with tokens as rows), then stages the V rows in the same place
+// (values transposed, channels as rows).  Rows past the window are zero and
+// their scores -inf.
 // ---------------------------------------------------------------------------
 
-constexpr int kResRow = kHeadDim + 8;  // halves per staged row (16-byte pad)
-constexpr int kResWarpBytes = 2 * kGroup * kResRow * 2;
-static_assert(kResWarps * kResWarpBytes <= 96 * 1024, "window staging fits");
+constexpr int kResRow = kHeadDim + 8;                    // halves per staged row (16-byte pad)
+constexpr int kResRowsBytes = kGroup * kResRow * 2;      // one 32-row K or V chunk
 
 __device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_addr(p)));
+               : "r"(smem_addr(p))
+               : "memory");
 }
 __device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_addr(p)));
+               : "r"(smem_addr(p))
+               : "memory");
+}
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(dst)), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
 }
 
-__device__ __forceinline__ void tc_resid_chunk(const __half* ks_s, const __half* vs_s, int n_tok,
-                                               const uint32_t (&qb)[16], const Lane& ln,
-                                               float scale_log2, TcState& st) {
+// Copy rows p0 .. p0 + 31 of one (sequence, kv-head) ring (fp16 [ring][128])
+// into `rows` ([32][kResRow]); rows at or past n_tok are zero-filled.
+__device__ __forceinline__ void stage_rows(__half* rows, const __half* ring_base, int p0, int n_tok,
+                                           int ring) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll 4
+  for (int e = lane; e < kGroup * 16; e += 32) {
+    const int row = e >> 4, piece = e & 15;
+    const bool ok = row < n_tok;
+    const long long off = ok ? (long long)((p0 + row) % ring) * kHeadDim : 0;
+    cp_async16(rows + row * kResRow + piece * 8, ring_base + off + piece * 8, ok ? 16u : 0u);
+  }
+  cp_async_wait_all();
+  __syncwarp();
+}
+
+__device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
+                                                const uint32_t (&qb)[16], const Lane& ln,
+                                                float scale_log2, TcState& st,
+                                                uint32_t (&pt)[1][2][2]) {
   const int lane = threadIdx.x & 31;
   const int mi = lane >> 3, r8 = lane & 7;
   float dk[2][4] = {};
@@ -844,7 +746,7 @@ __device__ __forceinline__ void tc_resid_chunk(const __half* ks_s, const __half*
       ldsm_x4(a, ks_s + (16 * mt + 8 * (mi & 1) + r8) * kResRow + 16 * ks + 8 * (mi >> 1));
       mma16816(dk[mt], a[0], a[1], a[2], a[3], qb[2 * ks], qb[2 * ks + 1]);
     }
-  float sc[4][2];
+  float sc[1][4][2];
 #pragma unroll
   for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
@@ -852,16 +754,15 @@ __device__ __forceinline__ void tc_resid_chunk(const __half* ks_s, const __half*
       const bool ok = 16 * mt + ln.gid + 8 * rh < n_tok;
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh)
-        sc[2 * mt + rh][hh] = ok ? dk[mt][2 * rh + hh] * scale_log2 : -INFINITY;
+        sc[0][2 * mt + rh][hh] = ok ? dk[mt][2 * rh + hh] * scale_log2 : -INFINITY;
     }
-  float sc1[1][4][2];
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    sc1[0][j][0] = sc[j][0];
-    sc1[0][j][1] = sc[j][1];
-  }
-  uint32_t pt[1][2][2];
-  tc_softmax<1>(sc1, st, ln, pt);
+  tc_softmax<1>(sc, st, ln, pt);
+}
+
+__device__ __forceinline__ void tc_resid_values(const __half* vs_s, const uint32_t (&pt)[1][2][2],
+                                                TcState& st) {
+  const int lane = threadIdx.x & 31;
+  const int mi = lane >> 3, r8 = lane & 7;
 #pragma unroll
   for (int ks = 0; ks < 2; ++ks)
 #pragma unroll
@@ -872,47 +773,165 @@ __device__ __forceinline__ void tc_resid_chunk(const __half* ks_s, const __half*
     }
 }
 
-__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(dst)), "l"(src),
-               "r"(src_bytes)
-               : "memory");
+// ---------------------------------------------------------------------------
+// Work of one (sequence, kv-head): nb packed blocks and n_res window chunks
+// over NV warps.  The last n_resw warps take the window chunks (strided), the
+// other np warps contiguous block ranges whose sizes differ by at most one.
+// ---------------------------------------------------------------------------
+
+struct Plan {
+  int Lq, nb, n_res, n_resw, np;
+};
+
+__host__ __device__ inline Plan make_plan(int L, int residual, int NV) {
+  Plan p;
+  p.Lq = packed_len(L, residual);
+  p.nb = p.Lq / kGroup;
+  p.n_res = (L - p.Lq + kGroup - 1) / kGroup;
+  const int cap = p.nb == 0 ? NV : (NV / 4 > 1 ? NV / 4 : 1);
+  p.n_resw = p.n_res < cap ? p.n_res : cap;
+  p.np = NV - p.n_resw;
+  return p;
 }
 
-// Residual split: tokens [Lq, L) of one (sequence, kv-head), fp16, from the
-// ring.  Warp w takes 32-token chunks w, w + kResWarps, ...; each chunk's K
-// and V rows are copied into shared memory with asynchronous 16-byte copies
-// (rows past L are zero-filled) before its MMAs.
+// Blocks [lo, hi) of packed warp v (v < np).
+__host__ __device__ inline void block_range(const Plan& p, int v, int& lo, int& hi) {
+  lo = (int)((long long)v * p.nb / p.np);
+  hi = (int)((long long)(v + 1) * p.nb / p.np);
+}
+
+// Blocks per ring slot and slots per warp for a page size.
+__host__ __device__ constexpr int ring_blocks(int page) { return page <= 3072 ? 2 : 1; }
+__host__ __device__ constexpr int ring_slots(int page) {
+  return kRingBudget / (kWarps * ring_blocks(page) * page) < 1   ? 1
+         : kRingBudget / (kWarps * ring_blocks(page) * page) > 4 ? 4
+                                                                 : kRingBudget / (kWarps * ring_blocks(page) * page);
+}
+// A warp's ring: its slots, and at least one 32-row K (or V) chunk of the
+// window, which a window warp stages there.
+__host__ __device__ constexpr int warp_ring_bytes(int page) {
+  return ((ring_slots(page) * ring_blocks(page) * page > kResRowsBytes
+               ? ring_slots(page) * ring_blocks(page) * page
+               : kResRowsBytes) +
+          127) / 128 * 128;
+}
+static_assert(kWarps * warp_ring_bytes(page_bytes_c(4, 8)) <= kRingBudget + 8 * 1024, "rings fit");
+
+// Packed warps stream their blocks through a private ring of slots.  A page
+// is written once, when its group leaves the window, and never changes
+// afterwards, so before waiting for the previous kernel (programmatic
+// dependent launch) lane 0 already streams the full slots of the range that
+// a length read before the wait gives (tc_pre_issue).  If the range after the
+// wait starts elsewhere those slots are consumed without use.
 template <int BK, int BV>
-__device__ void tc_resid_split(const Dims& d, const __half* ring_k, const __half* ring_v, int Lq,
-                               int L, unsigned char* smem, const __half* qh, int gq,
-                               float scale_log2, MergeArea& ma) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_res = (L - Lq + kGroup - 1) / kGroup;
-  TcState st;
+__device__ __forceinline__ void issue_slot(const char* pages_bh, char* ring, uint64_t* full, int R,
+                                           int s, int first, int nblk) {
+  constexpr int page = page_bytes_c(BK, BV);
+  constexpr int NB = ring_blocks(page);
+  uint64_t* bar = full + s % R;
+  const uint32_t bytes = (uint32_t)(nblk * page);
+  mbar_expect_tx(bar, bytes);
+  bulk_g2s(ring + (size_t)(s % R) * NB * page, pages_bh + (long long)first * page, bytes, bar);
+}
+
+template <int BK, int BV>
+__device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int hi_h, char* ring,
+                                            uint64_t* full, int R) {
+  constexpr int NB = ring_blocks(page_bytes_c(BK, BV));
+  const int pre = min(R, (hi_h - lo_h) / NB);
+  if ((threadIdx.x & 31) == 0)
+    for (int s = 0; s < pre; ++s) issue_slot<BK, BV>(pages_bh, ring, full, R, s, lo_h + s * NB, NB);
+  return pre;
+}
+
+// Fold blocks [lo, hi) into st; `pre` slots were streamed early for a range
+// starting at lo_h.
+template <int BK, int BV>
+__device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, int hi,
+                               char* ring, uint64_t* full, int R, const char* zero,
+                               const __half* qh, int gq, float scale_log2, unsigned* flag,
+                               TcState& st) {
+  constexpr int page = page_bytes_c(BK, BV);
+  constexpr int NB = ring_blocks(page);
+  const int lane = threadIdx.x & 31;
+  const int skip = (pre > 0 && lo == lo_h) ? 0 : pre;
+  const int n_units = (hi - lo + NB - 1) / NB;
+  const int total = skip + n_units;
+  int issued = pre;  // lane 0's count of issued slots
+  auto real_issue = [&](int s) {
+    const int u = s - skip;
+    issue_slot<BK, BV>(pages_bh, ring, full, R, s, lo + u * NB, min(NB, hi - lo - u * NB));
+    issued = s + 1;
+  };
+  if (lane == 0)
+    for (int s = pre; s < min(total, R); ++s) real_issue(s);
+
+  const Lane ln = make_lane<BK, BV>(lane);
+  uint32_t qb[16];
+  load_qb<true>(qb, qh, gq, ln);
+  int consumed = 0;
+  for (int s = 0; s < total; ++s) {
+    const int slot = s % R;
+    // every lane waits; the warp leaves together if any lane gave up
+    if (!__all_sync(0xffffffffu, mbar_wait(full + slot, (s / R) & 1))) {
+      if (lane == 0) atomicOr(flag, 2u);
+      break;
+    }
+    consumed = s + 1;
+    if (s >= skip) {
+      const int u = s - skip;
+      const char* base = ring + (size_t)slot * NB * page;
+      if (lo + u * NB + NB <= hi) {
+        const char* pg[NB];
+#pragma unroll
+        for (int i = 0; i < NB; ++i) pg[i] = base + i * page;
+        tc_unit<BK, BV, NB>(pg, zero, qb, ln, scale_log2, st);
+      } else {
+        const char* pg[1] = {base};
+        tc_unit<BK, BV, 1>(pg, zero, qb, ln, scale_log2, st);
+      }
+    }
+    __syncwarp();
+    if (lane == 0 && s + R < total) {
+      // this warp's reads of the slot precede the copy that overwrites it
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      real_issue(s + R);
+    }
+  }
+  // Copies issued but not consumed (a wait gave up, or the range shrank) land
+  // before the ring is reused; bounded waits.
+  if (lane == 0)
+    for (int s = max(consumed, issued - R); s < issued; ++s) mbar_wait(full + s % R, (s / R) & 1);
+  __syncwarp();
+}
+
+// Window warp: chunks c0, c0 + stride, ... of the fp16 window.
+template <int BK, int BV>
+__device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half* ring_v,
+                               const Plan& p, int L, int c0, int stride, char* area,
+                               const __half* qh, int gq, float scale_log2, TcState& st) {
+  const int lane = threadIdx.x & 31;
   const Lane ln = make_lane<BK, BV>(lane);
   uint32_t qb[16];
   load_qb<false>(qb, qh, gq, ln);
-  init_state(st);
-  __half* ks_s = reinterpret_cast<__half*>(smem + (size_t)warp * kResWarpBytes);
-  __half* vs_s = ks_s + kGroup * kResRow;
-  for (int u = warp; u < n_res; u += kResWarps) {
-    const int p0 = Lq + u * kGroup;
+  __half* rows = reinterpret_cast<__half*>(area);
+  for (int u = c0; u < p.n_res; u += stride) {
+    const int p0 = p.Lq + u * kGroup;
     const int n_tok = min(kGroup, L - p0);
-#pragma unroll 4
-    for (int e = lane; e < kGroup * 16; e += 32) {
-      const int row = e >> 4, piece = e & 15;
-      const bool ok = row < n_tok;
-      const long long off = ok ? (long long)((p0 + row) % d.ring) * kHeadDim : 0;
-      cp_async16(ks_s + row * kResRow + piece * 8, ring_k + off + piece * 8, ok ? 16u : 0u);
-      cp_async16(vs_s + row * kResRow + piece * 8, ring_v + off + piece * 8, ok ? 16u : 0u);
-    }
-    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+    uint32_t pt[1][2][2];
+    stage_rows(rows, ring_k, p0, n_tok, d.ring);
+    tc_resid_scores(rows, n_tok, qb, ln, scale_log2, st, pt);
     __syncwarp();
-    tc_resid_chunk(ks_s, vs_s, n_tok, qb, ln, scale_log2, st);
+    stage_rows(rows, ring_v, p0, n_tok, d.ring);
+    tc_resid_values(rows, pt, st);
     __syncwarp();
   }
-  __syncthreads();  // staging area free: the merge area overlaps it
-  tc_write_state<false, BV>(st, ma, warp, lane);
+}
+
+__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
+  unsigned old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
 }
 
 // ---------------------------------------------------------------------------
@@ -922,12 +941,14 @@ __device__ void tc_resid_split(const Dims& d, const __half* ring_k, const __half
 template <int BK, int BV, bool kTc>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     decode_attn_kernel(Dims d, kvq_cache c, const __half* __restrict__ q, float* __restrict__ out,
-                       float scale_log2, int S, int n_bufs, unsigned smem_size, Ws ws) {
+                       float scale_log2, int S, unsigned smem_size, Ws ws) {
   extern __shared__ __align__(128) unsigned char smem[];
-  MergeArea& ma = *reinterpret_cast<MergeArea*>(smem);
+  __shared__ MergeSmall ms;
 
-  const int s = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int h = blockIdx.y, b = blockIdx.z;
   const int gq = d.gq, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int NV = gridDim.x * kWarps;     // warps per (sequence, kv-head)
+  const int v = blockIdx.x * kWarps + warp;
   pdl_launch_dependents();
   const long long bh = (long long)b * d.hkv + h;
   const char* pages = static_cast<const char*>(c.pages) + bh * d.max_blocks * d.page_bytes;
@@ -936,101 +957,150 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   const __half* qh = q + ((long long)b * d.hq + (long long)h * gq) * kHeadDim;
   unsigned* flag = reinterpret_cast<unsigned*>(c.seq_len) + d.batch;
 
-  if (kTc && s < S - 1) {
-    tc_split<BK, BV>(d, pages, s, S - 1, c.seq_len + b, n_bufs, smem, qh, gq, scale_log2, flag,
-                     ma);
-  } else {
+  if constexpr (kTc) {
+    constexpr int page = page_bytes_c(BK, BV);
+    const int R = ring_slots(page);
+    const int wbytes = warp_ring_bytes(page);
+    char* ring = reinterpret_cast<char*>(smem) + (size_t)warp * wbytes;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kWarps * wbytes) + warp * R;
+    // 512 zero bytes at the end of shared memory: metadata rows of the
+    // zero-point MMAs that carry no block.
+    unsigned* zero = reinterpret_cast<unsigned*>(smem + smem_size - 16 - kZeroBytes);
+    for (int i = threadIdx.x; i < kZeroBytes / 4; i += kThreads) zero[i] = 0u;
+    int hint = 0;
+    if (lane == 0) {
+      for (int i = 0; i < R; ++i) mbar_init(full + i, 1);
+      fence_mbar_init();
+      hint = read_len(c.seq_len + b);
+    }
+    hint = __shfl_sync(0xffffffffu, hint, 0);
+    __syncwarp();
+    const Plan ph = make_plan(hint, d.residual, NV);
+    int lo_h = 0, hi_h = 0, pre = 0;
+    if (v < ph.np) {
+      block_range(ph, v, lo_h, hi_h);
+      pre = tc_pre_issue<BK, BV>(pages, lo_h, hi_h, ring, full, R);
+    }
+    __syncthreads();  // zero rows written
     pdl_wait();
-  }
-  const int L = read_len(c.seq_len + b);
-  const int Lq = packed_len(L, d.residual);
-  const int nb = Lq / kGroup;
-  if (kTc && s < S - 1) {
-  } else if (kTc) {
-    tc_resid_split<BK, BV>(d, ring_k, ring_v, Lq, L, smem, qh, gq, scale_log2, ma);
+    // q (written by the previous kernel) into L1 while the length is read
+    if (lane < gq * 2) asm volatile("prefetch.global.L1 [%0];" ::"l"(qh + lane * 64));
+    const int L = read_len(c.seq_len + b);
+    const Plan p = make_plan(L, d.residual, NV);
+    const bool packed = v < p.np;
+    TcState st;
+    init_state(st);
+    if (packed || pre > 0) {
+      // a warp that streamed early retires its slots even if it now has no blocks
+      int lo = 0, hi = 0;
+      if (packed) block_range(p, v, lo, hi);
+      tc_packed_warp<BK, BV>(pages, lo_h, pre, lo, hi, ring, full, R,
+                             reinterpret_cast<const char*>(zero), qh, gq, scale_log2, flag, st);
+    }
+    if (!packed)
+      tc_window_warp<BK, BV>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, qh, gq,
+                             scale_log2, st);
+    // the warp's ring is idle now: its state goes to the start of it
+    WarpState& mine = *reinterpret_cast<WarpState*>(ring);
+    if (packed) tc_write_state<true, BV>(st, mine, lane);
+    else tc_write_state<false, BV>(st, mine, lane);
   } else {
-    // SIMT path: every unit, split evenly (query groups wider than 4).
-    const int units = nb + (L - Lq + kGroup - 1) / kGroup;
-    const int per = (units + S - 1) / S;
-    const int u0 = min(units, s * per), u1 = min(units, u0 + per);
+    // SIMT path: every unit (packed blocks, then window chunks) in contiguous
+    // ranges over all warps (query groups wider than 4).
+    pdl_wait();
+    const int L = read_len(c.seq_len + b);
+    const Plan p = make_plan(L, d.residual, NV);
+    const int units = p.nb + p.n_res;
+    const int u0 = (int)((long long)v * units / NV), u1 = (int)((long long)(v + 1) * units / NV);
+    float (*qs)[kHeadDim] =
+        reinterpret_cast<float (*)[kHeadDim]>(smem + (size_t)kWarps * sizeof(WarpState));
     for (int e = threadIdx.x; e < gq * kHeadDim; e += kThreads)
-      ma.qs[e / kHeadDim][e % kHeadDim] = __half2float(qh[e]) * scale_log2;
+      qs[e / kHeadDim][e % kHeadDim] = __half2float(qh[e]) * scale_log2;
     __syncthreads();
-    if (warp < kConsumers) {
-      State st;
+    State st;
 #pragma unroll
-      for (int g = 0; g < kMaxGq; ++g) {
-        st.m[g] = -INFINITY;
-        st.l[g] = 0.0f;
+    for (int g = 0; g < kMaxGq; ++g) {
+      st.m[g] = -INFINITY;
+      st.l[g] = 0.0f;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) st.acc[g][i] = 0.0f;
+      for (int i = 0; i < 4; ++i) st.acc[g][i] = 0.0f;
+    }
+    for (int u = u0; u < u1; ++u) {
+      if (u < p.nb) {
+        simt_packed_unit<BK, BV>(st, qs, gq, pages + (long long)u * d.page_bytes);
+      } else {
+        const int p0 = p.Lq + (u - p.nb) * kGroup;
+        simt_resid_unit(st, qs, gq, ring_k, ring_v, p0, min(kGroup, L - p0), d.ring);
       }
-      for (int u = u0 + warp; u < u1; u += kConsumers) {
-        if (u < nb) {
-          simt_packed_unit<BK, BV>(st, ma.qs, gq, pages + (long long)u * d.page_bytes);
-        } else {
-          const int p0 = Lq + (u - nb) * kGroup;
-          simt_resid_unit(st, ma.qs, gq, ring_k, ring_v, p0, min(kGroup, L - p0), d.ring);
-        }
+    }
+    WarpState& mine = *reinterpret_cast<WarpState*>(smem + (size_t)warp * sizeof(WarpState));
+#pragma unroll
+    for (int g = 0; g < kMaxGq; ++g) {
+      if (g >= gq) break;
+      if (lane == 0) {
+        mine.m[g] = st.m[g];
+        mine.l[g] = st.l[g];
       }
 #pragma unroll
-      for (int g = 0; g < kMaxGq; ++g) {
-        if (g >= gq) break;
-        if (lane == 0) {
-          ma.wm[warp][g] = st.m[g];
-          ma.wl[warp][g] = st.l[g];
-        }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) ma.wo[warp][g][4 * lane + i] = st.acc[g][i];
-      }
+      for (int i = 0; i < 4; ++i) mine.o[g][4 * lane + i] = st.acc[g][i];
     }
   }
   __syncthreads();
 
-  // Merge the consumer warps and publish this split's partials.
-  const int cidx = threadIdx.x;  // one output channel per thread (threads 0..127)
-  if (cidx < kHeadDim) {
-    for (int g = 0; g < gq; ++g) {
-      float M = -INFINITY;
-      for (int w = 0; w < kConsumers; ++w) M = fmaxf(M, ma.wm[w][g]);
-      float l = 0.0f, o = 0.0f;
-      if (M != -INFINITY) {
-        for (int w = 0; w < kConsumers; ++w) {
-          const float f = exp2f(ma.wm[w][g] - M);
-          l += f * ma.wl[w][g];
-          o += f * ma.wo[w][g][cidx];
-        }
-      }
-      const long long row = ((long long)b * d.hq + (long long)h * gq + g) * S + s;
-      ws.o[row * kHeadDim + cidx] = o;
-      if (cidx == 0) {
-        ws.m[row] = M;
+  // ---- merge the warps of this CTA: one partial per query head ----
+  const size_t wstride = kTc ? (size_t)warp_ring_bytes(page_bytes_c(BK, BV)) : sizeof(WarpState);
+  auto wstate = [&](int w) -> const WarpState& {
+    return *reinterpret_cast<const WarpState*>(smem + (size_t)w * wstride);
+  };
+  if (threadIdx.x < kWarps * gq) {
+    const int w = threadIdx.x / gq, g = threadIdx.x % gq;
+    float M = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < kWarps; ++i) M = fmaxf(M, wstate(i).m[g]);
+    const float m = wstate(w).m[g];
+    ms.ww[w][g] = (m == -INFINITY) ? 0.0f : exp2f(m - M);
+    if (w == 0) ms.cta_m[g] = M;
+  }
+  __syncthreads();
+  const int n_items = gq * kHeadDim;
+  const long long head0 = (long long)b * d.hq + (long long)h * gq;
+  for (int it = threadIdx.x; it < n_items; it += kThreads) {
+    const int g = it / kHeadDim, ch = it % kHeadDim;
+    float o = 0.0f, l = 0.0f;
+#pragma unroll
+    for (int i = 0; i < kWarps; ++i) {
+      const float w = ms.ww[i][g];
+      o = fmaf(w, wstate(i).o[g][ch], o);
+      l = fmaf(w, wstate(i).l[g], l);
+    }
+    if (S == 1) {
+      out[(head0 + g) * kHeadDim + ch] = l > 0.0f ? o / l : 0.0f;
+    } else {
+      const long long row = (head0 + g) * S + blockIdx.x;
+      ws.o[row * kHeadDim + ch] = o;
+      if (ch == 0) {
+        ws.m[row] = ms.cta_m[g];
         ws.l[row] = l;
       }
     }
   }
+  if (S == 1) return;
+
+  // ---- the last CTA of this (sequence, kv-head) merges the S partials ----
   __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    const unsigned t = atomicAdd(&ws.tk[bh], 1u);
-    ma.last = (t == (unsigned)S - 1);
-  }
+  if (threadIdx.x == 0) ms.last = atom_add_acq_rel(&ws.tk[bh], 1u) == (unsigned)S - 1;
   __syncthreads();
-  const bool is_last = ma.last;
-  __syncthreads();  // the merge below reuses the shared memory that holds `last`
-  if (!is_last) return;
-  __threadfence();
-  // Last CTA: merge the S partials of every query head.  The partial rows of
-  // this (sequence, kv-head) are one contiguous range: one bulk copy brings
-  // them into shared memory when they fit, while the maxima and sums are
-  // loaded; each thread then reduces one (head, 4-channel) slice.
-  const long long head0 = (long long)b * d.hq + (long long)h * gq;
+  if (!ms.last) return;
+  // The partial rows of this (sequence, kv-head) are one contiguous range: a
+  // bulk copy brings them into shared memory (when they fit) while the maxima
+  // and sums are loaded and turned into weights.
   const size_t o_bytes = (size_t)gq * S * kHeadDim * sizeof(float);
-  const bool staged = o_bytes + (size_t)(2 * gq * S + gq) * sizeof(float) + 16 <= smem_size;
-  float* osm = reinterpret_cast<float*>(smem);
-  float* mv = staged ? osm + (size_t)gq * S * kHeadDim : osm;  // [gq][S] maxima, then weights
-  float* lv = mv + gq * S;                                      // [gq][S] sums
-  float* lsum = lv + gq * S;                                    // [gq]
+  float* wv = reinterpret_cast<float*>(smem);           // [gq][S] maxima, then weights
+  float* lv = wv + gq * S;                               // [gq][S] sums
+  float* lsum = lv + gq * S;                             // [gq]
+  float* osm = lsum + 16;                                // [gq][S][128]
+  const size_t head_bytes = (size_t)(2 * gq * S + 16) * sizeof(float);
+  const bool staged = head_bytes + o_bytes + 16 <= smem_size;
   uint64_t* mbar = reinterpret_cast<uint64_t*>(smem + smem_size - 16);
   if (staged && threadIdx.x == 0) {
     mbar_init(mbar, 1);
@@ -1040,20 +1110,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     bulk_g2s(osm, ws.o + head0 * S * kHeadDim, (uint32_t)o_bytes, mbar);
   }
   for (int i = threadIdx.x; i < gq * S; i += kThreads) {
-    mv[i] = __ldcg(ws.m + head0 * S + i);
+    wv[i] = __ldcg(ws.m + head0 * S + i);
     lv[i] = __ldcg(ws.l + head0 * S + i);
   }
   __syncthreads();
-  for (int g = warp; g < gq; g += kThreads / 32) {
+  for (int g = warp; g < gq; g += kWarps) {
     float M = -INFINITY;
-    for (int k = lane; k < S; k += 32) M = fmaxf(M, mv[g * S + k]);
+    for (int k = lane; k < S; k += 32) M = fmaxf(M, wv[g * S + k]);
     M = warp_max(M);
     float Ls = 0.0f;
     for (int k = lane; k < S; k += 32) {
-      const float m = mv[g * S + k];
+      const float m = wv[g * S + k];
       const float w = (m == -INFINITY) ? 0.0f : exp2f(m - M);
       Ls += w * lv[g * S + k];
-      mv[g * S + k] = w;
+      wv[g * S + k] = w;
     }
     Ls = warp_sum(Ls);
     if (lane == 0) lsum[g] = Ls;
@@ -1061,51 +1131,35 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   bool ok = true;
   if (staged) ok = mbar_wait(mbar, 0);
   __syncthreads();
-  for (int i = threadIdx.x; i < gq * (kHeadDim / 4); i += kThreads) {
-    const int g = i / (kHeadDim / 4), c4 = i % (kHeadDim / 4);
-    const float4* src = staged && ok
-                            ? reinterpret_cast<const float4*>(osm + (size_t)g * S * kHeadDim) + c4
-                            : reinterpret_cast<const float4*>(ws.o + (head0 + g) * S * kHeadDim) + c4;
-    float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  for (int it = threadIdx.x; it < n_items; it += kThreads) {
+    const int g = it / kHeadDim, ch = it % kHeadDim;
+    float o = 0.0f;
+    if (staged && ok) {
+      const float* src = osm + (size_t)g * S * kHeadDim + ch;
 #pragma unroll 8
-    for (int k = 0; k < S; ++k) {
-      const float w = mv[g * S + k];
-      const float4 o = staged && ok ? src[(long long)k * (kHeadDim / 4)]
-                                    : __ldcg(src + (long long)k * (kHeadDim / 4));
-      acc.x = fmaf(w, o.x, acc.x);
-      acc.y = fmaf(w, o.y, acc.y);
-      acc.z = fmaf(w, o.z, acc.z);
-      acc.w = fmaf(w, o.w, acc.w);
+      for (int k = 0; k < S; ++k) o = fmaf(wv[g * S + k], src[(size_t)k * kHeadDim], o);
+    } else {
+      const float* src = ws.o + (head0 + g) * S * kHeadDim + ch;
+#pragma unroll 8
+      for (int k = 0; k < S; ++k) o = fmaf(wv[g * S + k], __ldcg(src + (size_t)k * kHeadDim), o);
     }
     const float Ls = lsum[g];
-    const float inv = Ls > 0.0f ? 1.0f / Ls : 0.0f;
-    reinterpret_cast<float4*>(out + (head0 + g) * kHeadDim)[c4] =
-        make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+    out[(head0 + g) * kHeadDim + ch] = Ls > 0.0f ? o / Ls : 0.0f;
   }
   if (threadIdx.x == 0) ws.tk[bh] = 0u;
 }
 
-int blocks_per_warp(const Dims& d) {
-  return (kUnitBlocks > 1 && d.page_bytes <= 6144) ? kUnitBlocks : 1;
-}
-
-int stage_buffers(const Dims& d) {
-  const int stage = kConsumers * blocks_per_warp(d) * (int)d.page_bytes;
-  int n = kStageBudget / stage;
-  return n < 2 ? 2 : (n > 8 ? 8 : n);
-}
-
 size_t smem_bytes(const Dims& d, bool tc) {
-  size_t need = sizeof(MergeArea);
-  const size_t merge = (size_t)(2 * kMaxGq * kMaxSplits + kMaxGq) * sizeof(float);
-  if (need < merge) need = merge;
-  if (tc && need < (size_t)kResWarps * kResWarpBytes) need = (size_t)kResWarps * kResWarpBytes;
+  // SIMT path: warp states, then q * scale
+  size_t need = (size_t)kWarps * sizeof(WarpState) + sizeof(float) * kMaxGq * kHeadDim;
   if (tc) {
-    const size_t stages = (size_t)stage_buffers(d) * kConsumers * blocks_per_warp(d) * d.page_bytes +
-                          16 * stage_buffers(d);
-    if (stages > need) need = stages;
+    const int page = (int)d.page_bytes;
+    const size_t rings = (size_t)kWarps * warp_ring_bytes(page) +
+                         (size_t)kWarps * ring_slots(page) * sizeof(uint64_t);
+    if (rings > need) need = rings;
   }
-  return (need + 16 + 127) / 128 * 128;  // + the final merge's mbarrier
+  // + the zero rows of the packed warps and the final merge's mbarrier
+  return (need + kZeroBytes + 16 + 127) / 128 * 128;
 }
 
 template <int BK, int BV, bool kTc>
@@ -1115,9 +1169,6 @@ cudaError_t prepare(const Dims& d) {
 }
 
 // Kernel instance for (bits_k, bits_v, query-group width): Op::run<BK, BV, kTc>.
-template <typename Op>
-cudaError_t dispatch(const Dims& d, const Op& op);
-
 template <int BK, int BV, typename Op>
 cudaError_t dispatch_mode(const Dims& d, const Op& op) {
   return d.gq <= 4 ? op.template run<BK, BV, true>() : op.template run<BK, BV, false>();
@@ -1165,28 +1216,15 @@ struct LaunchOp {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV, kTc>, d, c, q, out, sl2, S,
-                           stage_buffers(d), (unsigned)smem_bytes(d, kTc), ws);
+                           (unsigned)smem_bytes(d, kTc), ws);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
 };
 
-struct OccupancyOp {
-  const Dims& d;
-  int* blocks;
-  template <int BK, int BV, bool kTc>
-  cudaError_t run() const {
-    cudaError_t e = prepare<BK, BV, kTc>(d);
-    if (e != cudaSuccess) return e;
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, decode_attn_kernel<BK, BV, kTc>,
-                                                         kThreads, smem_bytes(d, kTc));
-  }
-};
-
 }  // namespace
 
-// n_splits counts the packed-block splits; the kernel adds one split for the
-// residual window.
+// n_splits = CTAs per (sequence, kv-head); workspace rows for up to n_splits.
 size_t attn_workspace_bytes(const Dims& d, int n_splits) {
   const int S = n_splits + 1;
   const size_t nml = (size_t)d.batch * d.hq * S;
@@ -1196,26 +1234,19 @@ size_t attn_workspace_bytes(const Dims& d, int n_splits) {
 
 cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& c, const __half* q, float* out,
                                float scale_log2, int n_splits, void* workspace, cudaStream_t st) {
-  const int S = n_splits + 1;
-  const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, S);
-  return dispatch(d, LaunchOp{d, c, q, out, scale_log2, S, ws, st});
+  const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, n_splits);
+  return dispatch(d, LaunchOp{d, c, q, out, scale_log2, n_splits, ws, st});
 }
 
-// Packed splits per (sequence, kv-head) so that all CTAs (packed splits plus
-// the window split) are resident at once; at least ~16 blocks per split.
+// CTAs per (sequence, kv-head): enough for every resident CTA slot of the
+// GPU to hold one, with at least a few blocks per CTA.
 int attn_default_splits(const Dims& d, int sm_count) {
-  int occ = 0;
-  if (dispatch(d, OccupancyOp{d, &occ}) != cudaSuccess || occ < 1) {
-    cudaGetLastError();
-    occ = 1;
-  }
   const int bh = d.batch * d.hkv;
-  int n = occ * sm_count / bh - 1;
-  const int cap = (d.max_blocks + 15) / 16;
+  int n = kCtasPerSm * sm_count / bh;
+  const int cap = (d.max_blocks + 3) / 4;
   if (n > cap) n = cap;
   if (n > kMaxSplits - 1) n = kMaxSplits - 1;
-  if (n < 1) n = 1;
-  return n;
+  return n < 1 ? 1 : n;
 }
 
 // ---------------------------------------------------------------------------
@@ -1267,7 +1298,7 @@ cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& c, const _
   if (e != cudaSuccess) return e;
   // The array keeps the previous call's contents: the tickets must start at
   // zero, the partials are always written before they are read.
-  const Ws w = carve(ws, d.batch, d.hq, d.hkv, n_splits + 1);
+  const Ws w = carve(ws, d.batch, d.hq, d.hkv, n_splits);
   e = cudaMemsetAsync(w.tk, 0, (size_t)d.batch * d.hkv * sizeof(unsigned), st);
   if (e != cudaSuccess) return e;
   return launch_decode_attn(d, c, q, out, scale_log2, n_splits, ws, st);

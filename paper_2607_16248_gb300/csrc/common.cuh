@@ -30,6 +30,30 @@ __host__ __device__ inline int page_off_vmeta(int bits_k, int bits_v) {
   return 512 * (bits_k + bits_v) + 512;
 }
 
+// Positions inside a page (layouts documented in kvq.h).
+//
+// 1-bit codes are stored in mma fragment order: lane L = 4 * gid + tig of the
+// consuming warp reads its 128 codes as one 16-byte chunk (4 words) at byte
+// 16 * L, and rotating word w left by 4 * r puts the code of fragment row j
+// (j = 0..3) and half e at bit 10 + 16 e + j.  Keys: token t = 4 gid + j,
+// channel c = 16 ks + 4 tig + 2 h + e, word ks / 2, r = 2 (ks & 1) + h.
+// Values: channel c = 32 w + 4 gid + j, token t = 8 tig + r + 4 e.
+// The functions return the bit index inside the 512-byte code area.
+__host__ __device__ inline int key1_bit(int t, int c) {
+  const int gid = t >> 2, j = t & 3, ks = c >> 4, tig = (c >> 2) & 3;
+  const int h = (c >> 1) & 1, e = c & 1, r = 2 * (ks & 1) + h;
+  return (16 * gid + 4 * tig + (ks >> 1)) * 32 + ((10 + 16 * e + j - 4 * r) & 31);
+}
+__host__ __device__ inline int val1_bit(int t, int c) {
+  const int w = c >> 5, gid = (c >> 2) & 7, j = c & 3, tig = t >> 3, r = t & 3, e = (t >> 2) & 1;
+  return (16 * gid + 4 * tig + w) * 32 + ((10 + 16 * e + j - 4 * r) & 31);
+}
+// Value scale / zero of (group g, token t): tokens of each 8-token run are
+// stored in the order 0 4 1 5 2 6 3 7, so a 32-bit word holds tokens (t, t + 4).
+__host__ __device__ inline int vmeta_index(int g, int t) {
+  return 32 * g + 8 * (t >> 3) + 2 * (t & 3) + ((t >> 2) & 1);
+}
+
 // Tokens held in quantized blocks when L tokens are cached.
 __host__ __device__ inline int packed_len(int L, int residual) {
   int over = L - residual;

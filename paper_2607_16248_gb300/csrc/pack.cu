@@ -8,7 +8,8 @@
 //   code  = clamp(rint(RN32(RN32(x - zero) / scale)), 0, levels); 0 if scale == 0
 // Codes of a group fill b little-endian uint32 words, element i at bits
 // [(i*b) % 32, +b) of word (i*b) / 32.  Keys group 32 tokens of one channel,
-// values 32 channels of one token.
+// values 32 channels of one token.  1-bit codes are then scattered into the
+// fragment order the attention kernel reads (key1_bit / val1_bit).
 
 #include "common.cuh"
 
@@ -21,6 +22,8 @@ constexpr int kRowPad = 136;  // halves per smem row (128 + 8) to spread banks
 struct Tile {
   __half k[kGroup][kRowPad];
   __half v[kGroup][kRowPad];
+  uint32_t k1[kHeadDim];  // 1-bit key codes in fragment order
+  uint32_t v1[kHeadDim];  // 1-bit value codes in fragment order
 };
 
 // Quantize the 32 values x[] and return the packed words, scale and zero.
@@ -59,23 +62,32 @@ __device__ __forceinline__ void store_words(uint32_t* dst, const uint32_t (&w)[B
 }
 
 template <int B>
-__device__ __forceinline__ void quantize_key_channel(const Tile& t, int c, char* page, int bits_k) {
+__device__ __forceinline__ void quantize_key_channel(Tile& t, int c, char* page, int bits_k) {
   float x[kGroup];
 #pragma unroll
   for (int i = 0; i < kGroup; ++i) x[i] = __half2float(t.k[i][c]);
   uint32_t w[B];
   __half sc, z;
   quantize_group<B>(x, w, sc, z);
-  store_words<B>(reinterpret_cast<uint32_t*>(page) + c * B, w);
+  if (B == 1) {
+#pragma unroll 4
+    for (int i = 0; i < kGroup; ++i) {
+      const int bit = key1_bit(i, c);
+      if ((w[0] >> i) & 1u) atomicOr(&t.k1[bit >> 5], 1u << (bit & 31));
+    }
+  } else {
+    store_words<B>(reinterpret_cast<uint32_t*>(page) + c * B, w);
+  }
   __half* meta = reinterpret_cast<__half*>(page + page_off_kmeta(bits_k));
   meta[c] = sc;
   meta[kHeadDim + c] = z;
 }
 
-// Value groups are stored group-major: index = grp * 32 + tok; the 128
-// scales precede the 128 zeros.
+// Value codes of b >= 2 bits are stored group-major: group index
+// grp * 32 + tok.  Scales and zeros follow vmeta_index; the 128 scales
+// precede the 128 zeros.
 template <int B>
-__device__ __forceinline__ void quantize_value_group(const Tile& t, int pair, char* page,
+__device__ __forceinline__ void quantize_value_group(Tile& t, int pair, char* page,
                                                      int bits_k, int bits_v) {
   const int grp = pair >> 5, tok = pair & 31;
   float x[kGroup];
@@ -84,16 +96,29 @@ __device__ __forceinline__ void quantize_value_group(const Tile& t, int pair, ch
   uint32_t w[B];
   __half sc, z;
   quantize_group<B>(x, w, sc, z);
-  store_words<B>(reinterpret_cast<uint32_t*>(page + page_off_vcodes(bits_k)) + pair * B, w);
+  if (B == 1) {
+#pragma unroll 4
+    for (int i = 0; i < kGroup; ++i) {
+      const int bit = val1_bit(tok, grp * kGroup + i);
+      if ((w[0] >> i) & 1u) atomicOr(&t.v1[bit >> 5], 1u << (bit & 31));
+    }
+  } else {
+    store_words<B>(reinterpret_cast<uint32_t*>(page + page_off_vcodes(bits_k)) + pair * B, w);
+  }
   __half* meta = reinterpret_cast<__half*>(page + page_off_vmeta(bits_k, bits_v));
-  meta[pair] = sc;
-  meta[kHeadDim + pair] = z;
+  meta[vmeta_index(grp, tok)] = sc;
+  meta[kHeadDim + vmeta_index(grp, tok)] = z;
 }
 
 // 256 threads: 0..127 quantize one key channel each, 128..255 one
-// (32-channel group, token) value group each.
-__device__ void quantize_tile(const Tile& t, char* page, int bits_k, int bits_v) {
+// (32-channel group, token) value group each.  Called by every thread.
+__device__ void quantize_tile(Tile& t, char* page, int bits_k, int bits_v) {
   const int tid = threadIdx.x;
+  if (tid < kHeadDim) {
+    t.k1[tid] = 0u;
+    t.v1[tid] = 0u;
+  }
+  __syncthreads();
   if (tid < kHeadDim) {
     switch (bits_k) {
       case 1: quantize_key_channel<1>(t, tid, page, bits_k); break;
@@ -110,6 +135,10 @@ __device__ void quantize_tile(const Tile& t, char* page, int bits_k, int bits_v)
       default: quantize_value_group<8>(t, pair, page, bits_k, bits_v); break;
     }
   }
+  __syncthreads();
+  if (bits_k == 1 && tid < kHeadDim) reinterpret_cast<uint32_t*>(page)[tid] = t.k1[tid];
+  if (bits_v == 1 && tid >= kHeadDim)
+    reinterpret_cast<uint32_t*>(page + page_off_vcodes(bits_k))[tid - kHeadDim] = t.v1[tid - kHeadDim];
 }
 
 __device__ __forceinline__ char* page_ptr(const Dims& d, void* pages, int b, int h, int j) {
