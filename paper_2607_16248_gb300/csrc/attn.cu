@@ -838,7 +838,7 @@ template <int BK, int BV>
 __device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int hi_h, char* ring,
                                             uint64_t* full, int R) {
   constexpr int NB = ring_blocks(page_bytes_c(BK, BV));
-  const int pre = min(R, (hi_h - lo_h) / NB);
+  const int pre = hi_h > lo_h ? min(R, (hi_h - lo_h) / NB) : 0;
   if ((threadIdx.x & 31) == 0)
     for (int s = 0; s < pre; ++s) issue_slot<BK, BV>(pages_bh, ring, full, R, s, lo_h + s * NB, NB);
   return pre;
@@ -979,7 +979,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     int lo_h = 0, hi_h = 0, pre = 0;
     if (v < ph.np) {
       block_range(ph, v, lo_h, hi_h);
-      pre = tc_pre_issue<BK, BV>(pages, lo_h, hi_h, ring, full, R);
+      // the newest block may be the one the previous kernel is writing
+      pre = tc_pre_issue<BK, BV>(pages, lo_h, min(hi_h, ph.nb - 1), ring, full, R);
     }
     __syncthreads();  // zero rows written
     pdl_wait();

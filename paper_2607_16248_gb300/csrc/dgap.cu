@@ -11,6 +11,11 @@
 // sparse merge z[S_k] += Delta_k in place (Eq. 13).  Non-selected logits and
 // ungated rows are never written.
 //
+// The last CTA is latency-bound: every global read it makes is issued in one
+// round (chunk statistics and candidate lists into shared memory, the
+// corrector's first-layer weights by one bulk copy started as soon as the CTA
+// knows it is last, so the copy overlaps the merge and the detector).
+//
 // Candidates are ranked by an order-preserving uint32 key of the float
 // (-0 folded onto +0) and then by the lower index.
 
@@ -147,9 +152,19 @@ __device__ __forceinline__ void sort_desc(uint32_t (&k)[kPer], int (&ix)[kPer]) 
   }
 }
 
+constexpr int kCandStage = 4096;            // staged (key, index) candidates of a row
+constexpr size_t kW1StageMax = 176 * 1024;  // largest staged corrector W1
+
 struct Smem {
-  uint32_t sk[kPer][kT];
-  int si[kPer][kT];
+  union {
+    struct {
+      uint32_t sk[kPer][kT];
+      int si[kPer][kT];
+    } srt;                              // chunk phase
+    float w1[kW1StageMax / 4];          // finalize: corrector W1 (bulk copy)
+  } u;
+  uint2 cand[kCandStage];               // finalize: the row's candidate lists
+  uint64_t w1_bar;
   uint32_t wk[kWarpsD][kMaxK + 1];
   int wi[kWarpsD][kMaxK + 1];
   uint32_t fk[kMaxK + 1];
@@ -163,20 +178,59 @@ struct Smem {
   int last;
 };
 
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+// Whether the corrector's W1 is copied to shared memory in one bulk copy.
+__device__ __forceinline__ bool stage_w1(const DgapDims& d, const dgap_params& p) {
+  const size_t bytes = (size_t)d.hidden * (5 * d.K + 8) * sizeof(float);
+  return bytes <= kW1StageMax && bytes % 16 == 0 &&
+         (reinterpret_cast<uintptr_t>(p.cor_w1) & 15) == 0;
+}
+
 __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* logits, int row,
                              int32_t* topk_idx, float* topk_val, float* risk, uint8_t* gate,
                              int32_t* next_token, float* features, const DWs& ws, Smem& sm) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int K = d.K, K1 = d.K + 1, nc = d.n_chunks;
+  const int nin = 5 * K + 8;
   const float4* st = ws.stats + (size_t)row * nc;
 
-  // Merge the chunk statistics.
+  // The corrector's first layer, fetched while the window is formed (only
+  // used when the row is gated; always awaited before the CTA exits).
+  const bool w1s = stage_w1(d, p);
+  const uint32_t w1_bytes = (uint32_t)((size_t)d.hidden * nin * sizeof(float));
+  if (w1s && tid == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&sm.w1_bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(&sm.w1_bar)),
+                 "r"(w1_bytes)
+                 : "memory");
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_u32(sm.u.w1)),
+        "l"(p.cor_w1), "r"(w1_bytes), "r"(smem_u32(&sm.w1_bar))
+        : "memory");
+  }
+
+  // Chunk statistics and candidate lists in one round of loads.
+  const uint2* cand = ws.cand + (size_t)row * nc * K1;
+  const bool cs = nc * K1 <= kCandStage;
+  if (cs)
+    for (int i = tid; i < nc * K1; i += kT) sm.cand[i] = __ldcg(&cand[i]);
   float mloc = -INFINITY;
-  for (int c = tid; c < nc; c += kT) mloc = fmaxf(mloc, __ldcg(&st[c].x));
+  float4 sv[(kMaxChunks + kT - 1) / kT];
+#pragma unroll
+  for (int j = 0; j < (kMaxChunks + kT - 1) / kT; ++j) {
+    const int c = tid + j * kT;
+    sv[j] = c < nc ? __ldcg(&st[c]) : make_float4(-INFINITY, 0.0f, 0.0f, 0.0f);
+    mloc = fmaxf(mloc, sv[j].x);
+  }
   const float M = block_max(mloc, sm.red);
   float s1 = 0.0f, s2 = 0.0f;
-  for (int c = tid; c < nc; c += kT) {
-    const float4 v = __ldcg(&st[c]);
+#pragma unroll
+  for (int j = 0; j < (kMaxChunks + kT - 1) / kT; ++j) {
+    const float4 v = sv[j];
     if (v.y > 0.0f) {
       const float e = expf(v.x - M);
       s1 += v.y * e;
@@ -184,14 +238,13 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     }
   }
   const float S1 = block_sum(s1, sm.red);
-  const float S2 = block_sum(s2, sm.red);
+  const float S2 = block_sum(s2, sm.red);  // its barriers also publish sm.cand
 
   // Merge the chunk candidate lists: warp w takes lists w*32 + lane, then
   // warp 0 merges the eight warp results (n_chunks <= 256).
-  const uint2* cand = ws.cand + (size_t)row * nc * K1;
   const int li = warp * 32 + lane;
   warp_merge(li < nc ? K1 : 0, [&](int h, uint32_t& k, int& i) {
-    const uint2 v = __ldcg(&cand[(size_t)li * K1 + h]);
+    const uint2 v = cs ? sm.cand[li * K1 + h] : __ldcg(&cand[(size_t)li * K1 + h]);
     k = v.x;
     i = (int)v.y;
   }, K1, sm.wk[warp], sm.wi[warp]);
@@ -203,34 +256,41 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     }, K1, sm.fk, sm.fi);
   __syncthreads();
 
-  // Features phi (Sec. 4.2).
-  if (tid == 0) {
+  // Features phi (Sec. 4.2): warp 0, lanes over the window.
+  if (warp == 0) {
     const float z0 = key_value(sm.fk[0]);
-    float mass_e = 0.0f, wsum_e = 0.0f, mean = 0.0f, min_gap = INFINITY;
-    for (int k = 0; k < K; ++k) {
+    float mass_e = 0.0f, wsum_e = 0.0f, sum = 0.0f, min_gap = INFINITY;
+    for (int k = lane; k < K; k += 32) {
       const float zk = key_value(sm.fk[k]);
       const float e = expf(zk - M);
       mass_e += e;
       wsum_e += e * (zk - M);
-      mean += zk;
+      sum += zk;
       if (k + 1 < K) min_gap = fminf(min_gap, zk - key_value(sm.fk[k + 1]));
     }
-    mean /= (float)K;
+    mass_e = wsum(mass_e);
+    wsum_e = wsum(wsum_e);
+    const float mean = wsum(sum) / (float)K;
     float var = 0.0f;
-    for (int k = 0; k < K; ++k) {
+    for (int k = lane; k < K; k += 32) {
       const float dz = key_value(sm.fk[k]) - mean;
       var += dz * dz;
     }
-    var /= (float)K;
-    sm.phi[0] = logf(S1) - S2 / S1;
-    sm.phi[1] = mass_e / S1;
-    sm.phi[2] = expf(z0 - M) / S1;
-    sm.phi[3] = z0 - key_value(sm.fk[1]);
-    sm.phi[4] = (z0 - key_value(sm.fk[K - 1])) / (float)(K - 1);
-    sm.phi[5] = min_gap;
-    sm.phi[6] = sqrtf(var);
-    sm.phi[7] = logf(mass_e) - wsum_e / mass_e;
+    var = wsum(var) / (float)K;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) min_gap = fminf(min_gap, __shfl_xor_sync(0xffffffffu, min_gap, o));
+    if (lane == 0) {
+      sm.phi[0] = logf(S1) - S2 / S1;
+      sm.phi[1] = mass_e / S1;
+      sm.phi[2] = expf(z0 - M) / S1;
+      sm.phi[3] = z0 - key_value(sm.fk[1]);
+      sm.phi[4] = (z0 - key_value(sm.fk[K - 1])) / (float)(K - 1);
+      sm.phi[5] = min_gap;
+      sm.phi[6] = sqrtf(var);
+      sm.phi[7] = logf(mass_e) - wsum_e / mass_e;
+    }
   }
+  for (int k = tid; k < K; k += kT) sm.zt[k] = key_value(sm.fk[k]);
   __syncthreads();
 
   // Detector f = w2 . relu(W1 phi + b1) + b2 (Eq. 6).
@@ -244,13 +304,24 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
   const float f = block_sum(part, sm.red) + p.det_b2[0];
   const bool gated = f > d.logit_tau;
 
-  // Window values before the merge.
-  for (int k = tid; k < K; k += kT) sm.zt[k] = key_value(sm.fk[k]);
-  __syncthreads();
+  bool w1_ok = true;
+  if (w1s) {  // every thread observes the copy's completion (bounded wait)
+    const long long t0 = clock64();
+    uint32_t done = 0;
+    while (!done) {
+      asm volatile(
+          "{\n .reg .pred q;\n mbarrier.try_wait.parity.shared::cta.b64 q, [%1], 0;\n"
+          " selp.u32 %0, 1, 0, q;\n}"
+          : "=r"(done)
+          : "r"(smem_u32(&sm.w1_bar))
+          : "memory");
+      if (!done && clock64() - t0 > 4000000000LL) break;
+    }
+    w1_ok = __syncthreads_and(done != 0);
+  }
 
   if (gated) {
     // Candidate features xi (Sec. 4.3), rank-major, then phi.
-    const int nin = 5 * K + 8;
     const float lse = M + logf(S1);
     const float z0 = sm.zt[0];
     for (int k = tid; k < K; k += kT) {
@@ -264,25 +335,48 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     }
     if (tid < 8) sm.x[5 * K + tid] = sm.phi[tid];
     __syncthreads();
-    // Hidden layer: one warp per hidden unit, lanes over the inputs.
+    // Hidden layer: one warp per hidden unit, lanes over the inputs (W1 from
+    // shared memory when staged).
+    const float* w1 = (w1s && w1_ok) ? sm.u.w1 : p.cor_w1;
     for (int j = warp; j < d.hidden; j += kWarpsD) {
-      const float* wrow = p.cor_w1 + (size_t)j * nin;
+      const float* wrow = w1 + (size_t)j * nin;
       float a = 0.0f;
       for (int i = lane; i < nin; i += 32) a = fmaf(wrow[i], sm.x[i], a);
       a = wsum(a);
       if (lane == 0) sm.hb[j] = fmaxf(a + p.cor_b1[j], 0.0f);
     }
     __syncthreads();
-    // Output layer Delta_k, then the sparse merge (Eq. 13).
-    for (int k = warp; k < K; k += kWarpsD) {
-      const float* wrow = p.cor_w2 + (size_t)k * d.hidden;
-      float a = 0.0f;
-      for (int j = lane; j < d.hidden; j += 32) a = fmaf(wrow[j], sm.hb[j], a);
-      a = wsum(a);
-      if (lane == 0) {
-        const float zt = sm.zt[k] + (a + p.cor_b2[k]);
-        sm.zt[k] = zt;
-        logits[(size_t)row * d.vocab + sm.fi[k]] = zt;
+    // Output layer Delta_k (all of a warp's weight loads in one round), then
+    // the sparse merge (Eq. 13).
+    for (int k0 = warp * 4; k0 < K; k0 += kWarpsD * 4) {
+      float a[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      for (int j0 = 0; j0 < d.hidden; j0 += 256) {
+        float wv[4][8];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int t = 0; t < 8; ++t) {
+            const int j = j0 + lane + 32 * t;
+            wv[u][t] = (k0 + u < K && j < d.hidden) ? __ldg(p.cor_w2 + (size_t)(k0 + u) * d.hidden + j)
+                                                     : 0.0f;
+          }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int t = 0; t < 8; ++t) {
+            const int j = j0 + lane + 32 * t;
+            if (j < d.hidden) a[u] = fmaf(wv[u][t], sm.hb[j], a[u]);
+          }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float au = wsum(a[u]);
+        const int k = k0 + u;
+        if (lane == 0 && k < K) {
+          const float zt = sm.zt[k] + (au + p.cor_b2[k]);
+          sm.zt[k] = zt;
+          logits[(size_t)row * d.vocab + sm.fi[k]] = zt;
+        }
       }
     }
     __syncthreads();
@@ -316,6 +410,8 @@ __global__ void __launch_bounds__(kT)
                 float* features, DWs ws) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+  // programmatic dependent launch: the logits are the previous kernel's output
+  asm volatile("griddepcontrol.launch_dependents;\ngriddepcontrol.wait;" ::: "memory");
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int chunk = blockIdx.x, row = blockIdx.y, K1 = d.K + 1;
   const float* z = logits + (size_t)row * d.vocab;
@@ -356,13 +452,13 @@ __global__ void __launch_bounds__(kT)
   sort_desc(k, ix);
 #pragma unroll
   for (int i = 0; i < kPer; ++i) {
-    sm.sk[i][tid] = k[i];
-    sm.si[i][tid] = ix[i];
+    sm.u.srt.sk[i][tid] = k[i];
+    sm.u.srt.si[i][tid] = ix[i];
   }
   __syncwarp();
   warp_merge(kPer, [&](int h, uint32_t& kk, int& ii) {
-    kk = sm.sk[h][tid];
-    ii = sm.si[h][tid];
+    kk = sm.u.srt.sk[h][tid];
+    ii = sm.u.srt.si[h][tid];
   }, K1, sm.wk[warp], sm.wi[warp]);
   __syncthreads();
   uint2* out = ws.cand + ((size_t)row * d.n_chunks + chunk) * K1;
@@ -377,13 +473,12 @@ __global__ void __launch_bounds__(kT)
 
   __syncthreads();
   if (tid == 0) {
-    __threadfence();
-    const unsigned t = atomicAdd(&ws.tk[row], 1u);
+    unsigned t;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(t) : "l"(&ws.tk[row]) : "memory");
     sm.last = (t == (unsigned)d.n_chunks - 1);
   }
   __syncthreads();
   if (!sm.last) return;
-  __threadfence();
   finalize_row(d, p, logits, row, topk_idx, topk_val, risk, gate, next_token, features, ws, sm);
 }
 
@@ -403,10 +498,23 @@ cudaError_t launch_dgap(const DgapDims& d, const dgap_params& p, float* logits, 
                         float* features, void* workspace, cudaStream_t stream) {
   const DWs ws = carve(workspace, d.batch, d.n_chunks, d.K);
   const size_t smem = sizeof(Smem);
-  static_assert(sizeof(Smem) <= 48 * 1024, "DGAP shared memory must fit the default limit");
-  dim3 grid(d.n_chunks, d.batch);
-  dgap_kernel<<<grid, kT, smem, stream>>>(d, p, logits, topk_idx, topk_val, risk, gate, next_token,
-                                          features, ws);
+  static_assert(sizeof(Smem) <= 227 * 1024, "DGAP shared memory must fit one SM");
+  cudaError_t e = cudaFuncSetAttribute(dgap_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(d.n_chunks, d.batch);
+  cfg.blockDim = dim3(kT);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, dgap_kernel, d, p, logits, topk_idx, topk_val, risk, gate,
+                         next_token, features, ws);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

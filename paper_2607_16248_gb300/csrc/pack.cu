@@ -141,6 +141,12 @@ __device__ void quantize_tile(Tile& t, char* page, int bits_k, int bits_v) {
     reinterpret_cast<uint32_t*>(page + page_off_vcodes(bits_k))[tid - kHeadDim] = t.v1[tid - kHeadDim];
 }
 
+// Programmatic dependent launch: let the next kernel of the stream start
+// launching at once, then wait for the previous one (and its writes).
+__device__ __forceinline__ void pdl_enter() {
+  asm volatile("griddepcontrol.launch_dependents;\ngriddepcontrol.wait;" ::: "memory");
+}
+
 __device__ __forceinline__ char* page_ptr(const Dims& d, void* pages, int b, int h, int j) {
   return static_cast<char*>(pages) + (((long long)b * d.hkv + h) * d.max_blocks + j) * d.page_bytes;
 }
@@ -195,6 +201,7 @@ __global__ void __launch_bounds__(kPackThreads)
     pack_input_blocks_kernel(Dims d, kvq_cache c, const __half* __restrict__ k_new,
                              const __half* __restrict__ v_new, int n_new, int batch_begin) {
   __shared__ Tile tile;
+  pdl_enter();
   const int bi = blockIdx.z, b = batch_begin + bi, h = blockIdx.y;
   const int L0 = c.seq_len[b];
   const int L1 = L0 + n_new;
@@ -214,6 +221,7 @@ __global__ void __launch_bounds__(kPackThreads)
     pack_append_kernel(Dims d, kvq_cache c, const __half* __restrict__ k_new,
                        const __half* __restrict__ v_new, int n_new, int batch_begin) {
   __shared__ Tile tile;
+  pdl_enter();
   const int bi = blockIdx.y, b = batch_begin + bi, h = blockIdx.x;
   const int L0 = c.seq_len[b];
   const int L1 = L0 + n_new;
@@ -264,14 +272,24 @@ __global__ void __launch_bounds__(kPackThreads)
 cudaError_t launch_pack(const Dims& d, const kvq_cache& cache, const __half* k_new,
                         const __half* v_new, int n_new, int batch_begin, int batch_count,
                         cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kPackThreads);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e;
   if (n_new > kGroup) {
-    dim3 grid(n_new / kGroup + 1, d.hkv, batch_count);
-    pack_input_blocks_kernel<<<grid, kPackThreads, 0, stream>>>(d, cache, k_new, v_new, n_new,
-                                                                 batch_begin);
+    cfg.gridDim = dim3(n_new / kGroup + 1, d.hkv, batch_count);
+    e = cudaLaunchKernelEx(&cfg, pack_input_blocks_kernel, d, cache, k_new, v_new, n_new,
+                           batch_begin);
+    if (e != cudaSuccess) return e;
   }
-  dim3 grid2(d.hkv, batch_count);
-  pack_append_kernel<<<grid2, kPackThreads, 0, stream>>>(d, cache, k_new, v_new, n_new,
-                                                         batch_begin);
+  cfg.gridDim = dim3(d.hkv, batch_count);
+  e = cudaLaunchKernelEx(&cfg, pack_append_kernel, d, cache, k_new, v_new, n_new, batch_begin);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
