@@ -96,60 +96,117 @@ __device__ float block_max(float v, float* red) {
   return wmax(r);
 }
 
-// Merge up to 32 sorted lists (one per lane, `len` entries read by get(h))
-// into the first n entries of their common order; lane 0 writes ok/oi.
-template <typename Get>
-__device__ void warp_merge(int len, const Get& get, int n, uint32_t* ok, int* oi) {
-  const int lane = threadIdx.x & 31;
-  int head = 0;
-  uint32_t hk = 0u;
-  int hi = INT_MAX;
-  if (len > 0) get(0, hk, hi);
-  for (int r = 0; r < n; ++r) {
-    const uint32_t mk = __reduce_max_sync(0xffffffffu, hk);
-    const uint32_t mi = __reduce_min_sync(0xffffffffu, hk == mk ? (uint32_t)hi : 0xffffffffu);
-    if (lane == 0) {
-      ok[r] = mk;
-      oi[r] = (int)mi;
-    }
-    if (hk == mk && (uint32_t)hi == mi) {
-      ++head;
-      if (head < len) {
-        get(head, hk, hi);
-      } else {
-        hk = 0u;
-        hi = INT_MAX;
-      }
-    }
-  }
-  __syncwarp();
-}
+// ---------------------------------------------------------------------------
+// Block-wide top-n selection (256 threads).  Keys are order-preserving uint32
+// (larger is better; 0 marks padding); ties rank by the lower index.
+// ---------------------------------------------------------------------------
 
-// Sort kPer (key, index) pairs held in registers, best first (bitonic).
-__device__ __forceinline__ void sort_desc(uint32_t (&k)[kPer], int (&ix)[kPer]) {
+struct Sel {
+  unsigned hist[kT];   // one 8-bit digit's histogram
+  unsigned digit;      // the digit holding the n-th element
+  unsigned above;      // elements in higher digits
+  unsigned at;         // elements in that digit
+  unsigned pos;        // collection counter
+};
+
+// Key of the n-th largest key among the elements i < N with act(i) (which
+// must number at least n), and how many elements with that key belong to the
+// n largest: four passes of an 8-bit radix histogram, most significant first.
+template <typename KeyF, typename ActF>
+__device__ void radix_nth(int N, int n, const KeyF& key, const ActF& act, Sel& ss, uint32_t& T,
+                          int& need, int& n_at) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t prefix = 0u, mask = 0u;
+  unsigned rem = (unsigned)n;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    ss.hist[tid] = 0u;
+    __syncthreads();
+    for (int i = tid; i < N; i += kT) {
+      if (!act(i)) continue;
+      const uint32_t k = key(i);
+      if ((k & mask) == prefix) atomicAdd(&ss.hist[(k >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (warp == 0) {
+      // lane l takes digits 255 - 8 l .. 248 - 8 l, largest first
+      unsigned c[8], sum = 0u;
 #pragma unroll
-  for (int size = 2; size <= kPer; size <<= 1) {
+      for (int j = 0; j < 8; ++j) {
+        c[j] = ss.hist[255 - 8 * lane - j];
+        sum += c[j];
+      }
+      unsigned inc = sum;
 #pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned t = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += t;
+      }
+      unsigned acc = inc - sum;
+      if (acc < rem && rem <= inc) {
 #pragma unroll
-      for (int i = 0; i < kPer; ++i) {
-        const int j = i ^ stride;
-        if (j > i) {
-          const bool first_best = (i & size) == 0;
-          const bool swap = first_best ? before(k[j], ix[j], k[i], ix[i])
-                                       : before(k[i], ix[i], k[j], ix[j]);
-          if (swap) {
-            const uint32_t tk = k[i];
-            k[i] = k[j];
-            k[j] = tk;
-            const int ti = ix[i];
-            ix[i] = ix[j];
-            ix[j] = ti;
+        for (int j = 0; j < 8; ++j) {
+          if (acc < rem && rem <= acc + c[j]) {
+            ss.digit = 255u - 8u * lane - j;
+            ss.above = acc;
+            ss.at = c[j];
           }
+          acc += c[j];
         }
       }
     }
+    __syncthreads();
+    prefix |= ss.digit << shift;
+    mask |= 255u << shift;
+    rem -= ss.above;
+    n_at = (int)ss.at;
   }
+  T = prefix;
+  need = (int)rem;
+}
+
+// The n best of N elements (get(i, key, index)), sorted best first into
+// ok / oi; tk / ti hold n entries of scratch.
+template <typename GetF>
+__device__ void block_select(int N, int n, const GetF& get, Sel& ss, uint32_t* ok, int* oi,
+                             uint32_t* tk, int* ti) {
+  const int tid = threadIdx.x;
+  uint32_t T;
+  int need, n_at;
+  radix_nth(N, n, [&](int i) { uint32_t k; int x; get(i, k, x); return k; },
+            [](int) { return true; }, ss, T, need, n_at);
+  // Ties at T: the `need` lowest indices (largest ~index), unless all are taken.
+  uint32_t TI = 0u;
+  if (need < n_at) {
+    int need2, n_at2;
+    radix_nth(N, need, [&](int i) { uint32_t k; int x; get(i, k, x); return ~(uint32_t)x; },
+              [&](int i) { uint32_t k; int x; get(i, k, x); return k == T; }, ss, TI, need2,
+              n_at2);
+  }
+  if (tid == 0) ss.pos = 0u;
+  __syncthreads();
+  for (int i = tid; i < N; i += kT) {
+    uint32_t k;
+    int x;
+    get(i, k, x);
+    if (k > T || (k == T && ~(uint32_t)x >= TI)) {
+      const unsigned p = atomicAdd(&ss.pos, 1u);
+      if (p < (unsigned)n) {
+        tk[p] = k;
+        ti[p] = x;
+      }
+    }
+  }
+  __syncthreads();
+  if (tid < n) {  // rank sort (duplicates only among padding entries)
+    const uint32_t k = tk[tid];
+    const int x = ti[tid];
+    int r = 0;
+    for (int j = 0; j < n; ++j)
+      r += before(tk[j], ti[j], k, x) || (tk[j] == k && ti[j] == x && j < tid);
+    ok[r] = k;
+    oi[r] = x;
+  }
+  __syncthreads();
 }
 
 constexpr int kCandStage = 4096;            // staged (key, index) candidates of a row
@@ -158,13 +215,14 @@ constexpr size_t kW1StageMax = 176 * 1024;  // largest staged corrector W1
 struct Smem {
   union {
     struct {
-      uint32_t sk[kPer][kT];
-      int si[kPer][kT];
-    } srt;                              // chunk phase
+      uint32_t sk[kChunk];
+      int si[kChunk];
+    } srt;                              // chunk phase: the chunk's keys
     float w1[kW1StageMax / 4];          // finalize: corrector W1 (bulk copy)
   } u;
   uint2 cand[kCandStage];               // finalize: the row's candidate lists
   uint64_t w1_bar;
+  Sel sel;
   uint32_t wk[kWarpsD][kMaxK + 1];
   int wi[kWarpsD][kMaxK + 1];
   uint32_t fk[kMaxK + 1];
@@ -240,21 +298,12 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
   const float S1 = block_sum(s1, sm.red);
   const float S2 = block_sum(s2, sm.red);  // its barriers also publish sm.cand
 
-  // Merge the chunk candidate lists: warp w takes lists w*32 + lane, then
-  // warp 0 merges the eight warp results (n_chunks <= 256).
-  const int li = warp * 32 + lane;
-  warp_merge(li < nc ? K1 : 0, [&](int h, uint32_t& k, int& i) {
-    const uint2 v = cs ? sm.cand[li * K1 + h] : __ldcg(&cand[(size_t)li * K1 + h]);
+  // The window: the K + 1 best of all chunk candidates.
+  block_select(nc * K1, K1, [&](int i, uint32_t& k, int& x) {
+    const uint2 v = cs ? sm.cand[i] : __ldcg(&cand[i]);
     k = v.x;
-    i = (int)v.y;
-  }, K1, sm.wk[warp], sm.wi[warp]);
-  __syncthreads();
-  if (warp == 0)
-    warp_merge(lane < kWarpsD ? K1 : 0, [&](int h, uint32_t& k, int& i) {
-      k = sm.wk[lane][h];
-      i = sm.wi[lane][h];
-    }, K1, sm.fk, sm.fi);
-  __syncthreads();
+    x = (int)v.y;
+  }, sm.sel, sm.fk, sm.fi, &sm.wk[0][0], &sm.wi[0][0]);
 
   // Features phi (Sec. 4.2): warp 0, lanes over the window.
   if (warp == 0) {
@@ -335,15 +384,26 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     }
     if (tid < 8) sm.x[5 * K + tid] = sm.phi[tid];
     __syncthreads();
-    // Hidden layer: one warp per hidden unit, lanes over the inputs (W1 from
-    // shared memory when staged).
+    // The output layer's weight rows of this warp into L1 meanwhile.
+    for (int k = warp * 4 + (lane >> 3); k < K; k += kWarpsD * 4)
+      for (int j = (lane & 7) * 32; j < d.hidden; j += 256)
+        asm volatile("prefetch.global.L1 [%0];" ::"l"(p.cor_w2 + (size_t)k * d.hidden + j));
+    // Hidden layer: one thread per hidden unit (W1 from shared memory when
+    // staged); thread j starts at input j mod nin so that a warp's reads of
+    // its 32 rows fall in different banks.
     const float* w1 = (w1s && w1_ok) ? sm.u.w1 : p.cor_w1;
-    for (int j = warp; j < d.hidden; j += kWarpsD) {
+    for (int j = tid; j < d.hidden; j += kT) {
       const float* wrow = w1 + (size_t)j * nin;
-      float a = 0.0f;
-      for (int i = lane; i < nin; i += 32) a = fmaf(wrow[i], sm.x[i], a);
-      a = wsum(a);
-      if (lane == 0) sm.hb[j] = fmaxf(a + p.cor_b1[j], 0.0f);
+      float a0 = 0.0f, a1 = 0.0f;
+      int i = j % nin;
+      for (int c = 0; c + 1 < nin; c += 2) {
+        a0 = fmaf(wrow[i], sm.x[i], a0);
+        i = i + 1 == nin ? 0 : i + 1;
+        a1 = fmaf(wrow[i], sm.x[i], a1);
+        i = i + 1 == nin ? 0 : i + 1;
+      }
+      if (nin & 1) a0 = fmaf(wrow[i], sm.x[i], a0);
+      sm.hb[j] = fmaxf(a0 + a1 + p.cor_b1[j], 0.0f);
     }
     __syncthreads();
     // Output layer Delta_k (all of a warp's weight loads in one round), then
@@ -412,7 +472,7 @@ __global__ void __launch_bounds__(kT)
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
   // programmatic dependent launch: the logits are the previous kernel's output
   asm volatile("griddepcontrol.launch_dependents;\ngriddepcontrol.wait;" ::: "memory");
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tid = threadIdx.x;
   const int chunk = blockIdx.x, row = blockIdx.y, K1 = d.K + 1;
   const float* z = logits + (size_t)row * d.vocab;
   const int base = chunk * kChunk;
@@ -449,27 +509,19 @@ __global__ void __launch_bounds__(kT)
   s1 = block_sum(s1, sm.red);
   s2 = block_sum(s2, sm.red);
 
-  sort_desc(k, ix);
 #pragma unroll
   for (int i = 0; i < kPer; ++i) {
-    sm.u.srt.sk[i][tid] = k[i];
-    sm.u.srt.si[i][tid] = ix[i];
+    sm.u.srt.sk[i * kT + tid] = k[i];
+    sm.u.srt.si[i * kT + tid] = ix[i];
   }
-  __syncwarp();
-  warp_merge(kPer, [&](int h, uint32_t& kk, int& ii) {
-    kk = sm.u.srt.sk[h][tid];
-    ii = sm.u.srt.si[h][tid];
-  }, K1, sm.wk[warp], sm.wi[warp]);
-  __syncthreads();
+  // the barriers inside block_select publish the keys
+  block_select(kChunk, K1, [&](int i, uint32_t& kk, int& ii) {
+    kk = sm.u.srt.sk[i];
+    ii = sm.u.srt.si[i];
+  }, sm.sel, sm.fk, sm.fi, &sm.wk[0][0], &sm.wi[0][0]);
   uint2* out = ws.cand + ((size_t)row * d.n_chunks + chunk) * K1;
-  if (warp == 0) {
-    warp_merge(lane < kWarpsD ? K1 : 0, [&](int h, uint32_t& kk, int& ii) {
-      kk = sm.wk[lane][h];
-      ii = sm.wi[lane][h];
-    }, K1, sm.fk, sm.fi);
-    for (int r = lane; r < K1; r += 32) out[r] = make_uint2(sm.fk[r], (uint32_t)sm.fi[r]);
-    if (lane == 0) ws.stats[(size_t)row * d.n_chunks + chunk] = make_float4(m, s1, s2, 0.0f);
-  }
+  for (int r = tid; r < K1; r += kT) out[r] = make_uint2(sm.fk[r], (uint32_t)sm.fi[r]);
+  if (tid == 0) ws.stats[(size_t)row * d.n_chunks + chunk] = make_float4(m, s1, s2, 0.0f);
 
   __syncthreads();
   if (tid == 0) {
