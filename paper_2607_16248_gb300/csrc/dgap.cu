@@ -184,13 +184,23 @@ __device__ void block_select(int N, int n, const GetF& get, Sel& ss, uint32_t* o
   }
   if (tid == 0) ss.pos = 0u;
   __syncthreads();
-  for (int i = tid; i < N; i += kT) {
-    uint32_t k;
-    int x;
-    get(i, k, x);
-    if (k > T || (k == T && ~(uint32_t)x >= TI)) {
-      const unsigned p = atomicAdd(&ss.pos, 1u);
-      if (p < (unsigned)n) {
+  const int lane = tid & 31;
+  for (int b0 = 0; b0 < N; b0 += kT) {
+    const int i = b0 + tid;
+    uint32_t k = 0u;
+    int x = 0;
+    bool take = false;
+    if (i < N) {
+      get(i, k, x);
+      take = k > T || (k == T && ~(uint32_t)x >= TI);
+    }
+    const unsigned m = __ballot_sync(0xffffffffu, take);
+    if (m) {
+      unsigned p0 = 0u;
+      if (lane == __ffs(m) - 1) p0 = atomicAdd(&ss.pos, (unsigned)__popc(m));
+      p0 = __shfl_sync(0xffffffffu, p0, __ffs(m) - 1);
+      const unsigned p = p0 + __popc(m & ((1u << lane) - 1u));
+      if (take && p < (unsigned)n) {
         tk[p] = k;
         ti[p] = x;
       }
@@ -209,8 +219,91 @@ __device__ void block_select(int N, int n, const GetF& get, Sel& ss, uint32_t* o
   __syncthreads();
 }
 
-constexpr int kCandStage = 4096;            // staged (key, index) candidates of a row
-constexpr size_t kW1StageMax = 176 * 1024;  // largest staged corrector W1
+// Largest key of lane rank q - 1 in the warp (keys sorted descending across
+// lanes by a bitonic network of shuffles).
+__device__ __forceinline__ uint32_t warp_kth_key(uint32_t k, int q) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const uint32_t o = __shfl_xor_sync(0xffffffffu, k, stride);
+      const bool lower = (lane & stride) == 0;          // keeps the larger when descending
+      const bool desc = (lane & size) == 0 || size == 32;
+      k = (lower == desc) ? max(k, o) : min(k, o);
+    }
+  return __shfl_sync(0xffffffffu, k, q - 1);
+}
+
+constexpr int kSurvivors = 1024;  // candidates kept for the exact ranking
+
+// The n best (n <= 72) of the elements the CTA's threads hold in registers
+// (E per thread; key 0 marks padding), sorted best first into ok / oi.
+// Every warp's q = ceil(n / 8)-th largest per-thread maximum bounds the n-th
+// best key from below (8 q >= n elements reach it), so the elements at or
+// above the smallest of those bounds contain the n best.  They are packed
+// into sv as (key, ~index) words, whose order is the ranking order, and
+// ranked exactly.  With more than kSurvivors of them (heavy ties) every
+// thread calls fallback() instead.
+template <int E, typename Fallback>
+__device__ void select_top(const uint32_t (&k)[E], const int (&x)[E], int n, Sel& ss,
+                           unsigned long long* sv, uint32_t* ok, int* oi,
+                           const Fallback& fallback) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t mk = 0u;
+#pragma unroll
+  for (int i = 0; i < E; ++i) mk = max(mk, k[i]);
+  const uint32_t wq = warp_kth_key(mk, (n + kWarpsD - 1) / kWarpsD);
+  if (lane == 0) ss.hist[warp] = wq;
+  __syncthreads();
+  uint32_t T0 = ss.hist[0];
+#pragma unroll
+  for (int w = 1; w < kWarpsD; ++w) T0 = min(T0, ss.hist[w]);
+  int c = 0;
+#pragma unroll
+  for (int i = 0; i < E; ++i) c += k[i] >= T0;
+  int inc = c;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += t;
+  }
+  if (lane == 31) ss.hist[kWarpsD + warp] = (unsigned)inc;
+  __syncthreads();
+  int off = inc - c, S = 0;
+#pragma unroll
+  for (int w = 0; w < kWarpsD; ++w) {
+    const int cw = (int)ss.hist[kWarpsD + w];
+    off += w < warp ? cw : 0;
+    S += cw;
+  }
+  if (S > kSurvivors) {
+    __syncthreads();
+    fallback();
+    return;
+  }
+#pragma unroll
+  for (int i = 0; i < E; ++i)
+    if (k[i] >= T0) sv[off++] = ((unsigned long long)k[i] << 32) | (uint32_t)~x[i];
+  __syncthreads();
+  for (int t = tid; t < S; t += kT) {
+    const unsigned long long me = sv[t];
+    int r = 0;
+#pragma unroll 8
+    for (int j = 0; j < S; ++j) {
+      const unsigned long long o = sv[j];
+      r += (o > me) || (o == me && j < t);
+    }
+    if (r < n) {
+      ok[r] = (uint32_t)(me >> 32);
+      oi[r] = (int)~(uint32_t)me;
+    }
+  }
+  __syncthreads();
+}
+
+constexpr int kCandReg = 16;                // candidates of a row per thread (finalize)
+constexpr size_t kW1StageMax = 168 * 1024;  // largest staged corrector W1 (256 x 168)
 
 struct Smem {
   union {
@@ -220,9 +313,9 @@ struct Smem {
     } srt;                              // chunk phase: the chunk's keys
     float w1[kW1StageMax / 4];          // finalize: corrector W1 (bulk copy)
   } u;
-  uint2 cand[kCandStage];               // finalize: the row's candidate lists
   uint64_t w1_bar;
   Sel sel;
+  unsigned long long sv[kSurvivors];    // select_top: candidates above the bound
   uint32_t wk[kWarpsD][kMaxK + 1];
   int wi[kWarpsD][kMaxK + 1];
   uint32_t fk[kMaxK + 1];
@@ -273,9 +366,16 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
 
   // Chunk statistics and candidate lists in one round of loads.
   const uint2* cand = ws.cand + (size_t)row * nc * K1;
-  const bool cs = nc * K1 <= kCandStage;
-  if (cs)
-    for (int i = tid; i < nc * K1; i += kT) sm.cand[i] = __ldcg(&cand[i]);
+  const int n_cand = nc * K1;
+  uint32_t ck[kCandReg];
+  int cx[kCandReg];
+#pragma unroll
+  for (int e = 0; e < kCandReg; ++e) {
+    const int i = tid + e * kT;
+    const uint2 v = i < n_cand ? __ldcg(&cand[i]) : make_uint2(0u, (uint32_t)INT_MAX);
+    ck[e] = v.x;
+    cx[e] = (int)v.y;
+  }
   float mloc = -INFINITY;
   float4 sv[(kMaxChunks + kT - 1) / kT];
 #pragma unroll
@@ -296,14 +396,19 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     }
   }
   const float S1 = block_sum(s1, sm.red);
-  const float S2 = block_sum(s2, sm.red);  // its barriers also publish sm.cand
+  const float S2 = block_sum(s2, sm.red);
 
-  // The window: the K + 1 best of all chunk candidates.
-  block_select(nc * K1, K1, [&](int i, uint32_t& k, int& x) {
-    const uint2 v = cs ? sm.cand[i] : __ldcg(&cand[i]);
-    k = v.x;
-    x = (int)v.y;
-  }, sm.sel, sm.fk, sm.fi, &sm.wk[0][0], &sm.wi[0][0]);
+  // The window: the K + 1 best of all chunk candidates (the registers hold
+  // the first kCandReg * 256; a longer list goes the radix way).
+  auto from_global = [&]() {
+    block_select(n_cand, K1, [&](int i, uint32_t& k, int& x) {
+      const uint2 v = __ldcg(&cand[i]);
+      k = v.x;
+      x = (int)v.y;
+    }, sm.sel, sm.fk, sm.fi, &sm.wk[0][0], &sm.wi[0][0]);
+  };
+  if (n_cand > kCandReg * kT) from_global();
+  else select_top(ck, cx, K1, sm.sel, sm.sv, sm.fk, sm.fi, from_global);
 
   // Features phi (Sec. 4.2): warp 0, lanes over the window.
   if (warp == 0) {
@@ -464,7 +569,7 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
   }
 }
 
-__global__ void __launch_bounds__(kT)
+__global__ void __launch_bounds__(kT, 1)
     dgap_kernel(DgapDims d, dgap_params p, float* __restrict__ logits, int32_t* topk_idx,
                 float* topk_val, float* risk, uint8_t* gate, int32_t* next_token,
                 float* features, DWs ws) {
@@ -509,16 +614,18 @@ __global__ void __launch_bounds__(kT)
   s1 = block_sum(s1, sm.red);
   s2 = block_sum(s2, sm.red);
 
+  select_top(k, ix, K1, sm.sel, sm.sv, sm.fk, sm.fi, [&]() {
 #pragma unroll
-  for (int i = 0; i < kPer; ++i) {
-    sm.u.srt.sk[i * kT + tid] = k[i];
-    sm.u.srt.si[i * kT + tid] = ix[i];
-  }
-  // the barriers inside block_select publish the keys
-  block_select(kChunk, K1, [&](int i, uint32_t& kk, int& ii) {
-    kk = sm.u.srt.sk[i];
-    ii = sm.u.srt.si[i];
-  }, sm.sel, sm.fk, sm.fi, &sm.wk[0][0], &sm.wi[0][0]);
+    for (int i = 0; i < kPer; ++i) {
+      sm.u.srt.sk[i * kT + tid] = k[i];
+      sm.u.srt.si[i * kT + tid] = ix[i];
+    }
+    __syncthreads();
+    block_select(kChunk, K1, [&](int i, uint32_t& kk, int& ii) {
+      kk = sm.u.srt.sk[i];
+      ii = sm.u.srt.si[i];
+    }, sm.sel, sm.fk, sm.fi, &sm.wk[0][0], &sm.wi[0][0]);
+  });
   uint2* out = ws.cand + ((size_t)row * d.n_chunks + chunk) * K1;
   for (int r = tid; r < K1; r += kT) out[r] = make_uint2(sm.fk[r], (uint32_t)sm.fi[r]);
   if (tid == 0) ws.stats[(size_t)row * d.n_chunks + chunk] = make_float4(m, s1, s2, 0.0f);
