@@ -321,7 +321,7 @@ struct Smem {
   uint32_t fk[kMaxK + 1];
   int fi[kMaxK + 1];
   float zt[kMaxK];
-  float x[kMaxIn];
+  alignas(16) float x[kMaxIn];
   float hb[kMaxHidden];
   float phi[8];
   float red[32];
@@ -362,6 +362,15 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
             smem_u32(sm.u.w1)),
         "l"(p.cor_w1), "r"(w1_bytes), "r"(smem_u32(&sm.w1_bar))
         : "memory");
+  }
+
+  // This thread's detector unit (j = tid), loaded with the first round.
+  float dw[8], db1 = 0.0f, dw2 = 0.0f;
+  if (tid < d.hidden) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) dw[i] = __ldg(p.det_w1 + tid * 8 + i);
+    db1 = __ldg(p.det_b1 + tid);
+    dw2 = __ldg(p.det_w2 + tid);
   }
 
   // Chunk statistics and candidate lists in one round of loads.
@@ -422,17 +431,20 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
       sum += zk;
       if (k + 1 < K) min_gap = fminf(min_gap, zk - key_value(sm.fk[k + 1]));
     }
-    mass_e = wsum(mass_e);
-    wsum_e = wsum(wsum_e);
-    const float mean = wsum(sum) / (float)K;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {  // four independent reductions, interleaved
+      mass_e += __shfl_xor_sync(0xffffffffu, mass_e, o);
+      wsum_e += __shfl_xor_sync(0xffffffffu, wsum_e, o);
+      sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      min_gap = fminf(min_gap, __shfl_xor_sync(0xffffffffu, min_gap, o));
+    }
+    const float mean = sum / (float)K;
     float var = 0.0f;
     for (int k = lane; k < K; k += 32) {
       const float dz = key_value(sm.fk[k]) - mean;
       var += dz * dz;
     }
     var = wsum(var) / (float)K;
-#pragma unroll
-    for (int o = 16; o; o >>= 1) min_gap = fminf(min_gap, __shfl_xor_sync(0xffffffffu, min_gap, o));
     if (lane == 0) {
       sm.phi[0] = logf(S1) - S2 / S1;
       sm.phi[1] = mass_e / S1;
@@ -449,7 +461,13 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
 
   // Detector f = w2 . relu(W1 phi + b1) + b2 (Eq. 6).
   float part = 0.0f;
-  for (int j = tid; j < d.hidden; j += kT) {
+  if (tid < d.hidden) {
+    float a = db1;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a = fmaf(dw[i], sm.phi[i], a);
+    part = dw2 * fmaxf(a, 0.0f);
+  }
+  for (int j = tid + kT; j < d.hidden; j += kT) {
     float a = p.det_b1[j];
 #pragma unroll
     for (int i = 0; i < 8; ++i) a = fmaf(p.det_w1[j * 8 + i], sm.phi[i], a);
@@ -489,14 +507,44 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     }
     if (tid < 8) sm.x[5 * K + tid] = sm.phi[tid];
     __syncthreads();
-    // The output layer's weight rows of this warp into L1 meanwhile.
-    for (int k = warp * 4 + (lane >> 3); k < K; k += kWarpsD * 4)
-      for (int j = (lane & 7) * 32; j < d.hidden; j += 256)
-        asm volatile("prefetch.global.L1 [%0];" ::"l"(p.cor_w2 + (size_t)k * d.hidden + j));
+    // The output layer's weights of this thread (output k = tid / 8, every
+    // eighth hidden unit from tid mod 8) into registers meanwhile, when the
+    // layer is one pass of at most 256 units.
+    constexpr int kW2Reg = 32;
+    const bool w2r = K <= kT / 8 && d.hidden <= 8 * kW2Reg;
+    float w2v[kW2Reg];
+    if (w2r) {
+      const int k = tid >> 3, s8 = tid & 7;
+#pragma unroll
+      for (int i = 0; i < kW2Reg; ++i) {
+        const int j = s8 + 8 * i;
+        w2v[i] = (k < K && j < d.hidden) ? __ldg(p.cor_w2 + (size_t)k * d.hidden + j) : 0.0f;
+      }
+    }
     // Hidden layer: one thread per hidden unit (W1 from shared memory when
     // staged); thread j starts at input j mod nin so that a warp's reads of
     // its 32 rows fall in different banks.
     const float* w1 = (w1s && w1_ok) ? sm.u.w1 : p.cor_w1;
+    if (w1s && w1_ok && (nin & 3) == 0) {
+      // staged rows of 16-byte multiples: float4 reads, four accumulators
+      const float4* xv = reinterpret_cast<const float4*>(sm.x);
+      const int n4 = nin / 4;
+      for (int j = tid; j < d.hidden; j += kT) {
+        const float4* wr = reinterpret_cast<const float4*>(sm.u.w1 + (size_t)j * nin);
+        float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        int c = j % n4;  // skewed start: the eight rows of a phase hit different banks
+#pragma unroll 6
+        for (int t = 0; t < n4; ++t) {
+          const float4 w = wr[c], xx = xv[c];
+          a.x = fmaf(w.x, xx.x, a.x);
+          a.y = fmaf(w.y, xx.y, a.y);
+          a.z = fmaf(w.z, xx.z, a.z);
+          a.w = fmaf(w.w, xx.w, a.w);
+          c = c + 1 == n4 ? 0 : c + 1;
+        }
+        sm.hb[j] = fmaxf((a.x + a.y) + (a.z + a.w) + p.cor_b1[j], 0.0f);
+      }
+    } else
     for (int j = tid; j < d.hidden; j += kT) {
       const float* wrow = w1 + (size_t)j * nin;
       float a0 = 0.0f, a1 = 0.0f;
@@ -511,37 +559,28 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
       sm.hb[j] = fmaxf(a0 + a1 + p.cor_b1[j], 0.0f);
     }
     __syncthreads();
-    // Output layer Delta_k (all of a warp's weight loads in one round), then
-    // the sparse merge (Eq. 13).
-    for (int k0 = warp * 4; k0 < K; k0 += kWarpsD * 4) {
-      float a[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-      for (int j0 = 0; j0 < d.hidden; j0 += 256) {
-        float wv[4][8];
+    // Output layer Delta_k: eight threads per output, each over every eighth
+    // hidden unit (rows prefetched into L1 above), then the sparse merge
+    // (Eq. 13).
+    for (int k0 = 0; k0 < K; k0 += kT / 8) {
+      const int k = k0 + (tid >> 3), s8 = tid & 7;
+      float a = 0.0f;
+      if (w2r) {
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int t = 0; t < 8; ++t) {
-            const int j = j0 + lane + 32 * t;
-            wv[u][t] = (k0 + u < K && j < d.hidden) ? __ldg(p.cor_w2 + (size_t)(k0 + u) * d.hidden + j)
-                                                     : 0.0f;
-          }
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int t = 0; t < 8; ++t) {
-            const int j = j0 + lane + 32 * t;
-            if (j < d.hidden) a[u] = fmaf(wv[u][t], sm.hb[j], a[u]);
-          }
+        for (int i = 0; i < kW2Reg; ++i)
+          if (s8 + 8 * i < d.hidden) a = fmaf(w2v[i], sm.hb[s8 + 8 * i], a);
+      } else if (k < K) {
+        const float* wrow = p.cor_w2 + (size_t)k * d.hidden;
+#pragma unroll 8
+        for (int j = s8; j < d.hidden; j += 8) a = fmaf(__ldg(wrow + j), sm.hb[j], a);
       }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const float au = wsum(a[u]);
-        const int k = k0 + u;
-        if (lane == 0 && k < K) {
-          const float zt = sm.zt[k] + (au + p.cor_b2[k]);
-          sm.zt[k] = zt;
-          logits[(size_t)row * d.vocab + sm.fi[k]] = zt;
-        }
+      a += __shfl_xor_sync(0xffffffffu, a, 1);
+      a += __shfl_xor_sync(0xffffffffu, a, 2);
+      a += __shfl_xor_sync(0xffffffffu, a, 4);
+      if (k < K && s8 == 0) {
+        const float zt = sm.zt[k] + (a + p.cor_b2[k]);
+        sm.zt[k] = zt;
+        logits[(size_t)row * d.vocab + sm.fi[k]] = zt;
       }
     }
     __syncthreads();
