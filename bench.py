@@ -290,7 +290,9 @@ def reduce_max(x, world):
 
 
 class Step:
-    """Caches, inputs, workspaces and the three captured graphs of a step."""
+    """Caches, inputs, workspaces and the captured graphs of a step: the whole
+    step (per layer kvq_pack then kvq_decode_attn, then the logits and
+    dgap_restore), the step without dgap_restore, and each phase alone."""
 
     def __init__(self, spec, steps_total, device, rank):
         import torch
@@ -316,6 +318,8 @@ class Step:
                 del k, v
             self.caches.append(cache)
         torch.cuda.synchronize()
+        # lengths after the prefill: every measurement starts from them
+        self.seq0 = [c.seq_region().clone() for c in self.caches]
         g = synth.generator(seed + 1, device)
         self.q = torch.randn(layers, B, hq, 128, generator=g, device=device).half()
         self.k_new = torch.randn(layers, B, hkv, 1, 128, generator=g, device=device).half()
@@ -357,17 +361,43 @@ class Step:
     def _capture(self, kvq):
         import torch
         L = self.spec["layers"]
-        self.g_pack, self.g_attn, self.g_dgap = (torch.cuda.CUDAGraph() for _ in range(3))
+
+        def pack(l):
+            kvq.kvq_pack(self.caches[l], self.k_new[l], self.v_new[l])
+
+        def attn(l):
+            kvq.kvq_decode_attn(self.caches[l], self.q[l], out=self.out[l],
+                                n_splits=self.n_splits, workspace=self.ws_attn)
+
+        def epilogue():
+            self.dgap.restore(self.logits, outputs=self.dout, workspace=self.ws_dgap)
+
+        self.g_step, self.g_step_nd, self.g_pack, self.g_attn, self.g_dgap = (
+            torch.cuda.CUDAGraph() for _ in range(5))
+        for g, with_dgap in ((self.g_step, True), (self.g_step_nd, False)):
+            with torch.cuda.graph(g):
+                for l in range(L):
+                    pack(l)
+                    attn(l)
+                self.logits.copy_(self.logits0)  # stands in for the LM head's output
+                if with_dgap:
+                    epilogue()
         with torch.cuda.graph(self.g_pack):
             for l in range(L):
-                kvq.kvq_pack(self.caches[l], self.k_new[l], self.v_new[l])
+                pack(l)
         with torch.cuda.graph(self.g_attn):
             for l in range(L):
-                kvq.kvq_decode_attn(self.caches[l], self.q[l], out=self.out[l],
-                                    n_splits=self.n_splits, workspace=self.ws_attn)
+                attn(l)
         with torch.cuda.graph(self.g_dgap):
-            self.dgap.restore(self.logits, outputs=self.dout, workspace=self.ws_dgap)
+            epilogue()
         torch.cuda.synchronize()
+
+    def rewind(self):
+        """Set every cache back to its prefill lengths (the pages and window
+        rows written since stay in place and are overwritten again), so each
+        measurement runs at the workload's context length."""
+        for c, s0 in zip(self.caches, self.seq0):
+            c.seq_region().copy_(s0)
 
     def launches_per_step(self):
         return 2 * self.spec["layers"] + 1
@@ -387,32 +417,35 @@ def run_gpu(args, spec):
     device = torch.device("cuda", local if world > 1 else 0)
     K, W = args.steps, args.warmup
     e2e_on = not args.no_e2e
-    total_steps = (W + K) * (2 if e2e_on else 1)
+    # Each measurement (the headline, the step without the epilogue, the
+    # phases alone, the end-to-end run) replays W warm-up + K timed steps from
+    # the prefill lengths (Step.rewind).
+    total_steps = W + K
     st = Step(spec, total_steps, device, rank)
-    done = 0  # steps replayed so far (each appends one token per sequence and layer)
+    done = 0  # steps replayed since the last rewind (each appends one token)
 
-    def replay(n, ev=None):
+    def timed(replay_one, n_warm, n):
+        """Replay n_warm untimed and n timed steps back to back; device ms."""
         nonlocal done
-        for i in range(n):
-            if ev is not None:
-                ev[i][0].record()
-            st.g_pack.replay()
-            if ev is not None:
-                ev[i][1].record()
-            st.g_attn.replay()
-            if ev is not None:
-                ev[i][2].record()
-            st.logits.copy_(st.logits0)
-            if ev is not None:
-                ev[i][3].record()
-            st.g_dgap.replay()
-            if ev is not None:
-                ev[i][4].record()
+        for _ in range(n_warm):
+            replay_one()
+        done += n_warm
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        barrier(world)
+        t0.record()
+        for _ in range(n):
+            replay_one()
+        t1.record()
+        torch.cuda.synchronize()
         done += n
+        return reduce_max(t0.elapsed_time(t1), world)
 
-    replay(W)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # Headline: K whole steps, one graph each.
+    st.rewind()
+    for _ in range(W):
+        st.g_step.replay()
+    done += W
     step0 = done
     clocks = Clocks(torch.cuda.current_device())
     torch.cuda.synchronize()
@@ -421,29 +454,56 @@ def run_gpu(args, spec):
     time.sleep(0.25)  # let the sampler come up before the timed region
     torch.cuda.synchronize()
     wall0 = time.perf_counter()
-    t_start.record()
-    replay(K, ev)
-    t_end.record()
-    torch.cuda.synchronize()
+    total_ms = timed(st.g_step.replay, 0, K)
     wall = time.perf_counter() - wall0
-    barrier(world)
     clk = clocks.stop()
-
-    total_ms = reduce_max(t_start.elapsed_time(t_end), world)
-    attn_ms = sum(e[1].elapsed_time(e[2]) for e in ev)
-    pack_ms = sum(e[0].elapsed_time(e[1]) for e in ev)
-    epi_ms = sum(e[3].elapsed_time(e[4]) for e in ev)
     step_bytes = [st.bytes_for_step(step0 + i) for i in range(K)]
     bytes_total = sum(step_bytes)
+
+    # The epilogue's share of a step: the same steps without dgap_restore.
+    st.rewind()
+    done = 0
+    nd_ms = timed(st.g_step_nd.replay, W, K)
+    epi_ms = max(total_ms - nd_ms, 0.0)
+
+    # Phase breakdown: each phase's graph alone (one graph launch per step).
+    def phases():
+        st.g_pack.replay()
+        ev[0].record()
+        st.g_attn.replay()
+        ev[1].record()
+        st.logits.copy_(st.logits0)
+        st.g_dgap.replay()
+
+    st.rewind()
+    done = 0
+    attn_ms = 0.0
+    pack_ms = 0.0
+    ph_step0 = done + W
+    for i in range(W + K):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        e0 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        phases()
+        torch.cuda.synchronize()
+        if i >= W:
+            pack_ms += e0.elapsed_time(ev[0])
+            attn_ms += ev[0].elapsed_time(ev[1])
+    done += W + K
+    attn_ms = reduce_max(attn_ms, world)
+    attn_bytes_total = sum(st.bytes_for_step(ph_step0 + i) for i in range(K))
+
     value = world * bytes_total / (total_ms * 1e-3) / 1e9
     launches = K * st.launches_per_step()
     attn_launches = K * spec["layers"]
-    achieved = bytes_total / (attn_ms * 1e-3) / 1e9
+    achieved = attn_bytes_total / (attn_ms * 1e-3) / 1e9
     peak, peak_kind = measured_peak_hbm()
 
     e2e = None
     if e2e_on:
-        e2e = run_e2e(st, W, K, world)
+        st.rewind()
+        done = 0
+        e2e = run_e2e(st, W, K, world, done)
         done += W + K
 
     s = spec
@@ -457,8 +517,8 @@ def run_gpu(args, spec):
            "n_splits": st.n_splits,
            "l2": f"inputs larger than L2: {step_bytes[0] / 1e6:.0f} MB of packed KV read per "
                  f"step (distinct cache per layer), L2 129 MB",
-           "step": f"{s['layers']} x (kvq_pack + kvq_decode_attn) + dgap_restore, "
-                   f"3 CUDA graphs", "parallelism": f"replicas x{world}" if world > 1 else "1 GPU"}
+           "step": f"{s['layers']} x (kvq_pack, kvq_decode_attn) + logits copy + dgap_restore, "
+                   f"one CUDA graph per step", "parallelism": f"replicas x{world}" if world > 1 else "1 GPU"}
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": round(total_ms / K, 5),
@@ -472,12 +532,14 @@ def run_gpu(args, spec):
         "pack_us_per_step": round(pack_ms / K * 1e3, 3),
         "epilogue_us_per_step": round(epi_ms / K * 1e3, 3),
         "epilogue_frac_of_step_attn": round(epi_ms / attn_ms, 5),
+        "breakdown": "attn_us_per_layer / pack_us_per_step: each phase's graph alone; "
+                     "epilogue_us_per_step: step graph minus the same graph without dgap_restore",
         "gated_rows_fraction": float(st.dout["gate"].float().mean().item()),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "peak_source": f"{peak_kind} hbm_gbs (copy)",
                      "traffic": profiled_traffic(),
-                     "algorithmic_bytes_per_launch": round(bytes_total / attn_launches)},
+                     "algorithmic_bytes_per_launch": round(attn_bytes_total / attn_launches)},
         "gpu_launches": launches,
         "wall_s_timed": round(wall, 4),
         "clocks": clk,
@@ -495,7 +557,7 @@ def run_gpu(args, spec):
         dist.destroy_process_group()
 
 
-def run_e2e(st, W, K, world):
+def run_e2e(st, W, K, world, done):
     """The same metric through the public calls with host buffers: per step,
     copy the step's inputs from pinned host memory, replay the step, read the
     step's result (greedy token, window, risk, gate) back and synchronise."""
@@ -513,10 +575,8 @@ def run_e2e(st, W, K, world):
         st.q.copy_(h_q, non_blocking=True)
         st.k_new.copy_(h_k, non_blocking=True)
         st.v_new.copy_(h_v, non_blocking=True)
-        st.g_pack.replay()
-        st.g_attn.replay()
-        st.logits.copy_(h_z, non_blocking=True)
-        st.g_dgap.replay()
+        st.logits0.copy_(h_z, non_blocking=True)
+        st.g_step.replay()
         for h, d in zip(h_out, outs):
             h.copy_(d, non_blocking=True)
         torch.cuda.current_stream().synchronize()
@@ -535,7 +595,7 @@ def run_e2e(st, W, K, world):
     ms = reduce_max(t0.elapsed_time(t1), world)
     # The e2e steps continue the same decode: lengths kept growing.
     s = st.spec
-    start = 2 * W + K  # steps replayed before the first timed e2e step
+    start = done + W  # steps replayed before the first timed e2e step
     total = sum(st.bytes_for_step(start + i) for i in range(K))
     return {"value": round(world * total / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
             "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo,

@@ -103,7 +103,8 @@ typedef struct kvq_config {
  *         absolute position p sits in slot p mod (R + 32).
  * seq_len [batch + 2] int32: [0, batch) token counts L, [batch] the flag word
  *         (KVQ_FLAG_*), [batch + 1] reserved; followed by `batch` uint32
- *         tickets used by kvq_pack.  kvq_cache_reset zeroes all of it.
+ *         tickets used by kvq_pack and kvq_decode_step.  kvq_cache_reset
+ *         zeroes all of it.
  */
 typedef struct kvq_cache {
   void* pages;
@@ -207,6 +208,27 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache,
                            const uint16_t* q, float* out,
                            float softmax_scale, int32_t n_splits,
                            void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * kvq_decode_step — one decode step of one layer: kvq_pack of one token per
+ * sequence followed by kvq_decode_attn, in one kernel (Sec. 3.1 quantizer,
+ * Sec. 1 attention).  The token at position L = seq_len[b] is attended from
+ * k_new / v_new directly and written to its window slot; when it pushes a
+ * 32-token group out of the window, that group is quantized (bit-identical to
+ * kvq_pack) into its page and attended in quantized form; seq_len[b] becomes
+ * L + 1 when the kernel ends.  Query groups wider than 4 run kvq_pack's kernel
+ * and then the attention kernel.
+ *   k_new, v_new   device fp16 [batch][n_kv_heads][128], 16-byte aligned.
+ *   q, out, softmax_scale, n_splits, workspace, ws_bytes: as kvq_decode_attn.
+ * A sequence at max_len is not appended (KVQ_FLAG_OVERFLOW is set) and
+ * attends over its L tokens.  Results equal kvq_pack(n_new = 1) then
+ * kvq_decode_attn on the same inputs.
+ */
+kvq_status kvq_decode_step(const kvq_config* cfg, const kvq_cache* cache,
+                           const uint16_t* k_new, const uint16_t* v_new,
+                           const uint16_t* q, float* out, float softmax_scale,
+                           int32_t n_splits, void* workspace, size_t ws_bytes,
+                           void* stream);
 
 /*
  * kvq_decode_attn_noalloc — kvq_decode_attn without a caller workspace.

@@ -242,6 +242,43 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const 
                      "kvq_decode_attn launch");
 }
 
+kvq_status kvq_decode_step(const kvq_config* cfg, const kvq_cache* cache, const uint16_t* k_new,
+                           const uint16_t* v_new, const uint16_t* q, float* out,
+                           float softmax_scale, int32_t n_splits, void* workspace,
+                           size_t ws_bytes, void* stream) {
+  kvq_status s = check_config(cfg);
+  if (s != KVQ_OK) return s;
+  if ((s = check_cache(*cfg, cache)) != KVQ_OK) return s;
+  if (!k_new || !v_new || !q || !out) return fail(KVQ_ERR_ARG, "k_new / v_new / q / out is NULL");
+  if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(q) || !aligned16(out))
+    return fail(KVQ_ERR_ALIGN, "k_new / v_new / q / out must be 16-byte aligned");
+  if (!(softmax_scale >= 0.0f) || isinf(softmax_scale))
+    return fail(KVQ_ERR_ARG, "softmax_scale must be finite and >= 0");
+  if (n_splits == 0) n_splits = default_splits(*cfg);
+  if (n_splits < 1 || n_splits > kMaxSplits - 1)
+    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, n_splits);
+  Dims d = make_dims(*cfg);
+  const size_t need = attn_workspace_bytes(d, n_splits);
+  if (!workspace) return fail(KVQ_ERR_ARG, "workspace is NULL");
+  if (!aligned16(workspace)) return fail(KVQ_ERR_ALIGN, "workspace must be 16-byte aligned");
+  if (ws_bytes < need)
+    return fail(KVQ_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+  const float scale = softmax_scale == 0.0f ? 1.0f / sqrtf((float)kHeadDim) : softmax_scale;
+  const float scale_log2 = scale * 1.4426950408889634f;
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const __half* kn = reinterpret_cast<const __half*>(k_new);
+  const __half* vn = reinterpret_cast<const __half*>(v_new);
+  const __half* qh = reinterpret_cast<const __half*>(q);
+  if (d.gq > 4) {  // the SIMT attention path: the append runs as its own kernel
+    cudaError_t e = launch_pack(d, *cache, kn, vn, 1, 0, d.batch, st);
+    if (e == cudaSuccess) e = launch_decode_attn(d, *cache, qh, out, scale_log2, n_splits, workspace, st);
+    return cuda_status(e, "kvq_decode_step launch");
+  }
+  return cuda_status(launch_decode_step(d, *cache, kn, vn, qh, out, scale_log2, n_splits,
+                                        workspace, st),
+                     "kvq_decode_step launch");
+}
+
 kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache,
                                    const uint16_t* q, float* out, float softmax_scale,
                                    int32_t n_splits, void* stream) {

@@ -716,16 +716,20 @@ __device__ __forceinline__ void cp_async_wait_all() {
 }
 
 // Copy rows p0 .. p0 + 31 of one (sequence, kv-head) ring (fp16 [ring][128])
-// into `rows` ([32][kResRow]); rows at or past n_tok are zero-filled.
+// into `rows` ([32][kResRow]); rows at or past n_tok are zero-filled.  The row
+// of position p_new (a token appended by this kernel, not yet in the ring)
+// comes from new_row instead.
 __device__ __forceinline__ void stage_rows(__half* rows, const __half* ring_base, int p0, int n_tok,
-                                           int ring) {
+                                           int ring, int p_new = -1,
+                                           const __half* new_row = nullptr) {
   const int lane = threadIdx.x & 31;
 #pragma unroll 4
   for (int e = lane; e < kGroup * 16; e += 32) {
     const int row = e >> 4, piece = e & 15;
     const bool ok = row < n_tok;
-    const long long off = ok ? (long long)((p0 + row) % ring) * kHeadDim : 0;
-    cp_async16(rows + row * kResRow + piece * 8, ring_base + off + piece * 8, ok ? 16u : 0u);
+    const __half* src = ring_base + (ok ? (long long)((p0 + row) % ring) * kHeadDim : 0);
+    if (p0 + row == p_new) src = new_row;
+    cp_async16(rows + row * kResRow + piece * 8, src + piece * 8, ok ? 16u : 0u);
   }
   cp_async_wait_all();
   __syncwarp();
@@ -844,16 +848,95 @@ __device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int 
   return pre;
 }
 
+// Decode step with a flush: the 32-token block of positions [p0, p0 + 32),
+// still fp16 in the ring, leaves the window.  One warp quantizes it exactly as
+// kvq_pack does (same quantizer, same page layout) into a page image in
+// `image` (shared memory) and writes the page to `page_out`; the caller folds
+// the image into its state like any streamed block.  Kept out of line: it is
+// rare and its registers would otherwise crowd the streaming loop.
+template <int BK, int BV>
+__device__ __noinline__ void flush_block(const __half* ring_k, const __half* ring_v, int p0,
+                                         int ring, char* image, char* page_out) {
+  constexpr int page = page_bytes_c(BK, BV);
+  const int lane = threadIdx.x & 31;
+  uint32_t* kcodes = reinterpret_cast<uint32_t*>(image);
+  uint32_t* vcodes = reinterpret_cast<uint32_t*>(image + page_off_vcodes(BK));
+  __half* kmeta = reinterpret_cast<__half*>(image + page_off_kmeta(BK));
+  __half* vmeta = reinterpret_cast<__half*>(image + page_off_vmeta(BK, BV));
+  if (BK == 1)
+    for (int i = lane; i < kHeadDim; i += 32) kcodes[i] = 0u;
+  if (BV == 1)
+    for (int i = lane; i < kHeadDim; i += 32) vcodes[i] = 0u;
+  __syncwarp();
+  // keys: lane l quantizes channels 4l .. 4l+3 over the block's 32 tokens
+  for (int cc = 0; cc < 4; ++cc) {
+    const int c = 4 * lane + cc;
+    float x[kGroup];
+#pragma unroll
+    for (int t = 0; t < kGroup; ++t)
+      x[t] = __half2float(ring_k[(long long)((p0 + t) % ring) * kHeadDim + c]);
+    uint32_t w[BK];
+    __half sc, z;
+    quantize_group<BK>(x, w, sc, z);
+    if (BK == 1) {
+#pragma unroll 4
+      for (int t = 0; t < kGroup; ++t) {
+        const int bit = key1_bit(t, c);
+        if ((w[0] >> t) & 1u) atomicOr(&kcodes[bit >> 5], 1u << (bit & 31));
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < BK; ++j) kcodes[c * BK + j] = w[j];
+    }
+    kmeta[c] = sc;
+    kmeta[kHeadDim + c] = z;
+  }
+  // values: lane t quantizes the four 32-channel groups of token t
+  {
+    const int t = lane;
+    const __half* row = ring_v + (long long)((p0 + t) % ring) * kHeadDim;
+    for (int g = 0; g < 4; ++g) {
+      float x[kGroup];
+#pragma unroll
+      for (int i = 0; i < kGroup; ++i) x[i] = __half2float(row[g * kGroup + i]);
+      uint32_t w[BV];
+      __half sc, z;
+      quantize_group<BV>(x, w, sc, z);
+      if (BV == 1) {
+#pragma unroll 4
+        for (int i = 0; i < kGroup; ++i) {
+          const int bit = val1_bit(t, g * kGroup + i);
+          if ((w[0] >> i) & 1u) atomicOr(&vcodes[bit >> 5], 1u << (bit & 31));
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < BV; ++j) vcodes[(g * kGroup + t) * BV + j] = w[j];
+      }
+      vmeta[vmeta_index(g, t)] = sc;
+      vmeta[kHeadDim + vmeta_index(g, t)] = z;
+    }
+  }
+  __syncwarp();
+  for (int i = lane; i < page / 16; i += 32)
+    reinterpret_cast<uint4*>(page_out)[i] = reinterpret_cast<const uint4*>(image)[i];
+  __syncwarp();
+}
+
 // Fold blocks [lo, hi) into st; `pre` slots were streamed early for a range
 // starting at lo_h.
 template <int BK, int BV>
-__device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, int hi,
+__device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, int hi_all,
                                char* ring, uint64_t* full, int R, const char* zero,
                                const __half* qh, int gq, float scale_log2, unsigned* flag,
-                               TcState& st) {
+                               TcState& st, int flush_blk, const __half* ring_k,
+                               const __half* ring_v, int ring_size) {
   constexpr int page = page_bytes_c(BK, BV);
   constexpr int NB = ring_blocks(page);
   const int lane = threadIdx.x & 31;
+  // a block that leaves the window in this kernel has no page yet: it is
+  // quantized from the ring after the streamed ones
+  const bool flush = flush_blk >= lo && flush_blk == hi_all - 1;
+  const int hi = flush ? hi_all - 1 : hi_all;
   const int skip = (pre > 0 && lo == lo_h) ? 0 : pre;
   const int n_units = (hi - lo + NB - 1) / NB;
   const int total = skip + n_units;
@@ -903,13 +986,20 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, 
   if (lane == 0)
     for (int s = max(consumed, issued - R); s < issued; ++s) mbar_wait(full + s % R, (s / R) & 1);
   __syncwarp();
+  if (flush) {
+    flush_block<BK, BV>(ring_k, ring_v, flush_blk * kGroup, ring_size, ring,
+                        const_cast<char*>(pages_bh) + (long long)flush_blk * page);
+    const char* pg[1] = {ring};
+    tc_unit<BK, BV, 1>(pg, zero, qb, ln, scale_log2, st);
+  }
 }
 
 // Window warp: chunks c0, c0 + stride, ... of the fp16 window.
 template <int BK, int BV>
 __device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half* ring_v,
                                const Plan& p, int L, int c0, int stride, char* area,
-                               const __half* qh, int gq, float scale_log2, TcState& st) {
+                               const __half* qh, int gq, float scale_log2, TcState& st,
+                               int p_new, const __half* k_row, const __half* v_row) {
   const int lane = threadIdx.x & 31;
   const Lane ln = make_lane<BK, BV>(lane);
   uint32_t qb[16];
@@ -919,10 +1009,10 @@ __device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half
     const int p0 = p.Lq + u * kGroup;
     const int n_tok = min(kGroup, L - p0);
     uint32_t pt[1][2][2];
-    stage_rows(rows, ring_k, p0, n_tok, d.ring);
+    stage_rows(rows, ring_k, p0, n_tok, d.ring, p_new, k_row);
     tc_resid_scores(rows, n_tok, qb, ln, scale_log2, st, pt);
     __syncwarp();
-    stage_rows(rows, ring_v, p0, n_tok, d.ring);
+    stage_rows(rows, ring_v, p0, n_tok, d.ring, p_new, v_row);
     tc_resid_values(rows, pt, st);
     __syncwarp();
   }
@@ -941,9 +1031,11 @@ __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
 template <int BK, int BV, bool kTc>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     decode_attn_kernel(Dims d, kvq_cache c, const __half* __restrict__ q, float* __restrict__ out,
-                       float scale_log2, int S, unsigned smem_size, Ws ws) {
+                       float scale_log2, int S, unsigned smem_size, Ws ws,
+                       const __half* __restrict__ k_new, const __half* __restrict__ v_new) {
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ MergeSmall ms;
+  __shared__ int len_s[2];  // length attended, length before the append
 
   const int h = blockIdx.y, b = blockIdx.z;
   const int gq = d.gq, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -956,6 +1048,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   const __half* ring_v = reinterpret_cast<const __half*>(c.v_resid) + bh * d.ring * kHeadDim;
   const __half* qh = q + ((long long)b * d.hq + (long long)h * gq) * kHeadDim;
   unsigned* flag = reinterpret_cast<unsigned*>(c.seq_len) + d.batch;
+  // Decode step (k_new given, tensor-core path only): this kernel appends one
+  // token per sequence before attending.  seq_len[b] is read once per CTA;
+  // the last CTA of the sequence to have read it (ticket) publishes L0 + 1.
+  const bool append = kTc && k_new != nullptr;
+  unsigned seq_ticket = 0u;
 
   if constexpr (kTc) {
     constexpr int page = page_bytes_c(BK, BV);
@@ -974,6 +1071,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       hint = read_len(c.seq_len + b);
     }
     hint = __shfl_sync(0xffffffffu, hint, 0);
+    if (append && hint < d.max_len) ++hint;  // the length this kernel will attend
     __syncwarp();
     const Plan ph = make_plan(hint, d.residual, NV);
     int lo_h = 0, hi_h = 0, pre = 0;
@@ -986,8 +1084,32 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     pdl_wait();
     // q (written by the previous kernel) into L1 while the length is read
     if (lane < gq * 2) asm volatile("prefetch.global.L1 [%0];" ::"l"(qh + lane * 64));
-    const int L = read_len(c.seq_len + b);
+    if (threadIdx.x == 0) {
+      const int L0 = read_len(c.seq_len + b);
+      int L = L0;
+      if (append) {
+        if (L0 < d.max_len) L = L0 + 1;
+        else atomicOr(flag, (unsigned)KVQ_FLAG_OVERFLOW);
+      }
+      len_s[0] = L;
+      len_s[1] = L0;
+    }
+    __syncthreads();
+    const int L = len_s[0], L0 = len_s[1];
+    const bool grew = L > L0;  // this kernel appends the token at position L0
+    if (append && threadIdx.x == 0)
+      seq_ticket = atomicAdd(reinterpret_cast<unsigned*>(c.seq_len) + d.batch + 2 + b, 1u);
+    const __half* k_row = grew ? k_new + bh * kHeadDim : nullptr;
+    const __half* v_row = grew ? v_new + bh * kHeadDim : nullptr;
+    if (grew && blockIdx.x == 0 && warp == 0) {  // the new token into its ring slot
+      const long long slot = (long long)(L0 % d.ring) * kHeadDim;
+      __half* rk = const_cast<__half*>(ring_k) + slot;
+      __half* rv = const_cast<__half*>(ring_v) + slot;
+      if (lane < 16) reinterpret_cast<uint4*>(rk)[lane] = reinterpret_cast<const uint4*>(k_row)[lane];
+      else reinterpret_cast<uint4*>(rv)[lane - 16] = reinterpret_cast<const uint4*>(v_row)[lane - 16];
+    }
     const Plan p = make_plan(L, d.residual, NV);
+    const int flush_blk = grew && p.Lq > packed_len(L0, d.residual) ? p.nb - 1 : -1;
     const bool packed = v < p.np;
     TcState st;
     init_state(st);
@@ -996,11 +1118,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       int lo = 0, hi = 0;
       if (packed) block_range(p, v, lo, hi);
       tc_packed_warp<BK, BV>(pages, lo_h, pre, lo, hi, ring, full, R,
-                             reinterpret_cast<const char*>(zero), qh, gq, scale_log2, flag, st);
+                             reinterpret_cast<const char*>(zero), qh, gq, scale_log2, flag, st,
+                             flush_blk, ring_k, ring_v, d.ring);
     }
     if (!packed)
       tc_window_warp<BK, BV>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, qh, gq,
-                             scale_log2, st);
+                             scale_log2, st, grew ? L0 : -1, k_row, v_row);
     // the warp's ring is idle now: its state goes to the start of it
     WarpState& mine = *reinterpret_cast<WarpState*>(ring);
     if (packed) tc_write_state<true, BV>(st, mine, lane);
@@ -1084,6 +1207,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         ws.l[row] = l;
       }
     }
+  }
+  if (append && threadIdx.x == 0 &&
+      seq_ticket == (unsigned)(d.hkv * gridDim.x) - 1u) {  // every CTA of b has read L0
+    const int L1 = len_s[0];
+    __threadfence();
+    c.seq_len[b] = L1;
+    reinterpret_cast<unsigned*>(c.seq_len)[d.batch + 2 + b] = 0u;
   }
   if (S == 1) return;
 
@@ -1202,6 +1332,8 @@ struct LaunchOp {
   int S;
   const Ws& ws;
   cudaStream_t st;
+  const __half* k_new = nullptr;
+  const __half* v_new = nullptr;
   template <int BK, int BV, bool kTc>
   cudaError_t run() const {
     cudaError_t e = prepare<BK, BV, kTc>(d);
@@ -1217,7 +1349,7 @@ struct LaunchOp {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV, kTc>, d, c, q, out, sl2, S,
-                           (unsigned)smem_bytes(d, kTc), ws);
+                           (unsigned)smem_bytes(d, kTc), ws, k_new, v_new);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
@@ -1237,6 +1369,16 @@ cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& c, const __half* 
                                float scale_log2, int n_splits, void* workspace, cudaStream_t st) {
   const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, n_splits);
   return dispatch(d, LaunchOp{d, c, q, out, scale_log2, n_splits, ws, st});
+}
+
+cudaError_t launch_decode_step(const Dims& d, const kvq_cache& c, const __half* k_new,
+                               const __half* v_new, const __half* q, float* out,
+                               float scale_log2, int n_splits, void* workspace, cudaStream_t st) {
+  const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, n_splits);
+  LaunchOp op{d, c, q, out, scale_log2, n_splits, ws, st};
+  op.k_new = k_new;
+  op.v_new = v_new;
+  return dispatch(d, op);
 }
 
 // CTAs per (sequence, kv-head): enough for every resident CTA slot of the

@@ -54,6 +54,41 @@ __host__ __device__ inline int vmeta_index(int g, int t) {
   return 32 * g + 8 * (t >> 3) + 2 * (t & 3) + ((t >> 2) & 1);
 }
 
+// The KbVb quantizer of one 32-element group (Sec. 3.1), each step one IEEE
+// float32 operation with the stated rounding:
+//   zero  = min x                                   (exact, fp16)
+//   scale = RU16(RU32(RU32(max x - min x) / levels)) (stored fp16)
+//   code  = clamp(rint(RN32(RN32(x - zero) / scale)), 0, levels); 0 if scale == 0
+// Codes fill B little-endian words, element i at bits [(i*B) % 32, +B) of
+// word (i*B) / 32.  Used by kvq_pack and by the decode step's flush.
+template <int B>
+__device__ __forceinline__ void quantize_group(const float (&x)[kGroup], uint32_t (&w)[B],
+                                               __half& scale, __half& zero) {
+  constexpr float kLevels = float((1 << B) - 1);
+  float lo = x[0], hi = x[0];
+#pragma unroll
+  for (int i = 1; i < kGroup; ++i) {
+    lo = fminf(lo, x[i]);
+    hi = fmaxf(hi, x[i]);
+  }
+  const __half s_h = __float2half_ru(__fdiv_ru(__fsub_ru(hi, lo), kLevels));
+  const float s = __half2float(s_h);
+#pragma unroll
+  for (int j = 0; j < B; ++j) w[j] = 0u;
+#pragma unroll
+  for (int i = 0; i < kGroup; ++i) {
+    uint32_t c = 0u;
+    if (s > 0.0f) {
+      float t = rintf(__fdiv_rn(__fsub_rn(x[i], lo), s));
+      t = fminf(fmaxf(t, 0.0f), kLevels);
+      c = (uint32_t)t;
+    }
+    w[(i * B) / 32] |= c << ((i * B) % 32);
+  }
+  scale = s_h;
+  zero = __float2half_rn(lo);  // lo is an fp16 value: exact
+}
+
 // Tokens held in quantized blocks when L tokens are cached.
 __host__ __device__ inline int packed_len(int L, int residual) {
   int over = L - residual;
@@ -92,6 +127,12 @@ cudaError_t launch_pack(const Dims& d, const kvq_cache& cache, const __half* k_n
 cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& cache, const __half* q,
                                float* out, float scale_log2, int n_splits,
                                void* workspace, cudaStream_t stream);
+// Append one token per sequence (k_new / v_new [batch][n_kv_heads][128]) and
+// attend in the same kernel (query groups up to 4).
+cudaError_t launch_decode_step(const Dims& d, const kvq_cache& cache, const __half* k_new,
+                               const __half* v_new, const __half* q, float* out,
+                               float scale_log2, int n_splits, void* workspace,
+                               cudaStream_t stream);
 size_t attn_workspace_bytes(const Dims& d, int n_splits);
 int attn_default_splits(const Dims& d, int sm_count);
 size_t attn_static_scratch_bytes();

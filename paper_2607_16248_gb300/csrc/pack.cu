@@ -26,35 +26,6 @@ struct Tile {
   uint32_t v1[kHeadDim];  // 1-bit value codes in fragment order
 };
 
-// Quantize the 32 values x[] and return the packed words, scale and zero.
-template <int B>
-__device__ __forceinline__ void quantize_group(const float (&x)[kGroup], uint32_t (&w)[B],
-                                               __half& scale, __half& zero) {
-  constexpr float kLevels = float((1 << B) - 1);
-  float lo = x[0], hi = x[0];
-#pragma unroll
-  for (int i = 1; i < kGroup; ++i) {
-    lo = fminf(lo, x[i]);
-    hi = fmaxf(hi, x[i]);
-  }
-  const __half s_h = __float2half_ru(__fdiv_ru(__fsub_ru(hi, lo), kLevels));
-  const float s = __half2float(s_h);
-#pragma unroll
-  for (int j = 0; j < B; ++j) w[j] = 0u;
-#pragma unroll
-  for (int i = 0; i < kGroup; ++i) {
-    uint32_t c = 0u;
-    if (s > 0.0f) {
-      float t = rintf(__fdiv_rn(__fsub_rn(x[i], lo), s));
-      t = fminf(fmaxf(t, 0.0f), kLevels);
-      c = (uint32_t)t;
-    }
-    w[(i * B) / 32] |= c << ((i * B) % 32);
-  }
-  scale = s_h;
-  zero = __float2half_rn(lo);  // lo is an fp16 value: exact
-}
-
 template <int B>
 __device__ __forceinline__ void store_words(uint32_t* dst, const uint32_t (&w)[B]) {
 #pragma unroll

@@ -25,7 +25,8 @@ EXPORTS = (
     "kvq_last_error", "kvq_version", "kvq_validate_config", "kvq_page_bytes",
     "kvq_cache_layout", "kvq_cache_bind", "kvq_cache_reset", "kvq_pack",
     "kvq_attn_workspace_bytes", "kvq_attn_default_splits", "kvq_workspace_init",
-    "kvq_decode_attn", "kvq_decode_attn_noalloc", "dgap_workspace_bytes", "dgap_restore",
+    "kvq_decode_attn", "kvq_decode_step", "kvq_decode_attn_noalloc", "dgap_workspace_bytes",
+    "dgap_restore",
 )
 NOALLOC_SCRATCH_BYTES = 4 << 20
 
@@ -78,6 +79,7 @@ def lib():
             "kvq_attn_default_splits": (I32, [cfg_p]),
             "kvq_workspace_init": (I32, [P, SZ, P]),
             "kvq_decode_attn": (I32, [cfg_p, cache_p, P, P, F32, I32, P, SZ, P]),
+            "kvq_decode_step": (I32, [cfg_p, cache_p, P, P, P, P, F32, I32, P, SZ, P]),
             "kvq_decode_attn_noalloc": (I32, [cfg_p, cache_p, P, P, F32, I32, P]),
             "dgap_workspace_bytes": (SZ, [I32, I32, par_p]),
             "dgap_restore": (I32, [par_p, P, I32, I32, P, P, P, P, P, P, P, SZ, P]),
@@ -250,6 +252,32 @@ def kvq_decode_attn(cache: QuantKVCache, q, out=None, softmax_scale=0.0, n_split
         workspace = attn_workspace(cfg, n_splits, q.device)
     c = cfg.c()
     _check(lib().kvq_decode_attn(ctypes.byref(c), ctypes.byref(cache._c),
+                                 _dev(q, torch.float16, "q"), _dev(out, torch.float32, "out"),
+                                 float(softmax_scale), n_splits,
+                                 _dev(workspace, torch.uint8, "workspace"), workspace.numel(),
+                                 _stream(stream)))
+    return out
+
+
+def kvq_decode_step(cache: QuantKVCache, k_new, v_new, q, out=None, softmax_scale=0.0,
+                    n_splits=0, workspace=None, stream=None):
+    """Append one token per sequence (k_new / v_new fp16 [batch, n_kv_heads, 128])
+    and attend (q fp16 [batch, n_q_heads, 128] -> out fp32) in one call: the
+    same results as kvq_pack then kvq_decode_attn."""
+    cfg = cache.cfg
+    if q.shape != (cfg.batch, cfg.n_q_heads, cfg.head_dim):
+        raise ValueError(f"q must be [{cfg.batch}, {cfg.n_q_heads}, {cfg.head_dim}]")
+    for name, t in (("k_new", k_new), ("v_new", v_new)):
+        if t.shape != (cfg.batch, cfg.n_kv_heads, cfg.head_dim):
+            raise ValueError(f"{name} must be [{cfg.batch}, {cfg.n_kv_heads}, {cfg.head_dim}]")
+    if out is None:
+        out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+    if workspace is None:
+        workspace = attn_workspace(cfg, n_splits, q.device)
+    c = cfg.c()
+    _check(lib().kvq_decode_step(ctypes.byref(c), ctypes.byref(cache._c),
+                                 _dev(k_new, torch.float16, "k_new"),
+                                 _dev(v_new, torch.float16, "v_new"),
                                  _dev(q, torch.float16, "q"), _dev(out, torch.float32, "out"),
                                  float(softmax_scale), n_splits,
                                  _dev(workspace, torch.uint8, "workspace"), workspace.numel(),
