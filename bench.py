@@ -290,9 +290,9 @@ def reduce_max(x, world):
 
 
 class Step:
-    """Caches, inputs, workspaces and the captured graphs of a step: the whole
-    step (per layer kvq_pack then kvq_decode_attn, then the logits and
-    dgap_restore), the step without dgap_restore, and each phase alone."""
+    """Caches, inputs, workspaces and the captured graphs: the whole step (per
+    layer kvq_decode_step, which appends the token and attends, then the
+    logits and dgap_restore), the decode steps alone, and the epilogue."""
 
     def __init__(self, spec, steps_total, device, rank):
         import torch
@@ -322,8 +322,8 @@ class Step:
         self.seq0 = [c.seq_region().clone() for c in self.caches]
         g = synth.generator(seed + 1, device)
         self.q = torch.randn(layers, B, hq, 128, generator=g, device=device).half()
-        self.k_new = torch.randn(layers, B, hkv, 1, 128, generator=g, device=device).half()
-        self.v_new = torch.randn(layers, B, hkv, 1, 128, generator=g, device=device).half()
+        self.k_new = torch.randn(layers, B, hkv, 128, generator=g, device=device).half()
+        self.v_new = torch.randn(layers, B, hkv, 128, generator=g, device=device).half()
         self.out = torch.empty(layers, B, hq, 128, dtype=torch.float32, device=device)
         self.ws_attn = kvq.attn_workspace(self.cfg, 0, device)
         self.n_splits = kvq.default_splits(self.cfg)
@@ -362,34 +362,31 @@ class Step:
         import torch
         L = self.spec["layers"]
 
-        def pack(l):
-            kvq.kvq_pack(self.caches[l], self.k_new[l], self.v_new[l])
-
-        def attn(l):
-            kvq.kvq_decode_attn(self.caches[l], self.q[l], out=self.out[l],
-                                n_splits=self.n_splits, workspace=self.ws_attn)
+        def layer(l):
+            kvq.kvq_decode_step(self.caches[l], self.k_new[l], self.v_new[l], self.q[l],
+                                out=self.out[l], n_splits=self.n_splits,
+                                workspace=self.ws_attn)
 
         def epilogue():
             self.dgap.restore(self.logits, outputs=self.dout, workspace=self.ws_dgap)
 
-        self.g_step, self.g_step_nd, self.g_pack, self.g_attn, self.g_dgap = (
-            torch.cuda.CUDAGraph() for _ in range(5))
-        for g, with_dgap in ((self.g_step, True), (self.g_step_nd, False)):
-            with torch.cuda.graph(g):
-                for l in range(L):
-                    pack(l)
-                    attn(l)
-                self.logits.copy_(self.logits0)  # stands in for the LM head's output
-                if with_dgap:
-                    epilogue()
-        with torch.cuda.graph(self.g_pack):
+        self.g_step, self.g_attn, self.g_epi10, self.g_copy10 = (
+            torch.cuda.CUDAGraph() for _ in range(4))
+        with torch.cuda.graph(self.g_step):
             for l in range(L):
-                pack(l)
+                layer(l)
+            self.logits.copy_(self.logits0)  # stands in for the LM head's output
+            epilogue()
         with torch.cuda.graph(self.g_attn):
             for l in range(L):
-                attn(l)
-        with torch.cuda.graph(self.g_dgap):
-            epilogue()
+                layer(l)
+        with torch.cuda.graph(self.g_epi10):
+            for _ in range(10):
+                self.logits.copy_(self.logits0)
+                epilogue()
+        with torch.cuda.graph(self.g_copy10):
+            for _ in range(10):
+                self.logits.copy_(self.logits0)
         torch.cuda.synchronize()
 
     def rewind(self):
@@ -400,7 +397,7 @@ class Step:
             c.seq_region().copy_(s0)
 
     def launches_per_step(self):
-        return 2 * self.spec["layers"] + 1
+        return self.spec["layers"] + 1
 
     def bytes_for_step(self, step_index):
         """Attention bytes of the step whose pack made sequences L0 + i + 1 long."""
@@ -417,9 +414,9 @@ def run_gpu(args, spec):
     device = torch.device("cuda", local if world > 1 else 0)
     K, W = args.steps, args.warmup
     e2e_on = not args.no_e2e
-    # Each measurement (the headline, the step without the epilogue, the
-    # phases alone, the end-to-end run) replays W warm-up + K timed steps from
-    # the prefill lengths (Step.rewind).
+    # Each measurement (the headline, the decode-step kernels alone, the
+    # end-to-end run) replays W + K steps from the prefill lengths
+    # (Step.rewind).
     total_steps = W + K
     st = Step(spec, total_steps, device, rank)
     done = 0  # steps replayed since the last rewind (each appends one token)
@@ -460,37 +457,29 @@ def run_gpu(args, spec):
     step_bytes = [st.bytes_for_step(step0 + i) for i in range(K)]
     bytes_total = sum(step_bytes)
 
-    # The epilogue's share of a step: the same steps without dgap_restore.
+    # The epilogue: 10 x (logits copy, dgap_restore) against 10 x (logits copy)
+    # in one graph each, replays alternated.
+    for _ in range(W):
+        st.g_epi10.replay()
+        st.g_copy10.replay()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    torch.cuda.synchronize()
+    for e in evs:
+        e[0].record()
+        st.g_epi10.replay()
+        e[1].record()
+        st.g_copy10.replay()
+        e[2].record()
+    torch.cuda.synchronize()
+    with_ms = sum(e[0].elapsed_time(e[1]) for e in evs)
+    without_ms = sum(e[1].elapsed_time(e[2]) for e in evs)
+    epi_ms = reduce_max(max(with_ms - without_ms, 0.0) / 10.0, world)
+
+    # The decode-step kernels alone: the 32 launches of a step, one graph.
     st.rewind()
     done = 0
-    nd_ms = timed(st.g_step_nd.replay, W, K)
-    epi_ms = max(total_ms - nd_ms, 0.0)
-
-    # Phase breakdown: each phase's graph alone (one graph launch per step).
-    def phases():
-        st.g_pack.replay()
-        ev[0].record()
-        st.g_attn.replay()
-        ev[1].record()
-        st.logits.copy_(st.logits0)
-        st.g_dgap.replay()
-
-    st.rewind()
-    done = 0
-    attn_ms = 0.0
-    pack_ms = 0.0
     ph_step0 = done + W
-    for i in range(W + K):
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-        e0 = torch.cuda.Event(enable_timing=True)
-        e0.record()
-        phases()
-        torch.cuda.synchronize()
-        if i >= W:
-            pack_ms += e0.elapsed_time(ev[0])
-            attn_ms += ev[0].elapsed_time(ev[1])
-    done += W + K
-    attn_ms = reduce_max(attn_ms, world)
+    attn_ms = timed(st.g_attn.replay, W, K)
     attn_bytes_total = sum(st.bytes_for_step(ph_step0 + i) for i in range(K))
 
     value = world * bytes_total / (total_ms * 1e-3) / 1e9
@@ -517,8 +506,8 @@ def run_gpu(args, spec):
            "n_splits": st.n_splits,
            "l2": f"inputs larger than L2: {step_bytes[0] / 1e6:.0f} MB of packed KV read per "
                  f"step (distinct cache per layer), L2 129 MB",
-           "step": f"{s['layers']} x (kvq_pack, kvq_decode_attn) + logits copy + dgap_restore, "
-                   f"one CUDA graph per step", "parallelism": f"replicas x{world}" if world > 1 else "1 GPU"}
+           "step": f"{s['layers']} x kvq_decode_step (append + attention) + logits copy + "
+                   f"dgap_restore, one CUDA graph per step", "parallelism": f"replicas x{world}" if world > 1 else "1 GPU"}
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": round(total_ms / K, 5),
@@ -529,11 +518,11 @@ def run_gpu(args, spec):
         "attn_gbs": round(achieved, 2),
         "attn_frac_of_peak": round(achieved / peak, 4),
         "attn_us_per_layer": round(attn_ms / attn_launches * 1e3, 3),
-        "pack_us_per_step": round(pack_ms / K * 1e3, 3),
         "epilogue_us_per_step": round(epi_ms / K * 1e3, 3),
         "epilogue_frac_of_step_attn": round(epi_ms / attn_ms, 5),
-        "breakdown": "attn_us_per_layer / pack_us_per_step: each phase's graph alone; "
-                     "epilogue_us_per_step: step graph minus the same graph without dgap_restore",
+        "breakdown": "attn_us_per_layer: the step's kvq_decode_step launches (append + "
+                     "attention) alone in one graph; epilogue_us_per_step: a graph of 10 x (logits "
+                     "copy, dgap_restore) minus one of 10 x (logits copy), per call",
         "gated_rows_fraction": float(st.dout["gate"].float().mean().item()),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4),
