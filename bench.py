@@ -280,13 +280,21 @@ def barrier(world):
 
 
 def reduce_max(x, world):
+    """Largest x over the ranks (the job's time is its slowest rank's)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_gbs(world, bytes_per_rank, ms_max):
+    """Whole-job throughput: every rank moved bytes_per_rank (weak scaling,
+    identical replicas) in the slowest rank's time."""
+    return world * bytes_per_rank / (ms_max * 1e-3) / 1e9
 
 
 class Step:
@@ -482,7 +490,7 @@ def run_gpu(args, spec):
     attn_ms = timed(st.g_attn.replay, W, K)
     attn_bytes_total = sum(st.bytes_for_step(ph_step0 + i) for i in range(K))
 
-    value = world * bytes_total / (total_ms * 1e-3) / 1e9
+    value = job_gbs(world, bytes_total, total_ms)
     launches = K * st.launches_per_step()
     attn_launches = K * spec["layers"]
     achieved = attn_bytes_total / (attn_ms * 1e-3) / 1e9

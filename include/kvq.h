@@ -44,7 +44,9 @@ typedef enum kvq_status {
 } kvq_status;
 
 /* Device-side flag bits (cache flag word). */
-#define KVQ_FLAG_OVERFLOW 1u /* a kvq_pack would have passed max_len */
+#define KVQ_FLAG_OVERFLOW 1u /* an append would have passed max_len */
+#define KVQ_FLAG_WAIT_TIMEOUT 2u /* an attention kernel's copy wait gave up (~2 s);
+                                    its output for that call is not valid */
 
 /*
  * Cache configuration.  KbVb with b_k = bits_k and b_v = bits_v (Sec. 3.1

@@ -957,7 +957,7 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, 
     const int slot = s % R;
     // every lane waits; the warp leaves together if any lane gave up
     if (!__all_sync(0xffffffffu, mbar_wait(full + slot, (s / R) & 1))) {
-      if (lane == 0) atomicOr(flag, 2u);
+      if (lane == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
       break;
     }
     consumed = s + 1;

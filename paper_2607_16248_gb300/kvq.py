@@ -19,6 +19,7 @@ _lib = None
 STATUS_NAMES = {0: "KVQ_OK", 1: "KVQ_ERR_ARG", 2: "KVQ_ERR_SHAPE", 3: "KVQ_ERR_UNSUPPORTED",
                 4: "KVQ_ERR_CAPACITY", 5: "KVQ_ERR_ALIGN", 6: "KVQ_ERR_CUDA"}
 FLAG_OVERFLOW = 1
+FLAG_WAIT_TIMEOUT = 2
 
 # Every symbol include/kvq.h declares.
 EXPORTS = (
