@@ -711,29 +711,6 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t 
                "r"(src_bytes)
                : "memory");
 }
-__device__ __forceinline__ void cp_async_wait_all() {
-  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
-}
-
-// Copy rows p0 .. p0 + 31 of one (sequence, kv-head) ring (fp16 [ring][128])
-// into `rows` ([32][kResRow]); rows at or past n_tok are zero-filled.  The row
-// of position p_new (a token appended by this kernel, not yet in the ring)
-// comes from new_row instead.
-__device__ __forceinline__ void stage_rows(__half* rows, const __half* ring_base, int p0, int n_tok,
-                                           int ring, int p_new = -1,
-                                           const __half* new_row = nullptr) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll 4
-  for (int e = lane; e < kGroup * 16; e += 32) {
-    const int row = e >> 4, piece = e & 15;
-    const bool ok = row < n_tok;
-    const __half* src = ring_base + (ok ? (long long)((p0 + row) % ring) * kHeadDim : 0);
-    if (p0 + row == p_new) src = new_row;
-    cp_async16(rows + row * kResRow + piece * 8, src + piece * 8, ok ? 16u : 0u);
-  }
-  cp_async_wait_all();
-  __syncwarp();
-}
 
 __device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
                                                 const uint32_t (&qb)[16], const Lane& ln,
@@ -994,25 +971,77 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, 
   }
 }
 
+// Copy rows p0 .. p0 + 31 into padded `rows` with one bulk copy per row
+// (issued by the row's lane, completing on `bar`); rows at or past n_tok are
+// zeroed.  The row of position p_new comes from new_row.  Returns false if
+// the bounded wait gave up.
+__device__ __forceinline__ bool stage_rows_bulk(__half* rows, const __half* ring_base, int p0,
+                                                int n_tok, int ring, int p_new,
+                                                const __half* new_row, uint64_t* bar,
+                                                uint32_t parity) {
+  const int lane = threadIdx.x & 31;
+  __syncwarp();
+  if (lane >= n_tok) {
+    uint4* r = reinterpret_cast<uint4*>(rows + lane * kResRow);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) r[i] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  if (lane == 0) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    mbar_expect_tx(bar, (uint32_t)(n_tok * kHeadDim * 2));
+  }
+  __syncwarp();
+  if (lane < n_tok) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    const __half* src = p0 + lane == p_new ? new_row
+                                           : ring_base + (long long)((p0 + lane) % ring) * kHeadDim;
+    bulk_g2s(rows + lane * kResRow, src, kHeadDim * 2, bar);
+  }
+  const bool ok = __all_sync(0xffffffffu, mbar_wait(bar, parity));
+  __syncwarp();
+  return ok;
+}
+
+// Bring ring rows [p0, p0 + n) (one or two contiguous runs) into L2.
+__device__ __forceinline__ void prefetch_rows_l2(const __half* ring_base, int p0, int n, int ring) {
+  const int s0 = p0 % ring;
+  const int n1 = min(n, ring - s0);
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ring_base + (long long)s0 * kHeadDim),
+               "r"((uint32_t)(n1 * kHeadDim * 2))
+               : "memory");
+  if (n > n1)
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ring_base),
+                 "r"((uint32_t)((n - n1) * kHeadDim * 2))
+                 : "memory");
+}
+
 // Window warp: chunks c0, c0 + stride, ... of the fp16 window.
 template <int BK, int BV>
 __device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half* ring_v,
                                const Plan& p, int L, int c0, int stride, char* area,
                                const __half* qh, int gq, float scale_log2, TcState& st,
-                               int p_new, const __half* k_row, const __half* v_row) {
+                               int p_new, const __half* k_row, const __half* v_row,
+                               uint64_t* bar, unsigned* flag) {
   const int lane = threadIdx.x & 31;
   const Lane ln = make_lane<BK, BV>(lane);
   uint32_t qb[16];
   load_qb<false>(qb, qh, gq, ln);
   __half* rows = reinterpret_cast<__half*>(area);
+  uint32_t phase = 0u;
   for (int u = c0; u < p.n_res; u += stride) {
     const int p0 = p.Lq + u * kGroup;
     const int n_tok = min(kGroup, L - p0);
     uint32_t pt[1][2][2];
-    stage_rows(rows, ring_k, p0, n_tok, d.ring, p_new, k_row);
+    if (!stage_rows_bulk(rows, ring_k, p0, n_tok, d.ring, p_new, k_row, bar, phase++ & 1u)) {
+      if ((threadIdx.x & 31) == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
+      return;
+    }
     tc_resid_scores(rows, n_tok, qb, ln, scale_log2, st, pt);
     __syncwarp();
-    stage_rows(rows, ring_v, p0, n_tok, d.ring, p_new, v_row);
+    if (!stage_rows_bulk(rows, ring_v, p0, n_tok, d.ring, p_new, v_row, bar, phase++ & 1u)) {
+      if ((threadIdx.x & 31) == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
+      return;
+    }
     tc_resid_values(rows, pt, st);
     __syncwarp();
   }
@@ -1036,6 +1065,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ MergeSmall ms;
   __shared__ int len_s[2];  // length attended, length before the append
+  __shared__ __align__(16) __half q_s[4 * kHeadDim];  // tensor-core path: the query group
+  __shared__ __align__(8) uint64_t wbar[kWarps];      // a window warp's staging barrier
 
   const int h = blockIdx.y, b = blockIdx.z;
   const int gq = d.gq, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1067,6 +1098,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     int hint = 0;
     if (lane == 0) {
       for (int i = 0; i < R; ++i) mbar_init(full + i, 1);
+      mbar_init(&wbar[warp], 1);
       fence_mbar_init();
       hint = read_len(c.seq_len + b);
     }
@@ -1079,11 +1111,26 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       block_range(ph, v, lo_h, hi_h);
       // the newest block may be the one the previous kernel is writing
       pre = tc_pre_issue<BK, BV>(pages, lo_h, min(hi_h, ph.nb - 1), ring, full, R);
+    } else if (lane == 0) {
+      // window rows of the length read before the wait into L2 (rows below
+      // the newest token do not change; this is a hint, nothing waits on it)
+      const int last = hint - (append ? 1 : 0) - 1;  // newest row not yet written
+      for (int u = v - ph.np; u < ph.n_res; u += ph.n_resw) {
+        const int p0 = ph.Lq + u * kGroup;
+        const int n = min(kGroup, last - p0);
+        if (n > 0) {
+          prefetch_rows_l2(ring_k, p0, n, d.ring);
+          prefetch_rows_l2(ring_v, p0, n, d.ring);
+        }
+      }
     }
     __syncthreads();  // zero rows written
     pdl_wait();
-    // q (written by the previous kernel) into L1 while the length is read
-    if (lane < gq * 2) asm volatile("prefetch.global.L1 [%0];" ::"l"(qh + lane * 64));
+    // q (written by the previous kernel) into shared memory while the length
+    // is read: one round trip for both
+    if (threadIdx.x < gq * kHeadDim / 8)
+      cp_async16(q_s + threadIdx.x * 8, qh + threadIdx.x * 8, 16u);
+    asm volatile("cp.async.commit_group;" ::: "memory");
     if (threadIdx.x == 0) {
       const int L0 = read_len(c.seq_len + b);
       int L = L0;
@@ -1094,6 +1141,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       len_s[0] = L;
       len_s[1] = L0;
     }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
     __syncthreads();
     const int L = len_s[0], L0 = len_s[1];
     const bool grew = L > L0;  // this kernel appends the token at position L0
@@ -1118,12 +1166,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       int lo = 0, hi = 0;
       if (packed) block_range(p, v, lo, hi);
       tc_packed_warp<BK, BV>(pages, lo_h, pre, lo, hi, ring, full, R,
-                             reinterpret_cast<const char*>(zero), qh, gq, scale_log2, flag, st,
+                             reinterpret_cast<const char*>(zero), q_s, gq, scale_log2, flag, st,
                              flush_blk, ring_k, ring_v, d.ring);
     }
     if (!packed)
-      tc_window_warp<BK, BV>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, qh, gq,
-                             scale_log2, st, grew ? L0 : -1, k_row, v_row);
+      tc_window_warp<BK, BV>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, q_s, gq,
+                             scale_log2, st, grew ? L0 : -1, k_row, v_row, &wbar[warp], flag);
     // the warp's ring is idle now: its state goes to the start of it
     WarpState& mine = *reinterpret_cast<WarpState*>(ring);
     if (packed) tc_write_state<true, BV>(st, mine, lane);
