@@ -562,6 +562,19 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
     const uint4 z8 = *reinterpret_cast<const uint4*>(vzrow + 2 * (kHeadDim + 32 * (gid & 3) + 8 * tig));
     mma16816(st.zv, z8.x, 0u, z8.y, 0u, pt[bi][0][0], pt[bi][0][1]);
     mma16816(st.zv, z8.z, 0u, z8.w, 0u, pt[bi][1][0], pt[bi][1][1]);
+    // B = p * s in two fp16 parts, columns 0..3 and 4..7: the high part is
+    // RN16(p_hi s); the low part RN16(p_lo s + (p_hi s - RN16(p_hi s))), so
+    // rounding the product costs no accuracy.  Lanes of columns 4..7 hold p_lo
+    // after movmatrix and fetch p_hi from lane - 16.
+    uint32_t pa[2][2], pb[2][2];
+#pragma unroll
+    for (int ks = 0; ks < 2; ++ks)
+#pragma unroll
+      for (int dl = 0; dl < 2; ++dl) {
+        const uint32_t other = __shfl_xor_sync(0xffffffffu, pt[bi][ks][dl], 16);
+        pa[ks][dl] = lane < 16 ? pt[bi][ks][dl] : other;
+        pb[ks][dl] = lane < 16 ? 0u : pt[bi][ks][dl];
+      }
     uint4 vw1;
     if constexpr (BV == 1) vw1 = *reinterpret_cast<const uint4*>(vc + 16 * lane);
 #pragma unroll
@@ -587,7 +600,10 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
           am0[2 * dl + 1] = v[1];
           am1[2 * dl] = v[2];
           am1[2 * dl + 1] = v[3];
-          bv[dl] = h2u(__hmul2(u2h(pt[bi][ks][dl]), u2h(mw[ia])));
+          const __half2 sc = u2h(mw[ia]);
+          const __half2 t = __hmul2(u2h(pa[ks][dl]), sc);
+          const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hmul2(t, u2h(ln.neg_lo)));
+          bv[dl] = h2u(__hfma2(u2h(pb[ks][dl]), sc, err));
         }
         mma16816(st.acc[2 * g], am0[0], am0[1], am0[2], am0[3], bv[0], bv[1]);
         mma16816(st.acc[2 * g + 1], am1[0], am1[1], am1[2], am1[3], bv[0], bv[1]);
