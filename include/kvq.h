@@ -166,15 +166,16 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache,
 /*
  * Split-K workspace for kvq_decode_attn: per (sequence, query head, split)
  * partial max, sum and fp32 output row for up to n_splits + 1 splits, plus
- * one ticket per (sequence, kv-head).  n_splits = 0 means the library's
- * choice.  Returns 0 on an invalid config.
+ * one ticket per (sequence, kv-head, head group), sized one per query head.
+ * n_splits = 0 means the library's choice.  Returns 0 on an invalid config.
  */
 size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits);
 
 /*
  * The split count kvq_decode_attn uses when passed n_splits = 0: one
- * 512-thread CTA per SM over all (sequence, kv-head) pairs,
- * SMs / (batch * n_kv_heads), between 1 and 255.
+ * 512-thread CTA per SM over all (sequence, kv-head, head group) triples,
+ * SMs / (batch * n_kv_heads * ceil(group / 4)), between 1 and 255, where
+ * group = n_q_heads / n_kv_heads.
  */
 int32_t kvq_attn_default_splits(const kvq_config* cfg);
 
@@ -196,8 +197,11 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream);
  *                  fp32 accumulation result; rounding it to fp16 is left to
  *                  the caller).
  *   softmax_scale  0 selects 1/sqrt(128).
- *   n_splits       CTAs per (sequence, kv-head) that share its 32-token
- *                  blocks and window chunks; 0 = kvq_attn_default_splits(cfg);
+ *   n_splits       CTAs per (sequence, kv-head, head group) that share the
+ *                  kv-head's 32-token blocks and window chunks (a head group
+ *                  is a run of at most 4 query heads of one kv-head; a group
+ *                  of 5..8 heads has two, whose CTAs read the same pages);
+ *                  0 = kvq_attn_default_splits(cfg);
  *                  else 1..255.  With more than one, each CTA writes a partial
  *                  (max, sum, output row) to the workspace and the last to
  *                  finish merges them.
@@ -218,8 +222,7 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache,
  * k_new / v_new directly and written to its window slot; when it pushes a
  * 32-token group out of the window, that group is quantized (bit-identical to
  * kvq_pack) into its page and attended in quantized form; seq_len[b] becomes
- * L + 1 when the kernel ends.  Query groups wider than 4 run kvq_pack's kernel
- * and then the attention kernel.
+ * L + 1 when the kernel ends.
  *   k_new, v_new   device fp16 [batch][n_kv_heads][128], 16-byte aligned.
  *   q, out, softmax_scale, n_splits, workspace, ws_bytes: as kvq_decode_attn.
  * A sequence at max_len is not appended (KVQ_FLAG_OVERFLOW is set) and

@@ -269,11 +269,6 @@ kvq_status kvq_decode_step(const kvq_config* cfg, const kvq_cache* cache, const 
   const __half* kn = reinterpret_cast<const __half*>(k_new);
   const __half* vn = reinterpret_cast<const __half*>(v_new);
   const __half* qh = reinterpret_cast<const __half*>(q);
-  if (d.gq > 4) {  // the SIMT attention path: the append runs as its own kernel
-    cudaError_t e = launch_pack(d, *cache, kn, vn, 1, 0, d.batch, st);
-    if (e == cudaSuccess) e = launch_decode_attn(d, *cache, qh, out, scale_log2, n_splits, workspace, st);
-    return cuda_status(e, "kvq_decode_step launch");
-  }
   return cuda_status(launch_decode_step(d, *cache, kn, vn, qh, out, scale_log2, n_splits,
                                         workspace, st),
                      "kvq_decode_step launch");

@@ -1,15 +1,19 @@
 // kvq_decode_attn: one decode step of grouped-query attention
 // softmax(q K^T * scale) V (Sec. 1 of the paper) over the packed KbVb cache.
 //
-// Grid (S, n_kv_heads, batch) of 512-thread CTAs, one per SM.  The S CTAs
-// of one (sequence, kv-head) share its work: the packed 32-token blocks and
+// Grid (S, n_kv_heads * G, batch) of 512-thread CTAs, one per SM, where G =
+// ceil(group / 4): the query heads of a kv-head are cut into G head groups of
+// at most 4 (the MMA's head columns) and each head group has its own S CTAs.
+// The G CTA sets of a kv-head are launched next to each other and stream the
+// same pages at the same time, so all but one read of a page come from L2.
+// The S CTAs of one (sequence, kv-head, head group) share its work: the packed 32-token blocks and
 // the 32-token chunks of the fp16 residual window are cut into contiguous
 // ranges, one per warp (a warp takes only blocks or only window chunks).
 // Each warp streams its own pages into a private ring of shared-memory slots
 // with bulk asynchronous copies (cp.async.bulk + one mbarrier per slot) and
 // keeps a running softmax state.  The warps of a CTA merge in shared memory
 // into one partial (max, sum, unnormalised row) per query head; with S > 1
-// the last CTA of a (sequence, kv-head) to finish (atomic ticket, no
+// the last CTA of a (sequence, kv-head, head group) to finish (atomic ticket, no
 // waiting) merges the S partials:
 //   out = sum_s 2^{m_s - M} o_s / sum_s 2^{m_s - M} l_s.
 // Scores are kept in the log2 domain (scaled by softmax_scale * log2 e).
@@ -33,8 +37,7 @@
 // wider codes the code is OR-ed into the mantissa of 1024 and 1024 is
 // subtracted.  The resulting per-row power-of-two factors are undone on the
 // fp32 results.  The fp16 residual window takes the same MMAs with operands
-// loaded by ldmatrix from rows staged in shared memory.  Query-head groups
-// wider than 4 use the SIMT path for every unit.
+// loaded by ldmatrix from rows staged in shared memory.
 
 #include <float.h>
 
@@ -52,6 +55,10 @@ constexpr int kWarps = KVQ_ATTN_WARPS;            // warps per CTA
 constexpr int kThreads = 32 * kWarps;
 constexpr int kCtasPerSm = kWarps <= 8 ? 2 : 1;   // resident CTAs per SM
 constexpr int kRingBudget = (kCtasPerSm == 2 ? 96 : 192) * 1024;  // staged page bytes per CTA
+constexpr int kHeads = 4;  // query heads per CTA (the head columns of the MMAs)
+
+// Head groups per kv-head: its query heads in runs of at most kHeads.
+__host__ __device__ inline int head_groups(const Dims& d) { return (d.gq + kHeads - 1) / kHeads; }
 constexpr long long kWaitCycles = 4000000000LL;  // bounded mbarrier waits (~2 s)
 constexpr int kZeroBytes = 512;                   // all-zero metadata rows
 
@@ -59,7 +66,7 @@ struct Ws {
   float* m;       // [B][Hq][S]
   float* l;       // [B][Hq][S]
   float* o;       // [B][Hq][S][128]
-  unsigned* tk;   // [B][Hkv]
+  unsigned* tk;   // [B][Hkv][head groups] (sized [B][Hq])
 };
 
 __host__ __device__ inline size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -79,18 +86,17 @@ __host__ __device__ inline Ws carve(void* base, int batch, int hq, int hkv, int 
 }
 
 // A warp's final state (row maximum, row sum, unnormalised output row per
-// query head).  A tensor-core warp writes it at the start of its own ring as
-// soon as it is done; SIMT warps have a region each at the start of shared
-// memory.
+// query head of the CTA's head group), written at the start of the warp's own
+// ring as soon as it is done.
 struct WarpState {
-  float m[kMaxGq];
-  float l[kMaxGq];
-  float o[kMaxGq][kHeadDim];
+  float m[kHeads];
+  float l[kHeads];
+  float o[kHeads][kHeadDim];
 };
 // Small shared arrays of the merges (static shared memory).
 struct MergeSmall {
-  float ww[kWarps][kMaxGq];             // warp merge weights 2^(m_w - M)
-  float cta_m[kMaxGq];
+  float ww[kWarps][kHeads];             // warp merge weights 2^(m_w - M)
+  float cta_m[kHeads];
   int last;
 };
 
@@ -187,130 +193,6 @@ __device__ __forceinline__ uint32_t h2u(__half2 h) { return *reinterpret_cast<ui
 __device__ __forceinline__ __half2 u2h(uint32_t u) { return *reinterpret_cast<__half2*>(&u); }
 __device__ __forceinline__ uint32_t hsub1024(uint32_t x) {
   return h2u(__hsub2(u2h(x), u2h(0x64006400u)));
-}
-
-// ---------------------------------------------------------------------------
-// SIMT path: residual window (and every unit when the query group is wider
-// than 4).  Lane = token for scores; lane owns channels 4*lane.. for values.
-// ---------------------------------------------------------------------------
-
-struct State {
-  float m[kMaxGq], l[kMaxGq], acc[kMaxGq][4];
-};
-
-template <typename VRow>
-__device__ __forceinline__ void online_update(State& st, float (&sc)[kMaxGq], int gq, int n_tok,
-                                              const VRow& vrow) {
-  const int lane = threadIdx.x & 31;
-  float p[kMaxGq];
-#pragma unroll
-  for (int g = 0; g < kMaxGq; ++g) {
-    if (g >= gq) break;
-    const float s = lane < n_tok ? sc[g] : -INFINITY;
-    const float mx = warp_max(s);
-    const float mn = fmaxf(st.m[g], mx);
-    const float corr = exp2f(st.m[g] - mn);
-    p[g] = exp2f(s - mn);
-    st.l[g] = st.l[g] * corr + warp_sum(p[g]);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) st.acc[g][i] *= corr;
-    st.m[g] = mn;
-  }
-  for (int t = 0; t < n_tok; ++t) {
-    float v[4];
-    vrow(t, v);
-#pragma unroll
-    for (int g = 0; g < kMaxGq; ++g) {
-      if (g >= gq) break;
-      const float pt = __shfl_sync(0xffffffffu, p[g], t);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) st.acc[g][i] = fmaf(pt, v[i], st.acc[g][i]);
-    }
-  }
-}
-
-template <int BK, int BV>
-__device__ void simt_packed_unit(State& st, const float (*qs)[kHeadDim], int gq, const char* page) {
-  const int lane = threadIdx.x & 31;
-  const uint32_t* kc = reinterpret_cast<const uint32_t*>(page);
-  const __half* ksc = reinterpret_cast<const __half*>(page + page_off_kmeta(BK));  // [128] then zeros
-  const uint32_t* vc = reinterpret_cast<const uint32_t*>(page + page_off_vcodes(BK));
-  const __half* vsc = reinterpret_cast<const __half*>(page + page_off_vmeta(BK, BV));  // scales, zeros
-  constexpr uint32_t kMaskK = (1u << BK) - 1u, kMaskV = (1u << BV) - 1u;
-  float sc[kMaxGq];
-#pragma unroll
-  for (int g = 0; g < kMaxGq; ++g) sc[g] = 0.0f;
-  const int kword = (lane * BK) / 32, kshift = (lane * BK) % 32;
-  for (int c = 0; c < kHeadDim; ++c) {
-    uint32_t code;
-    if (BK == 1) {
-      const int bit = key1_bit(lane, c);
-      code = (kc[bit >> 5] >> (bit & 31)) & 1u;
-    } else {
-      code = (kc[c * BK + kword] >> kshift) & kMaskK;
-    }
-    const float kh = fmaf(__half2float(ksc[c]), (float)code, __half2float(ksc[kHeadDim + c]));
-#pragma unroll
-    for (int g = 0; g < kMaxGq; ++g) {
-      if (g >= gq) break;
-      sc[g] = fmaf(qs[g][c], kh, sc[g]);
-    }
-  }
-  const int grp = lane >> 3;
-  online_update(st, sc, gq, kGroup, [&](int t, float (&v)[4]) {
-    const int mi = vmeta_index(grp, t);
-    const float sv = __half2float(vsc[mi]), zv = __half2float(vsc[kHeadDim + mi]);
-    const uint32_t* w = vc + (grp * 32 + t) * BV;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      uint32_t code;
-      if (BV == 1) {
-        const int bit = val1_bit(t, 4 * lane + i);
-        code = (vc[bit >> 5] >> (bit & 31)) & 1u;
-      } else {
-        const int cc = (4 * lane + i) & 31;
-        code = (w[(cc * BV) / 32] >> ((cc * BV) % 32)) & kMaskV;
-      }
-      v[i] = fmaf(sv, (float)code, zv);
-    }
-  });
-}
-
-__device__ void simt_resid_unit(State& st, const float (*qs)[kHeadDim], int gq, const __half* ring_k,
-                                const __half* ring_v, int p0, int n_tok, int ring) {
-  const int lane = threadIdx.x & 31;
-  float sc[kMaxGq];
-#pragma unroll
-  for (int g = 0; g < kMaxGq; ++g) sc[g] = 0.0f;
-  if (lane < n_tok) {
-    const uint4* row =
-        reinterpret_cast<const uint4*>(ring_k + (long long)((p0 + lane) % ring) * kHeadDim);
-    for (int piece = 0; piece < 16; ++piece) {
-      const uint4 u = row[piece];
-      const __half2* h2 = reinterpret_cast<const __half2*>(&u);
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 f = __half22float2(h2[e]);
-        const int c = piece * 8 + 2 * e;
-#pragma unroll
-        for (int g = 0; g < kMaxGq; ++g) {
-          if (g >= gq) break;
-          sc[g] = fmaf(qs[g][c], f.x, sc[g]);
-          sc[g] = fmaf(qs[g][c + 1], f.y, sc[g]);
-        }
-      }
-    }
-  }
-  online_update(st, sc, gq, n_tok, [&](int t, float (&v)[4]) {
-    const uint2 u =
-        reinterpret_cast<const uint2*>(ring_v + (long long)((p0 + t) % ring) * kHeadDim)[lane];
-    const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
-    const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
-    v[0] = a.x;
-    v[1] = a.y;
-    v[2] = b.x;
-    v[3] = b.y;
-  });
 }
 
 // ---------------------------------------------------------------------------
@@ -844,7 +726,8 @@ __device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int 
 // Decode step with a flush: the 32-token block of positions [p0, p0 + 32),
 // still fp16 in the ring, leaves the window.  One warp quantizes it exactly as
 // kvq_pack does (same quantizer, same page layout) into a page image in
-// `image` (shared memory) and writes the page to `page_out`; the caller folds
+// `image` (shared memory) and, if `page_out` is set, writes the page there
+// (other head groups of the kv-head build the same image); the caller folds
 // the image into its state like any streamed block.  Kept out of line: it is
 // rare and its registers would otherwise crowd the streaming loop.
 template <int BK, int BV>
@@ -910,8 +793,9 @@ __device__ __noinline__ void flush_block(const __half* ring_k, const __half* rin
     }
   }
   __syncwarp();
-  for (int i = lane; i < page / 16; i += 32)
-    reinterpret_cast<uint4*>(page_out)[i] = reinterpret_cast<const uint4*>(image)[i];
+  if (page_out)
+    for (int i = lane; i < page / 16; i += 32)
+      reinterpret_cast<uint4*>(page_out)[i] = reinterpret_cast<const uint4*>(image)[i];
   __syncwarp();
 }
 
@@ -921,7 +805,7 @@ template <int BK, int BV>
 __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, int hi_all,
                                char* ring, uint64_t* full, int R, const char* zero,
                                const __half* qh, int gq, float scale_log2, unsigned* flag,
-                               TcState& st, int flush_blk, const __half* ring_k,
+                               TcState& st, int flush_blk, bool write_page, const __half* ring_k,
                                const __half* ring_v, int ring_size) {
   constexpr int page = page_bytes_c(BK, BV);
   constexpr int NB = ring_blocks(page);
@@ -981,7 +865,8 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, 
   __syncwarp();
   if (flush) {
     flush_block<BK, BV>(ring_k, ring_v, flush_blk * kGroup, ring_size, ring,
-                        const_cast<char*>(pages_bh) + (long long)flush_blk * page);
+                        write_page ? const_cast<char*>(pages_bh) + (long long)flush_blk * page
+                                   : nullptr);
     const char* pg[1] = {ring};
     tc_unit<BK, BV, 1>(pg, zero, qb, ln, scale_log2, st);
   }
@@ -1073,7 +958,7 @@ __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
 // The kernel
 // ---------------------------------------------------------------------------
 
-template <int BK, int BV, bool kTc>
+template <int BK, int BV>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     decode_attn_kernel(Dims d, kvq_cache c, const __half* __restrict__ q, float* __restrict__ out,
                        float scale_log2, int S, unsigned smem_size, Ws ws,
@@ -1081,27 +966,33 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ MergeSmall ms;
   __shared__ int len_s[2];  // length attended, length before the append
-  __shared__ __align__(16) __half q_s[4 * kHeadDim];  // tensor-core path: the query group
+  __shared__ __align__(16) __half q_s[kHeads * kHeadDim];  // the CTA's query heads
   __shared__ __align__(8) uint64_t wbar[kWarps];      // a window warp's staging barrier
 
-  const int h = blockIdx.y, b = blockIdx.z;
-  const int gq = d.gq, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int NV = gridDim.x * kWarps;     // warps per (sequence, kv-head)
+  // head group hg of kv-head h: query heads h * group + 4 hg + [0, gq)
+  const int n_hg = head_groups(d);
+  const int h = blockIdx.y / n_hg, hg = blockIdx.y - h * n_hg, b = blockIdx.z;
+  const int gq = min(kHeads, d.gq - kHeads * hg);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int NV = gridDim.x * kWarps;     // warps per (sequence, kv-head, head group)
   const int v = blockIdx.x * kWarps + warp;
   pdl_launch_dependents();
   const long long bh = (long long)b * d.hkv + h;
   const char* pages = static_cast<const char*>(c.pages) + bh * d.max_blocks * d.page_bytes;
   const __half* ring_k = reinterpret_cast<const __half*>(c.k_resid) + bh * d.ring * kHeadDim;
   const __half* ring_v = reinterpret_cast<const __half*>(c.v_resid) + bh * d.ring * kHeadDim;
-  const __half* qh = q + ((long long)b * d.hq + (long long)h * gq) * kHeadDim;
+  const long long head0 = (long long)b * d.hq + (long long)h * d.gq + kHeads * hg;
+  const __half* qh = q + head0 * kHeadDim;
   unsigned* flag = reinterpret_cast<unsigned*>(c.seq_len) + d.batch;
-  // Decode step (k_new given, tensor-core path only): this kernel appends one
-  // token per sequence before attending.  seq_len[b] is read once per CTA;
-  // the last CTA of the sequence to have read it (ticket) publishes L0 + 1.
-  const bool append = kTc && k_new != nullptr;
+  // Decode step (k_new given): this kernel appends one token per sequence
+  // before attending.  seq_len[b] is read once per CTA; the last CTA of the
+  // sequence to have read it (ticket) publishes L0 + 1.  Head group 0 writes
+  // the new ring row and flushed pages; the other groups compute the same
+  // values for their own use.
+  const bool append = k_new != nullptr;
   unsigned seq_ticket = 0u;
 
-  if constexpr (kTc) {
+  {
     constexpr int page = page_bytes_c(BK, BV);
     const int R = ring_slots(page);
     const int wbytes = warp_ring_bytes(page);
@@ -1165,7 +1056,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       seq_ticket = atomicAdd(reinterpret_cast<unsigned*>(c.seq_len) + d.batch + 2 + b, 1u);
     const __half* k_row = grew ? k_new + bh * kHeadDim : nullptr;
     const __half* v_row = grew ? v_new + bh * kHeadDim : nullptr;
-    if (grew && blockIdx.x == 0 && warp == 0) {  // the new token into its ring slot
+    if (grew && blockIdx.x == 0 && hg == 0 && warp == 0) {  // the new token into its ring slot
       const long long slot = (long long)(L0 % d.ring) * kHeadDim;
       __half* rk = const_cast<__half*>(ring_k) + slot;
       __half* rv = const_cast<__half*>(ring_v) + slot;
@@ -1183,7 +1074,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       if (packed) block_range(p, v, lo, hi);
       tc_packed_warp<BK, BV>(pages, lo_h, pre, lo, hi, ring, full, R,
                              reinterpret_cast<const char*>(zero), q_s, gq, scale_log2, flag, st,
-                             flush_blk, ring_k, ring_v, d.ring);
+                             flush_blk, hg == 0, ring_k, ring_v, d.ring);
     }
     if (!packed)
       tc_window_warp<BK, BV>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, q_s, gq,
@@ -1192,51 +1083,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     WarpState& mine = *reinterpret_cast<WarpState*>(ring);
     if (packed) tc_write_state<true, BV>(st, mine, lane);
     else tc_write_state<false, BV>(st, mine, lane);
-  } else {
-    // SIMT path: every unit (packed blocks, then window chunks) in contiguous
-    // ranges over all warps (query groups wider than 4).
-    pdl_wait();
-    const int L = read_len(c.seq_len + b);
-    const Plan p = make_plan(L, d.residual, NV);
-    const int units = p.nb + p.n_res;
-    const int u0 = (int)((long long)v * units / NV), u1 = (int)((long long)(v + 1) * units / NV);
-    float (*qs)[kHeadDim] =
-        reinterpret_cast<float (*)[kHeadDim]>(smem + (size_t)kWarps * sizeof(WarpState));
-    for (int e = threadIdx.x; e < gq * kHeadDim; e += kThreads)
-      qs[e / kHeadDim][e % kHeadDim] = __half2float(qh[e]) * scale_log2;
-    __syncthreads();
-    State st;
-#pragma unroll
-    for (int g = 0; g < kMaxGq; ++g) {
-      st.m[g] = -INFINITY;
-      st.l[g] = 0.0f;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) st.acc[g][i] = 0.0f;
-    }
-    for (int u = u0; u < u1; ++u) {
-      if (u < p.nb) {
-        simt_packed_unit<BK, BV>(st, qs, gq, pages + (long long)u * d.page_bytes);
-      } else {
-        const int p0 = p.Lq + (u - p.nb) * kGroup;
-        simt_resid_unit(st, qs, gq, ring_k, ring_v, p0, min(kGroup, L - p0), d.ring);
-      }
-    }
-    WarpState& mine = *reinterpret_cast<WarpState*>(smem + (size_t)warp * sizeof(WarpState));
-#pragma unroll
-    for (int g = 0; g < kMaxGq; ++g) {
-      if (g >= gq) break;
-      if (lane == 0) {
-        mine.m[g] = st.m[g];
-        mine.l[g] = st.l[g];
-      }
-#pragma unroll
-      for (int i = 0; i < 4; ++i) mine.o[g][4 * lane + i] = st.acc[g][i];
-    }
   }
   __syncthreads();
 
   // ---- merge the warps of this CTA: one partial per query head ----
-  const size_t wstride = kTc ? (size_t)warp_ring_bytes(page_bytes_c(BK, BV)) : sizeof(WarpState);
+  const size_t wstride = (size_t)warp_ring_bytes(page_bytes_c(BK, BV));
   auto wstate = [&](int w) -> const WarpState& {
     return *reinterpret_cast<const WarpState*>(smem + (size_t)w * wstride);
   };
@@ -1251,7 +1102,6 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   }
   __syncthreads();
   const int n_items = gq * kHeadDim;
-  const long long head0 = (long long)b * d.hq + (long long)h * gq;
   for (int it = threadIdx.x; it < n_items; it += kThreads) {
     const int g = it / kHeadDim, ch = it % kHeadDim;
     float o = 0.0f, l = 0.0f;
@@ -1273,7 +1123,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     }
   }
   if (append && threadIdx.x == 0 &&
-      seq_ticket == (unsigned)(d.hkv * gridDim.x) - 1u) {  // every CTA of b has read L0
+      seq_ticket == gridDim.y * gridDim.x - 1u) {  // every CTA of b has read L0
     const int L1 = len_s[0];
     __threadfence();
     c.seq_len[b] = L1;
@@ -1281,12 +1131,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   }
   if (S == 1) return;
 
-  // ---- the last CTA of this (sequence, kv-head) merges the S partials ----
+  // ---- the last CTA of this (sequence, kv-head, head group) merges the S partials ----
+  const long long bhg = (long long)b * gridDim.y + blockIdx.y;
   __syncthreads();
-  if (threadIdx.x == 0) ms.last = atom_add_acq_rel(&ws.tk[bh], 1u) == (unsigned)S - 1;
+  if (threadIdx.x == 0) ms.last = atom_add_acq_rel(&ws.tk[bhg], 1u) == (unsigned)S - 1;
   __syncthreads();
   if (!ms.last) return;
-  // The partial rows of this (sequence, kv-head) are one contiguous range: a
+  // The partial rows of this head group are one contiguous range: a
   // bulk copy brings them into shared memory (when they fit) while the maxima
   // and sums are loaded and turned into weights.
   const size_t o_bytes = (size_t)gq * S * kHeadDim * sizeof(float);
@@ -1341,40 +1192,30 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     const float Ls = lsum[g];
     out[(head0 + g) * kHeadDim + ch] = Ls > 0.0f ? o / Ls : 0.0f;
   }
-  if (threadIdx.x == 0) ws.tk[bh] = 0u;
+  if (threadIdx.x == 0) ws.tk[bhg] = 0u;
 }
 
-size_t smem_bytes(const Dims& d, bool tc) {
-  // SIMT path: warp states, then q * scale
-  size_t need = (size_t)kWarps * sizeof(WarpState) + sizeof(float) * kMaxGq * kHeadDim;
-  if (tc) {
-    const int page = (int)d.page_bytes;
-    const size_t rings = (size_t)kWarps * warp_ring_bytes(page) +
-                         (size_t)kWarps * ring_slots(page) * sizeof(uint64_t);
-    if (rings > need) need = rings;
-  }
+size_t smem_bytes(const Dims& d) {
+  const int page = (int)d.page_bytes;
+  const size_t rings = (size_t)kWarps * warp_ring_bytes(page) +
+                       (size_t)kWarps * ring_slots(page) * sizeof(uint64_t);
   // + the zero rows of the packed warps and the final merge's mbarrier
-  return (need + kZeroBytes + 16 + 127) / 128 * 128;
+  return (rings + kZeroBytes + 16 + 127) / 128 * 128;
 }
 
-template <int BK, int BV, bool kTc>
+template <int BK, int BV>
 cudaError_t prepare(const Dims& d) {
-  return cudaFuncSetAttribute(decode_attn_kernel<BK, BV, kTc>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes(d, kTc));
+  return cudaFuncSetAttribute(decode_attn_kernel<BK, BV>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes(d));
 }
 
-// Kernel instance for (bits_k, bits_v, query-group width): Op::run<BK, BV, kTc>.
-template <int BK, int BV, typename Op>
-cudaError_t dispatch_mode(const Dims& d, const Op& op) {
-  return d.gq <= 4 ? op.template run<BK, BV, true>() : op.template run<BK, BV, false>();
-}
 template <int BK, typename Op>
 cudaError_t dispatch_bv(const Dims& d, const Op& op) {
   switch (d.bits_v) {
-    case 1: return dispatch_mode<BK, 1>(d, op);
-    case 2: return dispatch_mode<BK, 2>(d, op);
-    case 4: return dispatch_mode<BK, 4>(d, op);
-    default: return dispatch_mode<BK, 8>(d, op);
+    case 1: return op.template run<BK, 1>();
+    case 2: return op.template run<BK, 2>();
+    case 4: return op.template run<BK, 4>();
+    default: return op.template run<BK, 8>();
   }
 }
 template <typename Op>
@@ -1398,22 +1239,22 @@ struct LaunchOp {
   cudaStream_t st;
   const __half* k_new = nullptr;
   const __half* v_new = nullptr;
-  template <int BK, int BV, bool kTc>
+  template <int BK, int BV>
   cudaError_t run() const {
-    cudaError_t e = prepare<BK, BV, kTc>(d);
+    cudaError_t e = prepare<BK, BV>(d);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(S, d.hkv, d.batch);
+    cfg.gridDim = dim3(S, d.hkv * head_groups(d), d.batch);
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = smem_bytes(d, kTc);
+    cfg.dynamicSmemBytes = smem_bytes(d);
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV, kTc>, d, c, q, out, sl2, S,
-                           (unsigned)smem_bytes(d, kTc), ws, k_new, v_new);
+    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV>, d, c, q, out, sl2, S,
+                           (unsigned)smem_bytes(d), ws, k_new, v_new);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
@@ -1421,12 +1262,14 @@ struct LaunchOp {
 
 }  // namespace
 
-// n_splits = CTAs per (sequence, kv-head); workspace rows for up to n_splits.
+// n_splits = CTAs per (sequence, kv-head, head group); workspace rows for up
+// to n_splits.  Tickets: one per (sequence, kv-head, head group), at most one
+// per query head.
 size_t attn_workspace_bytes(const Dims& d, int n_splits) {
   const int S = n_splits + 1;
   const size_t nml = (size_t)d.batch * d.hq * S;
   return align256(nml * 4) * 2 + align256(nml * kHeadDim * 4) +
-         align256((size_t)d.batch * d.hkv * 4);
+         align256((size_t)d.batch * d.hq * 4);
 }
 
 cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& c, const __half* q, float* out,
@@ -1445,10 +1288,10 @@ cudaError_t launch_decode_step(const Dims& d, const kvq_cache& c, const __half* 
   return dispatch(d, op);
 }
 
-// CTAs per (sequence, kv-head): enough for every resident CTA slot of the
-// GPU to hold one, with at least a few blocks per CTA.
+// CTAs per (sequence, kv-head, head group): enough for every resident CTA
+// slot of the GPU to hold one, with at least a few blocks per CTA.
 int attn_default_splits(const Dims& d, int sm_count) {
-  const int bh = d.batch * d.hkv;
+  const int bh = d.batch * d.hkv * head_groups(d);
   int n = kCtasPerSm * sm_count / bh;
   const int cap = (d.max_blocks + 3) / 4;
   if (n > cap) n = cap;
@@ -1506,7 +1349,7 @@ cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& c, const _
   // The array keeps the previous call's contents: the tickets must start at
   // zero, the partials are always written before they are read.
   const Ws w = carve(ws, d.batch, d.hq, d.hkv, n_splits);
-  e = cudaMemsetAsync(w.tk, 0, (size_t)d.batch * d.hkv * sizeof(unsigned), st);
+  e = cudaMemsetAsync(w.tk, 0, (size_t)d.batch * d.hq * sizeof(unsigned), st);
   if (e != cudaSuccess) return e;
   return launch_decode_attn(d, c, q, out, scale_log2, n_splits, ws, st);
 }
