@@ -673,10 +673,16 @@ __host__ __device__ inline Plan make_plan(int L, int residual, int NV) {
   return p;
 }
 
-// Blocks [lo, hi) of packed warp v (v < np).
+// Blocks [lo, hi) of packed warp v (v < np), in 32-bit arithmetic while
+// (v + 1) * nb fits (v < 4096 warps).
 __host__ __device__ inline void block_range(const Plan& p, int v, int& lo, int& hi) {
-  lo = (int)((long long)v * p.nb / p.np);
-  hi = (int)((long long)(v + 1) * p.nb / p.np);
+  if (p.nb < (1 << 20)) {
+    lo = (int)((unsigned)v * (unsigned)p.nb / (unsigned)p.np);
+    hi = (int)((unsigned)(v + 1) * (unsigned)p.nb / (unsigned)p.np);
+  } else {
+    lo = (int)((long long)v * p.nb / p.np);
+    hi = (int)((long long)(v + 1) * p.nb / p.np);
+  }
 }
 
 // Blocks per ring slot and slots per warp for a page size.
@@ -699,9 +705,10 @@ static_assert(kWarps * warp_ring_bytes(page_bytes_c(4, 8)) <= kRingBudget + 8 * 
 // Packed warps stream their blocks through a private ring of slots.  A page
 // is written once, when its group leaves the window, and never changes
 // afterwards, so before waiting for the previous kernel (programmatic
-// dependent launch) lane 0 already streams the full slots of the range that
-// a length read before the wait gives (tc_pre_issue).  If the range after the
-// wait starts elsewhere those slots are consumed without use.
+// dependent launch) lane 0 already streams the first slots of the range that
+// a length read before the wait gives (tc_pre_issue), up to the block before
+// the newest.  If the range after the wait does not begin with exactly those
+// slots they are consumed without use.
 template <int BK, int BV>
 __device__ __forceinline__ void issue_slot(const char* pages_bh, char* ring, uint64_t* full, int R,
                                            int s, int first, int nblk) {
@@ -713,14 +720,22 @@ __device__ __forceinline__ void issue_slot(const char* pages_bh, char* ring, uin
   bulk_g2s(ring + (size_t)(s % R) * NB * page, pages_bh + (long long)first * page, bytes, bar);
 }
 
+// Units (slots) of the range [lo_h, hi_h) that end at or before hi_safe:
+// streams them, returns their count and in `end` the block after them.
 template <int BK, int BV>
-__device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int hi_h, char* ring,
-                                            uint64_t* full, int R) {
+__device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int hi_h, int hi_safe,
+                                            char* ring, uint64_t* full, int R, int& end) {
   constexpr int NB = ring_blocks(page_bytes_c(BK, BV));
-  const int pre = hi_h > lo_h ? min(R, (hi_h - lo_h) / NB) : 0;
-  if ((threadIdx.x & 31) == 0)
-    for (int s = 0; s < pre; ++s) issue_slot<BK, BV>(pages_bh, ring, full, R, s, lo_h + s * NB, NB);
-  return pre;
+  int n = 0;
+  end = lo_h;
+  for (; n < R; ++n) {
+    const int b0 = lo_h + n * NB;
+    const int nblk = min(NB, hi_h - b0);
+    if (nblk <= 0 || b0 + nblk > hi_safe) break;
+    if ((threadIdx.x & 31) == 0) issue_slot<BK, BV>(pages_bh, ring, full, R, n, b0, nblk);
+    end = b0 + nblk;
+  }
+  return n;
 }
 
 // Decode step with a flush: the 32-token block of positions [p0, p0 + 32),
@@ -799,10 +814,10 @@ __device__ __noinline__ void flush_block(const __half* ring_k, const __half* rin
   __syncwarp();
 }
 
-// Fold blocks [lo, hi) into st; `pre` slots were streamed early for a range
-// starting at lo_h.
+// Fold blocks [lo, hi) into st; `pre` slots holding blocks [lo_h, pre_end)
+// were streamed early.
 template <int BK, int BV>
-__device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, int hi_all,
+__device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_end, int lo, int hi_all,
                                char* ring, uint64_t* full, int R, const char* zero,
                                const __half* qh, int gq, float scale_log2, unsigned* flag,
                                TcState& st, int flush_blk, bool write_page, const __half* ring_k,
@@ -814,7 +829,10 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int lo, 
   // quantized from the ring after the streamed ones
   const bool flush = flush_blk >= lo && flush_blk == hi_all - 1;
   const int hi = flush ? hi_all - 1 : hi_all;
-  const int skip = (pre > 0 && lo == lo_h) ? 0 : pre;
+  // the early slots are this range's first units if they start at lo and
+  // cover what its first `pre` units cover
+  const bool reuse = pre > 0 && lo == lo_h && min(lo + pre * NB, hi) == pre_end;
+  const int skip = reuse ? 0 : pre;
   const int n_units = (hi - lo + NB - 1) / NB;
   const int total = skip + n_units;
   int issued = pre;  // lane 0's count of issued slots
@@ -1013,11 +1031,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     if (append && hint < d.max_len) ++hint;  // the length this kernel will attend
     __syncwarp();
     const Plan ph = make_plan(hint, d.residual, NV);
-    int lo_h = 0, hi_h = 0, pre = 0;
+    int lo_h = 0, hi_h = 0, pre = 0, pre_end = 0;
     if (v < ph.np) {
       block_range(ph, v, lo_h, hi_h);
       // the newest block may be the one the previous kernel is writing
-      pre = tc_pre_issue<BK, BV>(pages, lo_h, min(hi_h, ph.nb - 1), ring, full, R);
+      pre = tc_pre_issue<BK, BV>(pages, lo_h, hi_h, ph.nb - 1, ring, full, R, pre_end);
     } else if (lane == 0) {
       // window rows of the length read before the wait into L2 (rows below
       // the newest token do not change; this is a hint, nothing waits on it)
@@ -1063,16 +1081,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       if (lane < 16) reinterpret_cast<uint4*>(rk)[lane] = reinterpret_cast<const uint4*>(k_row)[lane];
       else reinterpret_cast<uint4*>(rv)[lane - 16] = reinterpret_cast<const uint4*>(v_row)[lane - 16];
     }
-    const Plan p = make_plan(L, d.residual, NV);
+    const bool same = L == hint;  // the plan made before the wait holds
+    const Plan p = same ? ph : make_plan(L, d.residual, NV);
     const int flush_blk = grew && p.Lq > packed_len(L0, d.residual) ? p.nb - 1 : -1;
     const bool packed = v < p.np;
     TcState st;
     init_state(st);
     if (packed || pre > 0) {
       // a warp that streamed early retires its slots even if it now has no blocks
-      int lo = 0, hi = 0;
-      if (packed) block_range(p, v, lo, hi);
-      tc_packed_warp<BK, BV>(pages, lo_h, pre, lo, hi, ring, full, R,
+      int lo = lo_h, hi = hi_h;
+      if (!same) {
+        lo = hi = 0;
+        if (packed) block_range(p, v, lo, hi);
+      }
+      tc_packed_warp<BK, BV>(pages, lo_h, pre, pre_end, lo, hi, ring, full, R,
                              reinterpret_cast<const char*>(zero), q_s, gq, scale_log2, flag, st,
                              flush_blk, hg == 0, ring_k, ring_v, d.ring);
     }
