@@ -17,6 +17,7 @@ Modules
 quant      asymmetric b-bit group quantizer, bit packing, residual window
 attention  GQA decode attention softmax(q K^T / sqrt(d)) V over the cache
 dgap       top-K window, risk features, detector, gate, corrector, merge
+drift      offline drift metrics (C(alpha), c_t, d_loc, y_t) and the K_b rule
 """
 
-from . import quant, attention, dgap  # noqa: F401
+from . import quant, attention, dgap, drift  # noqa: F401
