@@ -9,6 +9,8 @@
  *   kvq_decode_attn  softmax(q K^T / sqrt(d)) V over that cache (Sec. 1)
  *   dgap_restore     features, detector, gate, top-K corrector, sparse merge
  *                    on the step's logits (Sec. 4.1-4.3, Eqs. 2, 6, 11-13)
+ *   kvq_drift_*      offline drift metrics on paired FP16 / low-bit logits and
+ *                    the recovery-window rule (Sec. 4.1, Sec. 4.2)
  *
  * Conventions for every call
  * --------------------------
@@ -321,6 +323,59 @@ kvq_status dgap_restore(const dgap_params* params, float* logits,
                         float* topk_val, float* risk, uint8_t* gate,
                         int32_t* next_token, float* features, void* workspace,
                         size_t ws_bytes, void* stream);
+
+/*
+ * Offline drift metrics (Sec. 4.1 "Adaptive recovery-window selection",
+ * Sec. 4.2 "Offline supervision and calibration").  Tooling for paired
+ * traces: each row holds one decode step's FP16-cache logits z_fp and
+ * low-bit-cache logits z_q.  With p = softmax(z), both orders taking values
+ * descending and the lowest index first among equal values:
+ *   C(alpha)  the shortest prefix of the z_fp order whose p_fp mass reaches
+ *             alpha (all of the vocabulary if it never does); M_t = |C|;
+ *   S         TopK(z_q, window);
+ *   c_t       sum of p_fp over C and S (recoverable coverage);
+ *   d_loc     || p_fp / p_fp(U) - p_q / p_q(U) ||_2 over U = C union S;
+ *   y_t       1 if d_loc > eps and c_t >= rho_c, else 0 (the label);
+ *   cov[k-1]  sum of p_fp over C and TopK(z_q, k), k = 1 .. k_max.
+ * The paper gives no values for alpha, eps, rho_c or rho_K.
+ */
+typedef struct kvq_drift_params {
+  float alpha;     /* FP16 candidate mass, 0 < alpha <= 1 */
+  int32_t window;  /* K of S, 1 <= window <= k_max */
+  int32_t k_max;   /* coverage curve length, 1 <= k_max <= 256 and <= vocab */
+  float eps;       /* d_loc threshold of the label, finite */
+  float rho_c;     /* coverage threshold of the label, finite */
+} kvq_drift_params;
+
+/* Largest vocab kvq_drift_metrics accepts (163840). */
+int32_t kvq_drift_max_vocab(void);
+
+/*
+ * kvq_drift_metrics — the metrics above for `rows` steps.
+ *   z_fp, z_q  device fp32 [rows][vocab], finite (no NaN or +inf; -inf is a
+ *              zero-probability logit), read only.  16-byte alignment of
+ *              each row (vocab a multiple of 4) gives vector loads.
+ *   m_t        device int32 [rows]; c_t, d_loc device fp32 [rows];
+ *   y_t        device uint8 [rows]; cov device fp32 [rows][k_max].
+ * Probabilities are e^(z - max z) in fp32, summed in fp64 (c_t, d_loc are
+ * the fp64 results rounded to fp32).  rows <= 65535, vocab <= 163840.
+ * No workspace; calls on different outputs may overlap.
+ */
+kvq_status kvq_drift_metrics(const float* z_fp, const float* z_q, int32_t rows,
+                             int32_t vocab, const kvq_drift_params* params,
+                             int32_t* m_t, float* c_t, float* d_loc,
+                             uint8_t* y_t, float* cov, void* stream);
+
+/*
+ * kvq_drift_window — K_b of Sec. 4.1: the smallest k whose coverage
+ * cov[.][k-1], averaged over the rows, reaches rho_k; 0 if none does.
+ *   cov       device fp32 [rows][k_max] (from kvq_drift_metrics).
+ *   mean_cov  device fp32 [k_max]: the column means (fp64 sums, row order).
+ *   k_b       device int32 [1].
+ */
+kvq_status kvq_drift_window(const float* cov, int32_t rows, int32_t k_max,
+                            float rho_k, float* mean_cov, int32_t* k_b,
+                            void* stream);
 
 #ifdef __cplusplus
 }

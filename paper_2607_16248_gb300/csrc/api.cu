@@ -356,4 +356,42 @@ kvq_status dgap_restore(const dgap_params* p, float* logits, int32_t batch, int3
                      "dgap_restore launch");
 }
 
+int32_t kvq_drift_max_vocab(void) { return drift_max_vocab(); }
+
+kvq_status kvq_drift_metrics(const float* z_fp, const float* z_q, int32_t rows, int32_t vocab,
+                             const kvq_drift_params* p, int32_t* m_t, float* c_t, float* d_loc,
+                             uint8_t* y_t, float* cov, void* stream) {
+  if (!p) return fail(KVQ_ERR_ARG, "params is NULL");
+  if (!z_fp || !z_q) return fail(KVQ_ERR_ARG, "z_fp / z_q is NULL");
+  if (!m_t || !c_t || !d_loc || !y_t || !cov) return fail(KVQ_ERR_ARG, "an output pointer is NULL");
+  if (rows < 1 || rows > 65535) return fail(KVQ_ERR_SHAPE, "rows must be in [1, 65535] (got %d)", rows);
+  if (vocab < 1) return fail(KVQ_ERR_SHAPE, "vocab must be >= 1 (got %d)", vocab);
+  if (vocab > drift_max_vocab())
+    return fail(KVQ_ERR_UNSUPPORTED, "vocab must be <= %d (got %d)", drift_max_vocab(), vocab);
+  if (!(p->alpha > 0.0f && p->alpha <= 1.0f))
+    return fail(KVQ_ERR_ARG, "alpha must be in (0, 1] (got %g)", (double)p->alpha);
+  if (p->k_max < 1 || p->k_max > drift_max_kcov() || p->k_max > vocab)
+    return fail(KVQ_ERR_ARG, "k_max must be in [1, min(%d, vocab)] (got %d)", drift_max_kcov(),
+                p->k_max);
+  if (p->window < 1 || p->window > p->k_max)
+    return fail(KVQ_ERR_ARG, "window must be in [1, k_max] (got %d)", p->window);
+  if (!isfinite(p->eps) || !isfinite(p->rho_c))
+    return fail(KVQ_ERR_ARG, "eps and rho_c must be finite");
+  return cuda_status(launch_drift(z_fp, z_q, rows, vocab, *p, m_t, c_t, d_loc, y_t, cov,
+                                  static_cast<cudaStream_t>(stream)),
+                     "kvq_drift_metrics launch");
+}
+
+kvq_status kvq_drift_window(const float* cov, int32_t rows, int32_t k_max, float rho_k,
+                            float* mean_cov, int32_t* k_b, void* stream) {
+  if (!cov || !mean_cov || !k_b) return fail(KVQ_ERR_ARG, "a pointer is NULL");
+  if (rows < 1) return fail(KVQ_ERR_SHAPE, "rows must be >= 1 (got %d)", rows);
+  if (k_max < 1 || k_max > drift_max_kcov())
+    return fail(KVQ_ERR_ARG, "k_max must be in [1, %d] (got %d)", drift_max_kcov(), k_max);
+  if (!isfinite(rho_k)) return fail(KVQ_ERR_ARG, "rho_k must be finite");
+  return cuda_status(launch_drift_window(cov, rows, k_max, rho_k, mean_cov, k_b,
+                                         static_cast<cudaStream_t>(stream)),
+                     "kvq_drift_window launch");
+}
+
 }  // extern "C"

@@ -147,6 +147,14 @@ struct DgapDims {
 size_t dgap_workspace_bytes_impl(int batch, int vocab, int K);
 int dgap_chunks(int vocab);
 int dgap_max_chunks();
+// Offline drift metrics (drift.cu).
+int drift_max_vocab();
+int drift_max_kcov();
+cudaError_t launch_drift(const float* z_fp, const float* z_q, int rows, int vocab,
+                         const kvq_drift_params& p, int32_t* m_t, float* c_t, float* d_loc,
+                         uint8_t* y_t, float* cov, cudaStream_t st);
+cudaError_t launch_drift_window(const float* cov, int rows, int k_max, float rho_k,
+                                float* mean_cov, int32_t* k_b, cudaStream_t st);
 cudaError_t launch_dgap(const DgapDims& d, const dgap_params& p, float* logits,
                         int32_t* topk_idx, float* topk_val, float* risk,
                         uint8_t* gate, int32_t* next_token, float* features,

@@ -27,7 +27,7 @@ EXPORTS = (
     "kvq_cache_layout", "kvq_cache_bind", "kvq_cache_reset", "kvq_pack",
     "kvq_attn_workspace_bytes", "kvq_attn_default_splits", "kvq_workspace_init",
     "kvq_decode_attn", "kvq_decode_step", "kvq_decode_attn_noalloc", "dgap_workspace_bytes",
-    "dgap_restore",
+    "dgap_restore", "kvq_drift_max_vocab", "kvq_drift_metrics", "kvq_drift_window",
 )
 NOALLOC_SCRATCH_BYTES = 4 << 20
 
@@ -47,6 +47,11 @@ class _Config(ctypes.Structure):
 class _Cache(ctypes.Structure):
     _fields_ = [("pages", ctypes.c_void_p), ("k_resid", ctypes.c_void_p),
                 ("v_resid", ctypes.c_void_p), ("seq_len", ctypes.c_void_p)]
+
+
+class _DriftParams(ctypes.Structure):
+    _fields_ = [("alpha", ctypes.c_float), ("window", ctypes.c_int32), ("k_max", ctypes.c_int32),
+                ("eps", ctypes.c_float), ("rho_c", ctypes.c_float)]
 
 
 class _DgapParams(ctypes.Structure):
@@ -84,6 +89,10 @@ def lib():
             "kvq_decode_attn_noalloc": (I32, [cfg_p, cache_p, P, P, F32, I32, P]),
             "dgap_workspace_bytes": (SZ, [I32, I32, par_p]),
             "dgap_restore": (I32, [par_p, P, I32, I32, P, P, P, P, P, P, P, SZ, P]),
+            "kvq_drift_max_vocab": (I32, []),
+            "kvq_drift_metrics": (I32, [P, P, I32, I32, ctypes.POINTER(_DriftParams),
+                                        P, P, P, P, P, P]),
+            "kvq_drift_window": (I32, [P, I32, I32, F32, P, P, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -385,3 +394,45 @@ def logit(tau):
     if tau <= 0.0:
         return -math.inf
     return math.log(tau / (1.0 - tau))
+
+
+# ---------------------------------------------------------------------------
+# Offline drift metrics (Sec. 4.1, Sec. 4.2)
+# ---------------------------------------------------------------------------
+
+def drift_metrics(z_fp, z_q, alpha, window, k_max, eps, rho_c, outputs=None, stream=None):
+    """kvq_drift_metrics on paired fp32 logits [rows, vocab].
+
+    Returns a dict of device tensors: m_t (int32), c_t, d_loc (fp32),
+    y_t (uint8) per row and cov [rows, k_max] (fp32)."""
+    if z_fp.dim() != 2 or z_fp.shape != z_q.shape:
+        raise ValueError("z_fp and z_q must both be [rows, vocab]")
+    R, V = z_fp.shape
+    dev = z_fp.device
+    if outputs is None:
+        outputs = dict(m_t=torch.empty(R, dtype=torch.int32, device=dev),
+                       c_t=torch.empty(R, dtype=torch.float32, device=dev),
+                       d_loc=torch.empty(R, dtype=torch.float32, device=dev),
+                       y_t=torch.empty(R, dtype=torch.uint8, device=dev),
+                       cov=torch.empty(R, k_max, dtype=torch.float32, device=dev))
+    o = outputs
+    p = _DriftParams(float(alpha), int(window), int(k_max), float(eps), float(rho_c))
+    _check(lib().kvq_drift_metrics(
+        _dev(z_fp, torch.float32, "z_fp"), _dev(z_q, torch.float32, "z_q"), R, V, ctypes.byref(p),
+        _dev(o["m_t"], torch.int32, "m_t"), _dev(o["c_t"], torch.float32, "c_t"),
+        _dev(o["d_loc"], torch.float32, "d_loc"), _dev(o["y_t"], torch.uint8, "y_t"),
+        _dev(o["cov"], torch.float32, "cov"), _stream(stream)))
+    return o
+
+
+def drift_window(cov, rho_k, stream=None):
+    """kvq_drift_window: (K_b as a device int32 [1], mean coverage [k_max])."""
+    if cov.dim() != 2:
+        raise ValueError("cov must be [rows, k_max]")
+    R, K = cov.shape
+    mean = torch.empty(K, dtype=torch.float32, device=cov.device)
+    kb = torch.empty(1, dtype=torch.int32, device=cov.device)
+    _check(lib().kvq_drift_window(_dev(cov, torch.float32, "cov"), R, K, float(rho_k),
+                                  _dev(mean, torch.float32, "mean_cov"),
+                                  _dev(kb, torch.int32, "k_b"), _stream(stream)))
+    return kb, mean

@@ -46,6 +46,16 @@ def logits(seed, batch, vocab, sigma=3.0, device="cpu"):
     return torch.randn(batch, vocab, generator=g, device=device) * sigma
 
 
+def paired_logits(seed, rows, vocab, sigma=3.0, noise=0.3, device="cpu"):
+    """Synthetic paired traces: FP16-cache logits z_fp (Gaussian, std sigma)
+    and low-bit-cache logits z_q = z_fp + Gaussian noise (std noise), fp32
+    [rows, vocab] each."""
+    g = generator(seed, device)
+    z_fp = torch.randn(rows, vocab, generator=g, device=device) * sigma
+    z_q = z_fp + torch.randn(rows, vocab, generator=g, device=device) * noise
+    return z_fp, z_q
+
+
 def ragged_lengths(seed, batch, lo=8192, hi=32768):
     """Per-sequence context lengths drawn uniformly from [lo, hi]."""
     g = generator(seed)
