@@ -16,6 +16,12 @@ roofline.  One JSON line is printed by rank 0.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the CPU oracle on the same config
+
+The drift workload (offline metrics on paired FP16 / low-bit logits, Sec. 4.1
+and 4.2) has its own line: a step is kvq_drift_metrics + kvq_drift_window on
+[rows, vocab] paired logits.
+
+  python bench.py --workload drift-paired-128k
 """
 
 import argparse
@@ -38,6 +44,13 @@ METRIC = "packed-KV decode attn HBM GB/s (% of GB300 peak); DGAP epilogue µs/st
 FALLBACK_HBM_GBS = 6800.0
 DGAP_K, DGAP_HIDDEN, DGAP_TAU = 32, 256, 0.60
 ATTN_PROFILE = ROOT / "profiles" / "attn_llama8b_k1v1_32k.md"
+DRIFT_PROFILE = ROOT / "profiles" / "drift_paired_128k.md"
+DRIFT_METRIC = "drift metrics on paired logits: HBM GB/s (% of GB300 peak)"
+# Offline drift tooling: 256 decode steps of paired Llama-vocabulary logits.
+DRIFT_WORKLOADS = {
+    "drift-paired-128k": dict(rows=256, vocab=128256, alpha=0.9, window=32, k_max=256,
+                              eps=0.02, rho_c=0.5, rho_k=0.9, sigma=3.0, noise=0.4, seed=11),
+}
 
 
 def parse():
@@ -94,18 +107,19 @@ def source_digest(*names):
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
-    """DRAM bytes per attention launch from the committed ncu summary, if it
-    was taken on the current attention source."""
-    if not ATTN_PROFILE.exists():
+def profiled_traffic(path=ATTN_PROFILE, sources=("attn.cu", "common.cuh"),
+                     sha_key="attn_source_sha"):
+    """DRAM bytes per launch of the profiled kernel from its committed ncu
+    summary, if it was taken on the current source."""
+    if not path.exists():
         return None
     fields = {}
-    for line in ATTN_PROFILE.read_text().splitlines():
+    for line in path.read_text().splitlines():
         if ":" in line and line.strip().startswith("- "):
             k, v = line.strip()[2:].split(":", 1)
             fields[k.strip()] = v.strip().strip("`")
     try:
-        if fields.get("attn_source_sha") != source_digest("attn.cu", "common.cuh"):
+        if fields.get(sha_key) != source_digest(*sources):
             return None
         return float(fields["dram_bytes_per_launch_full"])
     except (KeyError, ValueError):
@@ -600,6 +614,198 @@ def run_e2e(st, W, K, world, done):
 
 
 # ---------------------------------------------------------------------------
+# Drift workload (offline metrics on paired logits)
+# ---------------------------------------------------------------------------
+
+
+def drift_bytes(w):
+    """Algorithmic HBM bytes of one step: both logit rows read once, the
+    per-row results and the coverage curve written, the window rule's read of
+    the curve and its means."""
+    R, V, K = w["rows"], w["vocab"], w["k_max"]
+    metrics = 2 * R * V * 4 + R * (4 + 4 + 4 + 1) + R * K * 4
+    window = R * K * 4 + K * 4 + 4
+    return metrics, window
+
+
+def drift_cpu_worker(w, budget_s, n_rows=None):
+    """Oracle rows of the drift workload: time per row (1 thread)."""
+    import numpy as np
+    from oracle import drift
+    from paper_2607_16248_gb300 import synth
+    zf, zq = synth.paired_logits(w["seed"], min(w["rows"], 64), w["vocab"], w["sigma"],
+                                 w["noise"])
+    zf, zq = zf.double().numpy(), zq.double().numpy()
+    t0 = time.perf_counter()
+    n = 0
+    while (n_rows is None and (time.perf_counter() - t0 < budget_s or n == 0)) or \
+            (n_rows is not None and n < n_rows):
+        r = n % zf.shape[0]
+        drift.step_metrics(zf[r], zq[r], w["alpha"], w["window"], w["eps"], w["rho_c"],
+                           w["k_max"])
+        n += 1
+    return n, time.perf_counter() - t0
+
+
+def run_drift(args, w):
+    import torch
+    from paper_2607_16248_gb300 import kvq, synth
+    world, rank, local = dist_setup(args)
+    device = torch.device("cuda", local if world > 1 else 0)
+    K, W = args.steps, args.warmup
+    R, V, KM = w["rows"], w["vocab"], w["k_max"]
+    zf, zq = synth.paired_logits(w["seed"] + 7919 * rank, R, V, w["sigma"], w["noise"],
+                                 device=device)
+    out = dict(m_t=torch.empty(R, dtype=torch.int32, device=device),
+               c_t=torch.empty(R, dtype=torch.float32, device=device),
+               d_loc=torch.empty(R, dtype=torch.float32, device=device),
+               y_t=torch.empty(R, dtype=torch.uint8, device=device),
+               cov=torch.empty(R, KM, dtype=torch.float32, device=device))
+    kb = [None]
+
+    def metrics():
+        kvq.drift_metrics(zf, zq, w["alpha"], w["window"], KM, w["eps"], w["rho_c"], outputs=out)
+
+    def step():
+        metrics()
+        kb[0] = kvq.drift_window(out["cov"], w["rho_k"])
+
+    g_step, g_met = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    step()  # warm the launch path before capture
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g_step):
+        step()
+    with torch.cuda.graph(g_met):
+        metrics()
+    kb_dev = kb[0][0]
+
+    def timed(g, n_warm, n):
+        for _ in range(n_warm):
+            g.replay()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        barrier(world)
+        t0.record()
+        for _ in range(n):
+            g.replay()
+        t1.record()
+        torch.cuda.synchronize()
+        return reduce_max(t0.elapsed_time(t1), world)
+
+    for _ in range(W):
+        g_step.replay()
+    clocks = Clocks(torch.cuda.current_device())
+    torch.cuda.synchronize()
+    barrier(world)
+    clocks.start()
+    time.sleep(0.25)
+    total_ms = timed(g_step, 0, K)
+    clk = clocks.stop()
+    met_ms = timed(g_met, W, K)
+    b_met, b_win = drift_bytes(w)
+    value = job_gbs(world, (b_met + b_win) * K, total_ms)
+    achieved = b_met * K / (met_ms * 1e-3) / 1e9
+    peak, peak_kind = measured_peak_hbm()
+
+    e2e = None
+    if not args.no_e2e:
+        h_zf, h_zq = zf.cpu().pin_memory(), zq.cpu().pin_memory()
+        h_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                 for t in (out["m_t"], out["c_t"], out["d_loc"], out["y_t"], kb_dev)]
+        src = [out["m_t"], out["c_t"], out["d_loc"], out["y_t"], kb_dev]
+
+        def one():
+            zf.copy_(h_zf, non_blocking=True)
+            zq.copy_(h_zq, non_blocking=True)
+            g_step.replay()
+            for h, d in zip(h_out, src):
+                h.copy_(d, non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+
+        for _ in range(W):
+            one()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        barrier(world)
+        t0.record()
+        for _ in range(K):
+            one()
+        t1.record()
+        torch.cuda.synchronize()
+        ms = reduce_max(t0.elapsed_time(t1), world)
+        e2e = {"value": round(job_gbs(world, (b_met + b_win) * K, ms), 2), "unit": "GB/s",
+               "h2d_bytes_per_step": 2 * R * V * 4,
+               "d2h_bytes_per_step": sum(t.numel() * t.element_size() for t in h_out),
+               "ms_per_step": round(ms / K, 5)}
+
+    line = {
+        "metric": DRIFT_METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": round(total_ms / K, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": f"synthetic paired logits: z_fp ~ N(0, {w['sigma']}^2), "
+                f"z_q = z_fp + N(0, {w['noise']}^2)",
+        "config": {"workload": args.workload, "rows": R, "vocab": V, "alpha": w["alpha"],
+                   "window": w["window"], "k_max": KM, "eps": w["eps"], "rho_c": w["rho_c"],
+                   "rho_k": w["rho_k"],
+                   "l2": f"inputs larger than L2: {2 * R * V * 4 / 1e6:.0f} MB of paired logits "
+                         f"per step, L2 129 MB",
+                   "step": "kvq_drift_metrics + kvq_drift_window, one CUDA graph per step",
+                   "parallelism": f"replicas x{world}" if world > 1 else "1 GPU"},
+        "rows_per_s": round(world * R * K / (total_ms * 1e-3), 1),
+        "metrics_us_per_step": round(met_ms / K * 1e3, 3),
+        "k_b": int(kb_dev.item()),
+        "labeled_fraction": float(out["y_t"].float().mean().item()),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
+                     "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "peak_source": f"{peak_kind} hbm_gbs (copy)",
+                     "traffic": profiled_traffic(DRIFT_PROFILE, ("drift.cu", "common.cuh"),
+                                                 "drift_source_sha"),
+                     "algorithmic_bytes_per_launch": b_met},
+        "gpu_launches": 2 * K,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n, t = drift_cpu_worker(w, 12.0)
+        line["cpu_baseline"] = {
+            "value": round((b_met + b_win) / R * n / t / 1e9, 4), "unit": "GB/s", "cores": 1,
+            "kind": "oracle",
+            "sample": f"{n} rows of the workload ({V}-token vocabulary), float64 numpy, 1 thread"}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_drift_reference(args, w):
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    b_met, b_win = drift_bytes(w)
+    # each step: one oracle row; keep the run to a few minutes
+    n0, t0 = drift_cpu_worker(w, 0.0, n_rows=1)
+    steps = args.steps
+    if t0 * (steps + args.warmup) > 150.0:
+        steps = max(1, int(150.0 / t0) - args.warmup)
+    drift_cpu_worker(w, 0.0, n_rows=args.warmup)
+    n, t = drift_cpu_worker(w, 0.0, n_rows=steps)
+    per_row = (b_met + b_win) / w["rows"]
+    v = per_row * n / t / 1e9
+    line = {"impl": "reference", "metric": DRIFT_METRIC, "value": round(v, 4), "unit": "GB/s",
+            "n_gpus": world, "steps": steps, "warmup": args.warmup,
+            "ms_per_step": round(t / n * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "rows": w["rows"], "vocab": w["vocab"]},
+            "cpu_baseline": {"value": round(v, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                             "sample": "each step: one row of the workload, float64 numpy, "
+                                       "1 thread"},
+            "e2e": {"value": round(v, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+# ---------------------------------------------------------------------------
 # Reference arm: the CPU oracle, timed on the host cores
 # ---------------------------------------------------------------------------
 
@@ -649,6 +855,15 @@ def main():
         cpu_worker(sys.argv[j + 1], float(sys.argv[j + 2]), mode)
         return
     args = parse()
+    if args.workload in DRIFT_WORKLOADS:
+        w = DRIFT_WORKLOADS[args.workload]
+        if args.impl == "reference":
+            run_drift_reference(args, w)
+            return
+        from paper_2607_16248_gb300 import build
+        build.build()
+        run_drift(args, w)
+        return
     spec = workload_spec(args)
     if args.impl == "reference":
         run_reference(args, spec)

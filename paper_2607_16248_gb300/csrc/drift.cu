@@ -17,19 +17,23 @@
 // One cluster of 8 CTAs per row.  Each CTA stages an eighth of both logit
 // rows in shared memory once (the only HBM read) and the CTAs combine their
 // partial results through distributed shared memory:
-//   1. maxima, then the FP16 normaliser S_fp = sum e^{z - m} (fp64);
+//   1. maxima;
 //   2. the FP16 boundary: a 2048-bin histogram of the depth (m - z) * 64
-//      (count and mass per bin, the depth order is the FP16 order) finds the
-//      bin where the prefix mass reaches alpha S_fp; that bin's elements are
+//      (count and mass per bin, the depth order is the FP16 order) and, in
+//      the same pass, the normaliser S_fp = sum e^{z - m}, find the bin
+//      where the prefix mass reaches alpha S_fp; that bin's elements are
 //      sorted in one CTA and scanned for the exact element.  A bin with more
 //      than 2048 elements is narrowed by histograms of its key range first;
 //      a range of equal keys takes the lowest indices (counted per CTA in
 //      index order);
 //   3. the same selection by count on z_q gives the k_max-th element, then
 //      the k_max best elements are gathered and sorted (the TopK order);
-//   4. the sums over U (fp64), then d_loc from the renormalised vectors.
-// Weights are e = expf(z - m) in fp32 everywhere, summed in fp64, so every
-// decision between two elements uses the same numbers.
+//   4. one pass over U: its masses (fixed point) and the sums of e_fp^2,
+//      e_fp e_q, e_q^2 (double-float), from which d_loc follows.
+// A mass term e = expf(z - m) (fp32, in (0, 1]) is taken as an integer
+// multiple of 2^-40 (round to nearest) and every mass sum is an exact 64-bit
+// integer sum: the same numbers decide every comparison, in any order, and
+// no per-element fp64 arithmetic is needed.
 
 #include <float.h>
 
@@ -46,20 +50,28 @@ constexpr int kBins = 2048;          // histogram bins
 constexpr int kCap = 2048;           // largest boundary set sorted in one CTA
 constexpr int kMaxKcov = 256;        // longest coverage curve
 constexpr float kDepthScale = 64.0f; // bins per unit of depth m - z
-constexpr int kSlots = 64;           // exchange slots (one per cluster reduction)
+constexpr int kSlots = 32;           // exchange slots (one per cluster exchange)
+constexpr int kXw = 4;               // words per exchange
+typedef unsigned long long u64;
 
 struct Sm {
   float zf[kSlice];
   float zq[kSlice];
-  uint32_t hc[kBins];
-  float hm[kBins];
-  unsigned long long buf[kCap];     // rank 0: boundary set / TopK set
-  double xd[kSlots][2];             // per-CTA partials read by the peers
+  uint32_t hc[kBins];               // bin counts
+  uint32_t hm[3][kBins];            // bin masses: 14-bit chunks of the fixed-point terms
+  u64 buf[kCap];                    // rank 0: boundary set / TopK set
+  u64 xd[kSlots][kXw];              // per-CTA partials read by the peers
   uint32_t xu[kSlots][2];
-  double res_d[4];                  // rank 0: results of a selection
-  uint32_t res_u[8];
+  uint32_t res_u[8];                // rank 0: results of a selection
+  u64 res_q[4];                     // the boundary bin's owner: its result
   uint32_t nbuf;                    // rank 0: fill count of buf
-  double rd[kW];
+  u64 rq[kW];
+  // merged histogram of this CTA's eighth of the bins, and exchange scratch
+  uint32_t rc[kBins / kCl];
+  u64 rm[kBins / kCl];
+  u64 xin[kCl][kXw];                // values loaded from the eight CTAs
+  u64 wsel[kMaxKcov];               // coverage terms of the TopK list
+  float bc[4];                      // broadcast scalars
   uint32_t ru[kW];
   float rf[kW];
 };
@@ -82,14 +94,14 @@ __device__ __forceinline__ uint32_t peer_addr(const void* p, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
   return a;
 }
-__device__ __forceinline__ double ld_peer_f64(uint32_t a) {
-  double v;
-  asm volatile("ld.shared::cluster.f64 %0, [%1];" : "=d"(v) : "r"(a) : "memory");
-  return v;
-}
 __device__ __forceinline__ float ld_peer_f32(uint32_t a) {
   float v;
   asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ u64 ld_peer_u64(uint32_t a) {
+  u64 v;
+  asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(a) : "memory");
   return v;
 }
 __device__ __forceinline__ uint32_t ld_peer_u32(uint32_t a) {
@@ -119,6 +131,50 @@ __device__ __forceinline__ uint32_t fkey(float x) {
 __device__ __forceinline__ float fval(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
 }
+// A mass term e in [0, 1] as a multiple of 2^-40, rounded to nearest: e 2^20
+// splits exactly into its integer part and a fraction whose 2^20 multiple
+// fits a u32.
+__device__ __forceinline__ u64 fix40(float e) {
+  const float a = e * 1048576.0f;
+  const uint32_t hi = (uint32_t)a;
+  const uint32_t lo = __float2uint_rn((a - (float)hi) * 1048576.0f);
+  return ((u64)hi << 20) + lo;
+}
+constexpr double kFix = 1099511627776.0;  // 2^40
+
+// Double-float accumulator: an unevaluated sum hi + lo of two floats
+// (error-free transformations: two-sum and the fma product residual).
+struct Df {
+  float hi = 0.0f, lo = 0.0f;
+  __device__ __forceinline__ void add(float x) {
+    const float s = hi + x;
+    const float bb = s - hi;
+    const float e = (hi - (s - bb)) + (x - bb);
+    const float l = lo + e;
+    hi = s + l;
+    lo = l - (hi - s);
+  }
+  __device__ __forceinline__ void add(const Df& o) {
+    add(o.hi);
+    add(o.lo);
+  }
+  __device__ __forceinline__ void add_prod(float a, float b) {
+    const float p = a * b;
+    add(p);
+    add(fmaf(a, b, -p));
+  }
+  __device__ __forceinline__ u64 pack() const {
+    return ((u64)__float_as_uint(hi) << 32) | __float_as_uint(lo);
+  }
+  __device__ static Df unpack(u64 w) {
+    Df d;
+    d.hi = __uint_as_float((uint32_t)(w >> 32));
+    d.lo = __uint_as_float((uint32_t)w);
+    return d;
+  }
+  __device__ __forceinline__ double value() const { return (double)hi + (double)lo; }
+};
+
 // (key, index) packed so that a larger word ranks first: key descending,
 // index ascending.
 __device__ __forceinline__ unsigned long long pack(uint32_t k, uint32_t i) {
@@ -130,14 +186,35 @@ __device__ __forceinline__ uint32_t pk_idx(unsigned long long w) {
 }
 
 // ---- block reductions (all threads get the result) ----
-__device__ double block_sum_d(double v, Sm& s) {
+__device__ u64 block_sum_q(u64 v, Sm& s) {
 #pragma unroll
   for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   __syncthreads();
-  if ((threadIdx.x & 31) == 0) s.rd[threadIdx.x >> 5] = v;
+  if ((threadIdx.x & 31) == 0) s.rq[threadIdx.x >> 5] = v;
   __syncthreads();
-  double r = 0.0;
-  for (int w = 0; w < kW; ++w) r += s.rd[w];  // fixed order
+  u64 r = 0ull;
+  for (int w = 0; w < kW; ++w) r += s.rq[w];
+  return r;
+}
+__device__ Df block_sum_df(Df v, Sm& s) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    Df w;
+    w.hi = __shfl_xor_sync(0xffffffffu, v.hi, o);
+    w.lo = __shfl_xor_sync(0xffffffffu, v.lo, o);
+    // a fixed pairing order keeps every lane's result identical
+    if ((threadIdx.x & o) == 0) {
+      v.add(w);
+    } else {
+      w.add(v);
+      v = w;
+    }
+  }
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) s.rq[threadIdx.x >> 5] = v.pack();
+  __syncthreads();
+  Df r;
+  for (int w = 0; w < kW; ++w) r.add(Df::unpack(s.rq[w]));
   return r;
 }
 __device__ float block_max_f(float v, Sm& s) {
@@ -184,31 +261,31 @@ __device__ uint32_t block_max_u(uint32_t v, Sm& s) {
 // Cluster-wide reductions of two values per CTA: each CTA publishes its
 // partials in slot `slot`, and after the barrier every CTA combines all eight
 // in rank order (identical results everywhere).
-__device__ void cluster_sum2_d(Sm& s, int slot, double& a, double& b) {
+// Publish up to four words in slot `slot`; after the barrier threads load the
+// eight CTAs' words in parallel into s.xin[rank][word].
+__device__ void cluster_gather(Sm& s, int slot, u64 a, u64 b, u64 c = 0ull, u64 d = 0ull) {
   if (threadIdx.x == 0) {
     s.xd[slot][0] = a;
     s.xd[slot][1] = b;
+    s.xd[slot][2] = c;
+    s.xd[slot][3] = d;
   }
   cluster_sync();
-  double ra = 0.0, rb = 0.0;
-  for (uint32_t r = 0; r < kCl; ++r) {
-    ra += ld_peer_f64(peer_addr(&s.xd[slot][0], r));
-    rb += ld_peer_f64(peer_addr(&s.xd[slot][1], r));
-  }
-  a = ra;
-  b = rb;
+  if (threadIdx.x < kXw * kCl)
+    s.xin[threadIdx.x / kXw][threadIdx.x % kXw] =
+        ld_peer_u64(peer_addr(&s.xd[slot][threadIdx.x % kXw], threadIdx.x / kXw));
+  __syncthreads();
+}
+__device__ __forceinline__ void cluster_gather2(Sm& s, int slot, u64 a, u64 b) {
+  cluster_gather(s, slot, a, b);
 }
 // op 0: (sum, sum); op 1: (min, max); op 2: (max, max) on float bits >= 0
 __device__ void cluster_red2_u(Sm& s, int slot, uint32_t& a, uint32_t& b, int op) {
-  if (threadIdx.x == 0) {
-    s.xu[slot][0] = a;
-    s.xu[slot][1] = b;
-  }
-  cluster_sync();
+  cluster_gather2(s, slot, (u64)a, (u64)b);
   uint32_t ra = op == 1 ? 0xffffffffu : 0u, rb = 0u;
-  for (uint32_t r = 0; r < kCl; ++r) {
-    const uint32_t x = ld_peer_u32(peer_addr(&s.xu[slot][0], r));
-    const uint32_t y = ld_peer_u32(peer_addr(&s.xu[slot][1], r));
+  for (int r = 0; r < kCl; ++r) {
+    const uint32_t x = (uint32_t)s.xin[r][0];
+    const uint32_t y = (uint32_t)s.xin[r][1];
     if (op == 0) {
       ra += x;
       rb += y;
@@ -220,6 +297,7 @@ __device__ void cluster_red2_u(Sm& s, int slot, uint32_t& a, uint32_t& b, int op
       rb = max(rb, y);
     }
   }
+  __syncthreads();
   a = ra;
   b = rb;
 }
@@ -253,11 +331,6 @@ struct Ctx {
   uint32_t rank;  // cluster rank
 };
 
-// Weight of a logit in a selection: its FP16 mass term (weighted) or 1.
-__device__ __forceinline__ float weight(float z, float m, bool weighted) {
-  return weighted ? expf(z - m) : 1.0f;
-}
-
 // Result of a selection: the element (key, index) at which the prefix of
 // the order (key descending, index ascending) first reaches the target, and
 // the prefix length.  all = the target is never reached (everything).
@@ -266,93 +339,136 @@ struct Pick {
   bool all;
 };
 
-// Exclusive prefix over the histogram in bin order (bin 0 ranks first) of
-// the cluster-wide counts / masses; finds the bin where the prefix weight
-// reaches `target` (count or mass).  Histograms of all CTAs are reduced in
-// rank order.  If the total stays below the target: with `clamp` the last
-// non-empty bin is taken, else false is returned.
-__device__ bool boundary_bin(Sm& s, bool weighted, double target, int& bin, uint32_t& cnt_above,
-                             double& w_above, uint32_t& cnt_bin, bool clamp = false) {
-  cluster_sync();  // every CTA's histogram is complete
-  const int b0 = threadIdx.x * (kBins / kT);
-  uint32_t c[kBins / kT];
-  double m[kBins / kT];
-  uint32_t csum = 0u;
-  double msum = 0.0;
+// The bin where the prefix weight (count, or mass in fixed point) in bin
+// order (bin 0 ranks first) reaches `target`, over the histograms of all
+// eight CTAs.  CTA r merges bins [256 r, 256 r + 256) of the eight
+// histograms and publishes their total; the CTA whose range holds the target
+// finds the bin and publishes it.  If the total stays below the target: with
+// `clamp` the last non-empty bin is taken, else false is returned (in every
+// CTA alike).
+// With `norm` set, each CTA's *norm holds its part of S_fp on entry and the
+// target is ceil(alpha S_fp) over the cluster: *norm and target return it.
+__device__ bool boundary_bin(Sm& s, const Ctx& cx, bool weighted, u64& target, int& slot, int& bin,
+                             uint32_t& cnt_above, u64& w_above, uint32_t& cnt_bin,
+                             bool clamp = false, u64* norm = nullptr, double alpha = 0.0) {
+  constexpr int kR = kBins / kCl;  // bins per CTA range
+  cluster_sync();                  // every CTA's histogram is complete
+  const int t = threadIdx.x;
+  __shared__ uint32_t part_c[kT];
+  __shared__ u64 part_m[kT];
+  {
+    // thread t merges bin (t % kR) of its range from four of the CTAs
+    const int b = (int)cx.rank * kR + (t % kR);
+    const uint32_t r0 = (uint32_t)(t / kR) * (kCl / (kT / kR));
+    uint32_t c = 0u, m0 = 0u, m1 = 0u, m2 = 0u;
 #pragma unroll
-  for (int j = 0; j < kBins / kT; ++j) {
-    c[j] = 0u;
-    m[j] = 0.0;
-    for (uint32_t r = 0; r < kCl; ++r) {
-      c[j] += ld_peer_u32(peer_addr(&s.hc[b0 + j], r));
-      if (weighted) m[j] += (double)ld_peer_f32(peer_addr(&s.hm[b0 + j], r));
-    }
-    if (!weighted) m[j] = (double)c[j];
-    csum += c[j];
-    msum += m[j];
-  }
-  // block exclusive scan of (csum, msum) over threads, in thread order
-  __shared__ double sc_m[kT];
-  __shared__ uint32_t sc_c[kT];
-  __shared__ int found_bin, last_bin;
-  __shared__ uint32_t found_ca, found_cb;
-  __shared__ double found_wa;
-  sc_m[threadIdx.x] = msum;
-  sc_c[threadIdx.x] = csum;
-  if (threadIdx.x == 0) {
-    found_bin = -1;
-    last_bin = -1;
-  }
-  __syncthreads();
-  for (int o = 1; o < kT; o <<= 1) {
-    const double tm = threadIdx.x >= o ? sc_m[threadIdx.x - o] : 0.0;
-    const uint32_t tc = threadIdx.x >= o ? sc_c[threadIdx.x - o] : 0u;
-    __syncthreads();
-    sc_m[threadIdx.x] += tm;
-    sc_c[threadIdx.x] += tc;
-    __syncthreads();
-  }
-  const double wa0 = sc_m[threadIdx.x] - msum;  // exclusive prefix of this thread
-  const uint32_t ca0 = sc_c[threadIdx.x] - csum;
-  double wa = wa0;
-  uint32_t ca = ca0;
-  int last = -1;
-#pragma unroll
-  for (int j = 0; j < kBins / kT; ++j) {
-    if (wa < target && target <= wa + m[j] && c[j] > 0u) {
-      found_bin = b0 + j;
-      found_wa = wa;
-      found_ca = ca;
-      found_cb = c[j];
-    }
-    if (c[j] > 0u) last = b0 + j;
-    wa += m[j];
-    ca += c[j];
-  }
-  if (last >= 0) atomicMax(&last_bin, last);
-  __syncthreads();
-  if (clamp && found_bin < 0 && last_bin >= b0 && last_bin < b0 + kBins / kT) {
-    // the last non-empty bin: everything before it ranks above
-    wa = wa0;
-    ca = ca0;
-    for (int j = 0; j < kBins / kT; ++j) {
-      if (b0 + j == last_bin) {
-        found_bin = last_bin;
-        found_wa = wa;
-        found_ca = ca;
-        found_cb = c[j];
+    for (uint32_t r = 0; r < kCl / (kT / kR); ++r) {
+      c += ld_peer_u32(peer_addr(&s.hc[b], r0 + r));
+      if (weighted) {
+        m0 += ld_peer_u32(peer_addr(&s.hm[0][b], r0 + r));
+        m1 += ld_peer_u32(peer_addr(&s.hm[1][b], r0 + r));
+        m2 += ld_peer_u32(peer_addr(&s.hm[2][b], r0 + r));
       }
-      wa += m[j];
-      ca += c[j];
+    }
+    part_c[t] = c;
+    part_m[t] = weighted ? (u64)m0 + ((u64)m1 << 14) + ((u64)m2 << 28) : (u64)c;
+  }
+  __syncthreads();
+  // exclusive prefix over this range's bins (warp scans, then warp totals)
+  __shared__ uint32_t wtot_c[kR / 32];
+  __shared__ u64 wtot_m[kR / 32];
+  uint32_t c = 0u, ic = 0u;
+  u64 m = 0ull, im = 0ull;
+  if (t < kR) {
+    c = part_c[t] + part_c[t + kR];
+    m = part_m[t] + part_m[t + kR];
+    s.rc[t] = c;
+    s.rm[t] = m;
+    ic = c;
+    im = m;
+    const int l = t & 31;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t tc = __shfl_up_sync(0xffffffffu, ic, o);
+      const u64 tm = __shfl_up_sync(0xffffffffu, im, o);
+      if (l >= o) {
+        ic += tc;
+        im += tm;
+      }
+    }
+    if (l == 31) {
+      wtot_c[t >> 5] = ic;
+      wtot_m[t >> 5] = im;
     }
   }
-  cluster_sync();  // peers finished reading this CTA's histogram
   __syncthreads();
-  bin = found_bin;
-  if (bin < 0) return false;
-  cnt_above = found_ca;
-  w_above = found_wa;
-  cnt_bin = found_cb;
+  uint32_t tot_c = 0u;
+  u64 tot_m = 0ull;
+  for (int w = 0; w < kR / 32; ++w) {
+    tot_c += wtot_c[w];
+    tot_m += wtot_m[w];
+  }
+  uint32_t ex_c = ic - c;
+  u64 ex_m = im - m;
+  if (t < kR)
+    for (int w = 0; w < (t >> 5); ++w) {
+      ex_c += wtot_c[w];
+      ex_m += wtot_m[w];
+    }
+  // range totals of all eight CTAs (and their S_fp parts), in rank order
+  cluster_gather(s, slot++, (u64)tot_c, tot_m, norm ? *norm : 0ull);
+  if (norm) {
+    u64 sf = 0ull;
+    for (int r = 0; r < kCl; ++r) sf += s.xin[r][2];
+    *norm = sf;
+    // prefix mass >= alpha S  <=>  prefix >= ceil(alpha S) in fixed point
+    target = (u64)ceil(alpha * (double)sf);
+  }
+  u64 pre_m[kCl + 1];
+  uint32_t pre_c[kCl + 1];
+  pre_m[0] = 0ull;
+  pre_c[0] = 0u;
+  int owner = -1, last = -1;
+  for (int r = 0; r < kCl; ++r) {
+    pre_c[r + 1] = pre_c[r] + (uint32_t)s.xin[r][0];
+    pre_m[r + 1] = pre_m[r] + s.xin[r][1];
+    if (owner < 0 && pre_m[r] < target && target <= pre_m[r + 1] && s.xin[r][0] > 0ull) owner = r;
+    if (s.xin[r][0] > 0ull) last = r;
+  }
+  __syncthreads();
+  bool use_last = false;
+  if (owner < 0) {
+    if (!clamp || last < 0) {
+      cluster_sync();  // peers finished reading this CTA's histogram (all return alike)
+      return false;
+    }
+    owner = last;
+    use_last = true;
+  }
+  if ((int)cx.rank == owner && t < kR) {
+    const u64 wa = pre_m[owner] + ex_m;
+    bool hit;
+    if (use_last) {
+      // the last non-empty bin of the range: no later bin has a count
+      hit = c > 0u && ex_c + c == tot_c;
+    } else {
+      hit = c > 0u && wa < target && target <= wa + m;
+    }
+    if (hit) {
+      s.res_q[0] = (u64)(owner * kR + t);
+      s.res_q[1] = (u64)(pre_c[owner] + ex_c);
+      s.res_q[2] = wa;
+      s.res_q[3] = (u64)c;
+    }
+  }
+  cluster_sync();
+  if (t < 4) s.xin[t][0] = ld_peer_u64(peer_addr(&s.res_q[t], (uint32_t)owner));
+  __syncthreads();
+  bin = (int)s.xin[0][0];
+  cnt_above = (uint32_t)s.xin[1][0];
+  w_above = s.xin[2][0];
+  cnt_bin = (uint32_t)s.xin[3][0];
+  cluster_sync();  // every CTA read the owner's result; histograms may be rewritten
   return true;
 }
 
@@ -388,29 +504,48 @@ __device__ uint32_t nth_tie(Sm& s, const Ctx& cx, const float* a, uint32_t key, 
   return ans_s;
 }
 
+__device__ void clear_hist(Sm& s) {
+  for (int i = threadIdx.x; i < kBins; i += kT) {
+    s.hc[i] = 0u;
+    s.hm[0][i] = 0u;
+    s.hm[1][i] = 0u;
+    s.hm[2][i] = 0u;
+  }
+  __syncthreads();
+}
+// Count one element in bin b and (weighted) its mass term in three 14-bit
+// chunks: each chunk's sum over a CTA stays below 2^28.
+__device__ __forceinline__ u64 add_hist(Sm& s, int b, bool weighted, float z, float m) {
+  atomicAdd(&s.hc[b], 1u);
+  if (!weighted) return 0ull;
+  const u64 q = fix40(expf(z - m));
+  atomicAdd(&s.hm[0][b], (uint32_t)(q & 0x3fffu));
+  atomicAdd(&s.hm[1][b], (uint32_t)((q >> 14) & 0x3fffu));
+  atomicAdd(&s.hm[2][b], (uint32_t)(q >> 28));
+  return q;
+}
+
 // Selection over array a (maximum m): the first element of the order at
 // which the prefix weight reaches target.  `slot` counts exchange slots.
 __device__ Pick select(Sm& s, const Ctx& cx, const float* a, float m, bool weighted,
-                       double target, int& slot) {
+                       u64 target, int& slot, u64* norm = nullptr, double alpha = 0.0) {
   Pick pk;
   pk.all = false;
   // ---- round 0: depth bins ----
-  for (int i = threadIdx.x; i < kBins; i += kT) {
-    s.hc[i] = 0u;
-    s.hm[i] = 0.0f;
-  }
-  __syncthreads();
+  clear_hist(s);
+  u64 part = 0ull;
   for (int i = threadIdx.x; i < cx.n; i += kT) {
     const float z = a[i];
     const float t = (m - z) * kDepthScale;
     const int b = t < (float)(kBins - 1) ? (int)t : kBins - 1;
-    atomicAdd(&s.hc[b], 1u);
-    if (weighted) atomicAdd(&s.hm[b], weight(z, m, true));
+    part += add_hist(s, b, weighted, z, m);
   }
+  if (norm) *norm = block_sum_q(part, s);
   int bin;
   uint32_t cnt_above, n_set;
-  double w_above;
-  if (!boundary_bin(s, weighted, target, bin, cnt_above, w_above, n_set)) {
+  u64 w_above;
+  if (!boundary_bin(s, cx, weighted, target, slot, bin, cnt_above, w_above, n_set, false, norm,
+                    alpha)) {
     pk.all = true;
     pk.key = 0u;
     pk.idx = 0xffffffffu;
@@ -447,24 +582,20 @@ __device__ Pick select(Sm& s, const Ctx& cx, const float* a, float m, bool weigh
     if (klo == khi || round >= 3) break;  // equal keys: ties
     // sub-bins of the key range, largest key first
     const unsigned long long span = (unsigned long long)(khi - klo) + 1ull;
-    for (int i = threadIdx.x; i < kBins; i += kT) {
-      s.hc[i] = 0u;
-      s.hm[i] = 0.0f;
-    }
-    __syncthreads();
+    clear_hist(s);
     for (int i = threadIdx.x; i < cx.n; i += kT) {
       const uint32_t k = fkey(a[i]);
       if (k < klo || k > khi) continue;
       const int sb = (int)(((unsigned long long)(khi - k) * kBins) / span);
-      atomicAdd(&s.hc[sb], 1u);
-      if (weighted) atomicAdd(&s.hm[sb], weight(a[i], m, true));
+      add_hist(s, sb, weighted, a[i], m);
     }
     int sbin;
     uint32_t ca, cb;
-    double wa;
+    u64 wa;
     // (rounding can leave the narrowed set below the target: its last
     // non-empty sub-bin is taken)
-    boundary_bin(s, weighted, target - w_above, sbin, ca, wa, cb, true);
+    u64 rel = target - w_above;
+    boundary_bin(s, cx, weighted, rel, slot, sbin, ca, wa, cb, true);
     cnt_above += ca;
     w_above += wa;
     n_set = cb;
@@ -489,19 +620,18 @@ __device__ Pick select(Sm& s, const Ctx& cx, const float* a, float m, bool weigh
 
   if (n_set > (uint32_t)kCap) {
     // all keys equal (klo == khi): the lowest indices come first
-    const float zt = fval(klo);
-    const double wt = (double)weight(zt, m, weighted);
-    double need_d = weighted ? ceil((target - w_above) / wt) : (target - w_above);
-    uint32_t need = need_d < 1.0 ? 1u : (need_d > (double)n_set ? n_set : (uint32_t)need_d);
+    const u64 wt = weighted ? fix40(expf(fval(klo) - m)) : 1ull;
+    const u64 rest = target > w_above ? target - w_above : 0ull;
+    const u64 need_q = wt == 0ull ? (u64)n_set : (rest + wt - 1ull) / wt;
+    const uint32_t need = need_q < 1ull ? 1u : (need_q > (u64)n_set ? n_set : (uint32_t)need_q);
     // ties per CTA, in rank (index) order
     uint32_t mine = 0u;
     for (int i = threadIdx.x; i < cx.n; i += kT) mine += fkey(a[i]) == klo;
     mine = block_sum_u(mine, s);
-    if (threadIdx.x == 0) s.xu[slot][0] = mine;
-    cluster_sync();
+    cluster_gather2(s, slot++, (u64)mine, 0ull);
     uint32_t before = 0u;
-    for (uint32_t r = 0; r < cx.rank; ++r) before += ld_peer_u32(peer_addr(&s.xu[slot][0], r));
-    ++slot;
+    for (uint32_t r = 0; r < cx.rank; ++r) before += (uint32_t)s.xin[r][0];
+    __syncthreads();
     if (cluster_rank() == 0 && threadIdx.x == 0) s.res_u[0] = 0xffffffffu;
     cluster_sync();
     if (need > before && need <= before + mine) {
@@ -509,8 +639,10 @@ __device__ Pick select(Sm& s, const Ctx& cx, const float* a, float m, bool weigh
       if (threadIdx.x == 0) st_peer_u32(peer_addr(&s.res_u[0], 0), gi);
     }
     cluster_sync();
+    if (threadIdx.x == 0) s.xin[0][0] = ld_peer_u32(peer_addr(&s.res_u[0], 0));
+    __syncthreads();
     pk.key = klo;
-    pk.idx = ld_peer_u32(peer_addr(&s.res_u[0], 0));
+    pk.idx = (uint32_t)s.xin[0][0];
     pk.len = cnt_above + need;
     cluster_sync();  // everyone has read rank 0's result
     return pk;
@@ -542,16 +674,16 @@ __device__ Pick select(Sm& s, const Ctx& cx, const float* a, float m, bool weigh
     if (threadIdx.x < 32) {
       // first element whose prefix weight (above + own) reaches the target
       const int l = threadIdx.x;
-      double run = w_above;
+      u64 run = w_above;
       int hit = -1;
       for (int j0 = 0; j0 < n && hit < 0; j0 += 32) {
         const int j = j0 + l;
-        double w = 0.0;
-        if (j < n) w = (double)weight(fval(pk_key(s.buf[j])), m, weighted);
-        double inc = w;
+        u64 w = 0ull;
+        if (j < n) w = weighted ? fix40(expf(fval(pk_key(s.buf[j])) - m)) : 1ull;
+        u64 inc = w;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-          const double t = __shfl_up_sync(0xffffffffu, inc, o);
+          const u64 t = __shfl_up_sync(0xffffffffu, inc, o);
           if (l >= o) inc += t;
         }
         const bool ok = j < n && run + inc >= target;
@@ -568,9 +700,11 @@ __device__ Pick select(Sm& s, const Ctx& cx, const float* a, float m, bool weigh
     }
   }
   cluster_sync();
-  pk.key = ld_peer_u32(peer_addr(&s.res_u[0], 0));
-  pk.idx = ld_peer_u32(peer_addr(&s.res_u[1], 0));
-  pk.len = ld_peer_u32(peer_addr(&s.res_u[2], 0));
+  if (threadIdx.x < 3) s.xin[threadIdx.x][0] = ld_peer_u32(peer_addr(&s.res_u[threadIdx.x], 0));
+  __syncthreads();
+  pk.key = (uint32_t)s.xin[0][0];
+  pk.idx = (uint32_t)s.xin[1][0];
+  pk.len = (uint32_t)s.xin[2][0];
   cluster_sync();  // everyone has read rank 0's result
   return pk;
 }
@@ -632,15 +766,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kT, 1)
     mq = fval(b);
   }
 
-  // ---- FP16 normaliser ----
-  double sf = 0.0, dummy = 0.0;
-  for (int i = threadIdx.x; i < cx.n; i += kT) sf += (double)expf(s.zf[i] - mf);
-  sf = block_sum_d(sf, s);
-  cluster_sum2_d(s, slot++, sf, dummy);
-
-  // ---- C(alpha) and TopK(z_q, k_max) boundaries ----
-  const Pick pf = select(s, cx, s.zf, mf, true, (double)p.alpha * sf, slot);
-  const Pick pq = select(s, cx, s.zq, mq, false, (double)p.k_max, slot);
+  // ---- C(alpha) (with S_fp) and TopK(z_q, k_max) boundaries ----
+  u64 sf = 0ull;
+  const Pick pf = select(s, cx, s.zf, mf, true, 0ull, slot, &sf, (double)p.alpha);
+  const Pick pq = select(s, cx, s.zq, mq, false, (u64)p.k_max, slot);
 
   // ---- the k_max best of z_q, sorted, in rank 0 ----
   if (cx.rank == 0 && threadIdx.x == 0) s.nbuf = 0u;
@@ -673,73 +802,104 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kT, 1)
     }
   }
   cluster_sync();
+  if (threadIdx.x < 2) s.xin[threadIdx.x][0] = ld_peer_u32(peer_addr(&s.res_u[4 + threadIdx.x], 0));
+  __syncthreads();
   Pick ps;
   ps.all = false;
-  ps.key = ld_peer_u32(peer_addr(&s.res_u[4], 0));
-  ps.idx = ld_peer_u32(peer_addr(&s.res_u[5], 0));
+  ps.key = (uint32_t)s.xin[0][0];
+  ps.idx = (uint32_t)s.xin[1][0];
   ps.len = (uint32_t)p.window;
+  __syncthreads();
 
-  // ---- sums over U = C union S ----
-  double A = 0.0, B = 0.0, Cs = 0.0;
+  // ---- one pass over U = C union S ----
+  // masses A = e_fp(U), B = e_q(U), c = e_fp(C and S) in fixed point; the
+  // sums of e_fp^2, e_fp e_q, e_q^2 in double-float for
+  //   d_loc^2 = Saa / A^2 - 2 Sab / (A B) + Sbb / B^2.
+  u64 A = 0ull, B = 0ull, Cs = 0ull;
+  Df saa, sab, sbb;
   for (int i = threadIdx.x; i < cx.n; i += kT) {
     const uint32_t gi = cx.i0 + (uint32_t)i;
     const bool inc = ranks_in(fkey(s.zf[i]), gi, pf);
     const bool ins = ranks_in(fkey(s.zq[i]), gi, ps);
     if (inc || ins) {
-      const double ef = (double)expf(s.zf[i] - mf);
-      A += ef;
-      B += (double)expf(s.zq[i] - mq);
-      if (inc && ins) Cs += ef;
+      const float a = expf(s.zf[i] - mf), b = expf(s.zq[i] - mq);
+      const u64 qa = fix40(a);
+      A += qa;
+      B += fix40(b);
+      if (inc && ins) Cs += qa;
+      saa.add_prod(a, a);
+      sab.add_prod(a, b);
+      sbb.add_prod(b, b);
     }
   }
-  A = block_sum_d(A, s);
-  B = block_sum_d(B, s);
-  Cs = block_sum_d(Cs, s);
-  cluster_sum2_d(s, slot++, A, B);
-  double c_sum = Cs;
-  cluster_sum2_d(s, slot++, c_sum, dummy);
-  double D = 0.0;
-  for (int i = threadIdx.x; i < cx.n; i += kT) {
-    const uint32_t gi = cx.i0 + (uint32_t)i;
-    if (ranks_in(fkey(s.zf[i]), gi, pf) || ranks_in(fkey(s.zq[i]), gi, ps)) {
-      const double d = (double)expf(s.zf[i] - mf) / A - (double)expf(s.zq[i] - mq) / B;
-      D += d * d;
-    }
+  A = block_sum_q(A, s);
+  B = block_sum_q(B, s);
+  Cs = block_sum_q(Cs, s);
+  saa = block_sum_df(saa, s);
+  sab = block_sum_df(sab, s);
+  sbb = block_sum_df(sbb, s);
+  cluster_gather(s, slot++, A, B, Cs);
+  u64 c_sum = 0ull;
+  A = B = 0ull;
+  for (int r = 0; r < kCl; ++r) {
+    A += s.xin[r][0];
+    B += s.xin[r][1];
+    c_sum += s.xin[r][2];
   }
-  D = block_sum_d(D, s);
-  cluster_sum2_d(s, slot++, D, dummy);
+  __syncthreads();
+  cluster_gather(s, slot++, saa.pack(), sab.pack(), sbb.pack());
+  Df taa, tab, tbb;
+  for (int r = 0; r < kCl; ++r) {
+    taa.add(Df::unpack(s.xin[r][0]));
+    tab.add(Df::unpack(s.xin[r][1]));
+    tbb.add(Df::unpack(s.xin[r][2]));
+  }
+  __syncthreads();
+  double Dsum = 0.0;
+  if (threadIdx.x == 0) {
+    const double ia = kFix / (double)A, ib = kFix / (double)B;
+    Dsum = taa.value() * ia * ia - 2.0 * tab.value() * ia * ib + tbb.value() * ib * ib;
+    if (Dsum < 0.0) Dsum = 0.0;  // rounding of an exact zero
+  }
 
   // ---- outputs (rank 0) ----
   if (cx.rank == 0) {
-    const double c = c_sum / sf;
-    const double d = sqrt(D);
     if (threadIdx.x == 0) {
+      const double c = (double)c_sum / (double)sf;
+      const double d = sqrt(Dsum);
       m_t[row] = pf.all ? vocab : (int32_t)pf.len;
       c_t[row] = (float)c;
       d_loc[row] = (float)d;
       y_t[row] = (uint8_t)(d > (double)p.eps && c >= (double)p.rho_c);
     }
+    // coverage curve: prefix sums of p_fp over TopK(z_q, k) within C; the
+    // FP16 logits of the list come from the CTAs that hold them
+    const int sl = ((vocab + kCl - 1) / kCl + 3) & ~3;
+    if (threadIdx.x < p.k_max) {
+      const uint32_t gi = pk_idx(s.buf[threadIdx.x]);
+      u64 w = 0ull;
+      if (gi < (uint32_t)vocab) {
+        const uint32_t owner = gi / (uint32_t)sl;
+        const float zf = ld_peer_f32(peer_addr(&s.zf[gi - owner * (uint32_t)sl], owner));
+        if (ranks_in(fkey(zf), gi, pf)) w = fix40(expf(zf - mf));
+      }
+      s.wsel[threadIdx.x] = w;
+    }
+    if (threadIdx.x == 0) s.bc[2] = (float)(1.0 / (double)sf);
+    __syncthreads();
     if (threadIdx.x < 32) {
-      // coverage curve: prefix sums of p_fp over TopK(z_q, k) within C
       const int l = threadIdx.x;
-      double run = 0.0;
+      const float inv = s.bc[2];
+      u64 run = 0ull;
       for (int j0 = 0; j0 < p.k_max; j0 += 32) {
         const int j = j0 + l;
-        double w = 0.0;
-        if (j < p.k_max) {
-          const uint32_t gi = pk_idx(s.buf[j]);
-          if (gi < (uint32_t)vocab) {
-            const float zf = z_fp[(long long)row * vocab + gi];
-            if (ranks_in(fkey(zf), gi, pf)) w = (double)expf(zf - mf);
-          }
-        }
-        double inc = w;
+        u64 inc = j < p.k_max ? s.wsel[j] : 0ull;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-          const double t = __shfl_up_sync(0xffffffffu, inc, o);
+          const u64 t = __shfl_up_sync(0xffffffffu, inc, o);
           if (l >= o) inc += t;
         }
-        if (j < p.k_max) cov[(long long)row * p.k_max + j] = (float)((run + inc) / sf);
+        if (j < p.k_max) cov[(long long)row * p.k_max + j] = (float)(run + inc) * inv;
         run += __shfl_sync(0xffffffffu, inc, 31);
       }
     }
