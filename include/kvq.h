@@ -24,6 +24,8 @@
  * - Errors that only the device can see (a sequence pushed past max_len)
  *   never fault the GPU: the kernel skips the write and sets a bit in the
  *   cache's flag word (see kvq_cache).
+ * - KVQ_TRACE=1 in the environment prints one line per launch to stderr
+ *   (entry point, shapes, grid and split choices).
  */
 #ifndef KVQ_H
 #define KVQ_H

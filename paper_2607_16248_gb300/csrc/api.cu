@@ -5,6 +5,7 @@
 #include <math.h>
 #include <stdarg.h>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include "common.cuh"
@@ -37,6 +38,25 @@ static kvq_status cuda_status(cudaError_t e, const char* what) {
 }
 
 static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// KVQ_TRACE=1 in the environment: one line per launch on stderr (entry
+// point, shapes, grid choices).  Read once per process.
+static bool tracing() {
+  static const int on = [] {
+    const char* v = getenv("KVQ_TRACE");
+    return v && v[0] && strcmp(v, "0") != 0 ? 1 : 0;
+  }();
+  return on != 0;
+}
+static void trace(const char* fmt, ...) {
+  if (!tracing()) return;
+  va_list ap;
+  va_start(ap, fmt);
+  fputs("kvq: ", stderr);
+  vfprintf(stderr, fmt, ap);
+  fputc('\n', stderr);
+  va_end(ap);
+}
 
 static size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -188,6 +208,8 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache, const uint16_
     return fail(KVQ_ERR_SHAPE, "batch range [%d, %d) outside [0, %d)", batch_begin,
                 batch_begin + batch_count, cfg->batch);
   Dims d = make_dims(*cfg);
+  trace("kvq_pack batch [%d, %d) n_new %d bits K%dV%d", batch_begin, batch_begin + batch_count,
+        n_new, d.bits_k, d.bits_v);
   return cuda_status(launch_pack(d, *cache, reinterpret_cast<const __half*>(k_new),
                                  reinterpret_cast<const __half*>(v_new), n_new, batch_begin,
                                  batch_count, static_cast<cudaStream_t>(stream)),
@@ -236,6 +258,9 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const 
     return fail(KVQ_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", ws_bytes, need);
   const float scale = softmax_scale == 0.0f ? 1.0f / sqrtf((float)kHeadDim) : softmax_scale;
   const float scale_log2 = scale * 1.4426950408889634f;
+  trace("kvq_decode_attn batch %d heads %d/%d bits K%dV%d grid (%d, %d, %d) x 512, %d splits",
+        d.batch, d.hq, d.hkv, d.bits_k, d.bits_v, n_splits, d.hkv * ((d.gq + 3) / 4), d.batch,
+        n_splits);
   return cuda_status(launch_decode_attn(d, *cache, reinterpret_cast<const __half*>(q),
                                         out, scale_log2, n_splits,
                                         workspace, static_cast<cudaStream_t>(stream)),
@@ -269,6 +294,9 @@ kvq_status kvq_decode_step(const kvq_config* cfg, const kvq_cache* cache, const 
   const __half* kn = reinterpret_cast<const __half*>(k_new);
   const __half* vn = reinterpret_cast<const __half*>(v_new);
   const __half* qh = reinterpret_cast<const __half*>(q);
+  trace("kvq_decode_step batch %d heads %d/%d bits K%dV%d grid (%d, %d, %d) x 512, %d splits",
+        d.batch, d.hq, d.hkv, d.bits_k, d.bits_v, n_splits, d.hkv * ((d.gq + 3) / 4), d.batch,
+        n_splits);
   return cuda_status(launch_decode_step(d, *cache, kn, vn, qh, out, scale_log2, n_splits,
                                         workspace, st),
                      "kvq_decode_step launch");
@@ -351,6 +379,8 @@ kvq_status dgap_restore(const dgap_params* p, float* logits, int32_t batch, int3
     d.logit_tau = -INFINITY;
   else
     d.logit_tau = (float)log((double)p->tau / (1.0 - (double)p->tau));
+  trace("dgap_restore batch %d vocab %d K %d hidden %d tau %g grid (%d, %d) x 256", batch, vocab,
+        p->K, p->hidden, (double)p->tau, d.n_chunks, batch);
   return cuda_status(launch_dgap(d, *p, logits, topk_idx, topk_val, risk, gate, next_token,
                                  features, workspace, static_cast<cudaStream_t>(stream)),
                      "dgap_restore launch");
@@ -377,6 +407,8 @@ kvq_status kvq_drift_metrics(const float* z_fp, const float* z_q, int32_t rows, 
     return fail(KVQ_ERR_ARG, "window must be in [1, k_max] (got %d)", p->window);
   if (!isfinite(p->eps) || !isfinite(p->rho_c))
     return fail(KVQ_ERR_ARG, "eps and rho_c must be finite");
+  trace("kvq_drift_metrics rows %d vocab %d alpha %g window %d k_max %d grid (8, %d) x 512, "
+        "clusters of 8", rows, vocab, (double)p->alpha, p->window, p->k_max, rows);
   return cuda_status(launch_drift(z_fp, z_q, rows, vocab, *p, m_t, c_t, d_loc, y_t, cov,
                                   static_cast<cudaStream_t>(stream)),
                      "kvq_drift_metrics launch");
