@@ -1166,8 +1166,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   float* wv = reinterpret_cast<float*>(smem);           // [gq][S] maxima, then weights
   float* lv = wv + gq * S;                               // [gq][S] sums
   float* lsum = lv + gq * S;                             // [gq]
-  float* osm = lsum + 16;                                // [gq][S][128]
-  const size_t head_bytes = (size_t)(2 * gq * S + 16) * sizeof(float);
+  // the bulk copy's destination starts on a 128-byte boundary
+  const size_t head_bytes = ((size_t)(2 * gq * S + 16) * sizeof(float) + 127) / 128 * 128;
+  float* osm = reinterpret_cast<float*>(smem + head_bytes);  // [gq][S][128]
   const bool staged = head_bytes + o_bytes + 16 <= smem_size;
   uint64_t* mbar = reinterpret_cast<uint64_t*>(smem + smem_size - 16);
   if (staged && threadIdx.x == 0) {
