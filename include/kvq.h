@@ -184,6 +184,17 @@ size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits);
 int32_t kvq_attn_default_splits(const kvq_config* cfg);
 
 /*
+ * A split count for kvq_decode_attn / kvq_decode_step from the sequence
+ * lengths, which the caller knows on the host (the library keeps them on the
+ * device).  lengths: host int32 [batch], each in [0, max_len].  Equals
+ * kvq_attn_default_splits unless the (sequence, kv-head, head group) triples
+ * fill more than half the SMs and the longest length exceeds the mean by
+ * more than 15%: then about four waves of CTAs (a ragged batch is balanced
+ * by the CTA scheduler).  Returns 0 on an invalid argument.
+ */
+int32_t kvq_attn_splits_for_lengths(const kvq_config* cfg, const int32_t* lengths);
+
+/*
  * Zero a workspace (attention or DGAP) once after allocating it.  Both
  * kernels leave their tickets at zero when they finish, so one
  * initialisation serves any number of calls.

@@ -216,6 +216,20 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache, const uint16_
                      "kvq_pack launch");
 }
 
+int32_t kvq_attn_splits_for_lengths(const kvq_config* cfg, const int32_t* lengths) {
+  if (check_config(cfg) != KVQ_OK) return 0;
+  if (!lengths) {
+    fail(KVQ_ERR_ARG, "lengths is NULL");
+    return 0;
+  }
+  for (int b = 0; b < cfg->batch; ++b)
+    if (lengths[b] < 0 || lengths[b] > cfg->max_len) {
+      fail(KVQ_ERR_ARG, "lengths[%d] = %d outside [0, max_len]", b, lengths[b]);
+      return 0;
+    }
+  return attn_splits_for_lengths(make_dims(*cfg), sm_count(), lengths);
+}
+
 int32_t kvq_attn_default_splits(const kvq_config* cfg) {
   if (check_config(cfg) != KVQ_OK) return 0;
   return default_splits(*cfg);

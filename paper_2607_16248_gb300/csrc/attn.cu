@@ -1322,6 +1322,28 @@ int attn_default_splits(const Dims& d, int sm_count) {
   return n < 1 ? 1 : n;
 }
 
+// Split count from the sequence lengths, known to the caller on the host.
+// Up to half the SMs' worth of (sequence, kv-head, head group) triples: one
+// wave, as attn_default_splits.  More: one split each for lengths within 15%
+// of their mean; for a ragged batch about four waves of CTAs, so the
+// scheduler's dynamic fill evens out the long and short sequences.
+int attn_splits_for_lengths(const Dims& d, int sm_count, const int32_t* lengths) {
+  const int bh = d.batch * d.hkv * head_groups(d);
+  if (2 * bh <= sm_count) return attn_default_splits(d, sm_count);
+  long long sum = 0;
+  int mx = 0;
+  for (int b = 0; b < d.batch; ++b) {
+    sum += lengths[b];
+    mx = lengths[b] > mx ? lengths[b] : mx;
+  }
+  if ((double)mx <= 1.15 * (double)sum / d.batch) return attn_default_splits(d, sm_count);
+  int n = (4 * sm_count + bh / 2) / bh;
+  const int cap = (d.max_blocks + 3) / 4;
+  if (n > cap) n = cap;
+  if (n > kMaxSplits - 1) n = kMaxSplits - 1;
+  return n < 1 ? 1 : n;
+}
+
 // ---------------------------------------------------------------------------
 // Decode attention without caller-supplied scratch (kvq_decode_attn_noalloc).
 //

@@ -25,7 +25,8 @@ FLAG_WAIT_TIMEOUT = 2
 EXPORTS = (
     "kvq_last_error", "kvq_version", "kvq_validate_config", "kvq_page_bytes",
     "kvq_cache_layout", "kvq_cache_bind", "kvq_cache_reset", "kvq_pack",
-    "kvq_attn_workspace_bytes", "kvq_attn_default_splits", "kvq_workspace_init",
+    "kvq_attn_workspace_bytes", "kvq_attn_default_splits", "kvq_attn_splits_for_lengths",
+    "kvq_workspace_init",
     "kvq_decode_attn", "kvq_decode_step", "kvq_decode_attn_noalloc", "dgap_workspace_bytes",
     "dgap_restore", "kvq_drift_max_vocab", "kvq_drift_metrics", "kvq_drift_window",
 )
@@ -83,6 +84,7 @@ def lib():
             "kvq_pack": (I32, [cfg_p, cache_p, P, P, I32, I32, I32, P]),
             "kvq_attn_workspace_bytes": (SZ, [cfg_p, I32]),
             "kvq_attn_default_splits": (I32, [cfg_p]),
+            "kvq_attn_splits_for_lengths": (I32, [cfg_p, ctypes.POINTER(I32)]),
             "kvq_workspace_init": (I32, [P, SZ, P]),
             "kvq_decode_attn": (I32, [cfg_p, cache_p, P, P, F32, I32, P, SZ, P]),
             "kvq_decode_step": (I32, [cfg_p, cache_p, P, P, P, P, F32, I32, P, SZ, P]),
@@ -247,6 +249,16 @@ def attn_workspace(cfg: CacheConfig, n_splits=0, device="cuda"):
 def default_splits(cfg: CacheConfig):
     c = cfg.c()
     return lib().kvq_attn_default_splits(ctypes.byref(c))
+
+
+def splits_for_lengths(cfg: CacheConfig, lengths):
+    """kvq_attn_splits_for_lengths: a split count from host-known lengths."""
+    c = cfg.c()
+    arr = (ctypes.c_int32 * cfg.batch)(*[int(x) for x in lengths])
+    n = lib().kvq_attn_splits_for_lengths(ctypes.byref(c), arr)
+    if n == 0:
+        raise KvqError(1, last_error())
+    return n
 
 
 def kvq_decode_attn(cache: QuantKVCache, q, out=None, softmax_scale=0.0, n_splits=0,

@@ -86,6 +86,23 @@ def test_workspace_sizes(L):
     assert L.dgap_workspace_bytes(4, 32, ctypes.byref(p)) == 0  # K must be < vocab
 
 
+def test_splits_for_lengths(L):
+    def n(cfg, lengths):
+        c = cfg.c()
+        return L.kvq_attn_splits_for_lengths(ctypes.byref(c), (ctypes.c_int32 * cfg.batch)(*lengths))
+
+    big = kvq.CacheConfig(batch=16, n_q_heads=32, n_kv_heads=8, bits_k=2, bits_v=2, max_len=32800)
+    d = L.kvq_attn_default_splits(ctypes.byref(big.c()))
+    assert n(big, [20000] * 16) == d  # uniform lengths: the default
+    assert n(big, [20000] * 15 + [22000]) == d  # within 15% of the mean
+    ragged = [8192 + 1500 * i for i in range(16)]
+    assert 3 <= n(big, ragged) <= 8 and n(big, ragged) > d  # about four waves
+    one = kvq.CacheConfig(batch=1, n_q_heads=32, n_kv_heads=8, bits_k=1, bits_v=1, max_len=32800)
+    assert n(one, [32768]) == L.kvq_attn_default_splits(ctypes.byref(one.c()))
+    assert n(big, [20000] * 15 + [40000]) == 0  # beyond max_len
+    assert n(big, [-1] + [20000] * 15) == 0
+
+
 def test_compute_entry_points_reject_bad_arguments(L):
     cfg = _cfg()
     c = cfg.c()
