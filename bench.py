@@ -347,8 +347,8 @@ class Step:
         self.k_new = torch.randn(layers, B, hkv, 128, generator=g, device=device).half()
         self.v_new = torch.randn(layers, B, hkv, 128, generator=g, device=device).half()
         self.out = torch.empty(layers, B, hq, 128, dtype=torch.float32, device=device)
-        self.ws_attn = kvq.attn_workspace(self.cfg, 0, device)
         self.n_splits = kvq.splits_for_lengths(self.cfg, self.lengths0)
+        self.ws_attn = kvq.attn_workspace(self.cfg, self.n_splits, device)
         self.dgap = kvq.DGAP(synth.dgap_weights(seed, K=DGAP_K, hidden=DGAP_HIDDEN), K=DGAP_K,
                              tau=DGAP_TAU, device=device)
         self.logits0 = synth.logits(seed, B, V, device=device)
