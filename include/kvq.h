@@ -170,16 +170,15 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache,
 /*
  * Split-K workspace for kvq_decode_attn: per (sequence, query head, split)
  * partial max, sum and fp32 output row for up to n_splits + 1 splits, plus
- * one ticket per (sequence, kv-head, head group), sized one per query head.
+ * one ticket per (sequence, kv-head) (the size allows one per query head).
  * n_splits = 0 means the library's choice.  Returns 0 on an invalid config.
  */
 size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits);
 
 /*
  * The split count kvq_decode_attn uses when passed n_splits = 0: one
- * 512-thread CTA per SM over all (sequence, kv-head, head group) triples,
- * SMs / (batch * n_kv_heads * ceil(group / 4)), between 1 and 255, where
- * group = n_q_heads / n_kv_heads.
+ * 512-thread CTA per SM over all (sequence, kv-head) pairs,
+ * SMs / (batch * n_kv_heads), between 1 and 255.
  */
 int32_t kvq_attn_default_splits(const kvq_config* cfg);
 
@@ -187,8 +186,8 @@ int32_t kvq_attn_default_splits(const kvq_config* cfg);
  * A split count for kvq_decode_attn / kvq_decode_step from the sequence
  * lengths, which the caller knows on the host (the library keeps them on the
  * device).  lengths: host int32 [batch], each in [0, max_len].  Equals
- * kvq_attn_default_splits unless the (sequence, kv-head, head group) triples
- * fill more than half the SMs and the longest length exceeds the mean by
+ * kvq_attn_default_splits unless the (sequence, kv-head) pairs fill more
+ * than half the SMs and the longest length exceeds the mean by
  * more than 15%: then about four waves of CTAs (a ragged batch is balanced
  * by the CTA scheduler).  Returns 0 on an invalid argument.
  */
@@ -212,11 +211,8 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream);
  *                  fp32 accumulation result; rounding it to fp16 is left to
  *                  the caller).
  *   softmax_scale  0 selects 1/sqrt(128).
- *   n_splits       CTAs per (sequence, kv-head, head group) that share the
- *                  kv-head's 32-token blocks and window chunks (a head group
- *                  is a run of at most 4 query heads of one kv-head; a group
- *                  of 5..8 heads has two, whose CTAs read the same pages);
- *                  0 = kvq_attn_default_splits(cfg);
+ *   n_splits       CTAs per (sequence, kv-head) that share its 32-token
+ *                  blocks and window chunks; 0 = kvq_attn_default_splits(cfg);
  *                  else 1..255.  With more than one, each CTA writes a partial
  *                  (max, sum, output row) to the workspace and the last to
  *                  finish merges them.

@@ -1,19 +1,15 @@
 // kvq_decode_attn: one decode step of grouped-query attention
 // softmax(q K^T * scale) V (Sec. 1 of the paper) over the packed KbVb cache.
 //
-// Grid (S, n_kv_heads * G, batch) of 512-thread CTAs, one per SM, where G =
-// ceil(group / 4): the query heads of a kv-head are cut into G head groups of
-// at most 4 (the MMA's head columns) and each head group has its own S CTAs.
-// The G CTA sets of a kv-head are launched next to each other and stream the
-// same pages at the same time, so all but one read of a page come from L2.
-// The S CTAs of one (sequence, kv-head, head group) share its work: the packed 32-token blocks and
+// Grid (S, n_kv_heads, batch) of 512-thread CTAs, one per SM.  The S CTAs
+// of one (sequence, kv-head) share its work: the packed 32-token blocks and
 // the 32-token chunks of the fp16 residual window are cut into contiguous
 // ranges, one per warp (a warp takes only blocks or only window chunks).
 // Each warp streams its own pages into a private ring of shared-memory slots
 // with bulk asynchronous copies (cp.async.bulk + one mbarrier per slot) and
 // keeps a running softmax state.  The warps of a CTA merge in shared memory
 // into one partial (max, sum, unnormalised row) per query head; with S > 1
-// the last CTA of a (sequence, kv-head, head group) to finish (atomic ticket, no
+// the last CTA of a (sequence, kv-head) to finish (atomic ticket, no
 // waiting) merges the S partials:
 //   out = sum_s 2^{m_s - M} o_s / sum_s 2^{m_s - M} l_s.
 // Scores are kept in the log2 domain (scaled by softmax_scale * log2 e).
@@ -24,13 +20,17 @@
 //
 //   keys    S[t][h] = sum_c code[t][c] * (q_h[c] s_c) + sum_c q_h[c] z_c
 //           A = codes (M = tokens, K = channels), B = q*s split into an fp16
-//           high part (columns 0..3) and its exact fp16 residual (columns
-//           4..7, the padding of the 4 query heads), so the products are
+//           high part and its exact fp16 residual, so the products are
 //           exact; the zero-point term is one more MMA with A = z, B = q.
 //   values  o[c][h] += sum_t code[t][c] * (p_h[t] s_t,g) + sum_t p_h[t] z_t,g
 //           A = codes (M = channels, K = tokens), B = p*s with p split into
-//           high / low fp16 parts in columns 0..3 / 4..7; P moves from the
-//           score (accumulator) layout to the B layout with movmatrix.
+//           high / low fp16 parts; P moves from the score (accumulator)
+//           layout to the B layout with movmatrix.
+// The B operand's 8 columns hold, for query groups of up to 4 heads, the
+// high parts of the 4 heads in columns 0..3 and the low parts in 4..7 (one
+// MMA per operand pair, "narrow"); for groups of 5..8 heads one head per
+// column, and the high and low parts are two MMAs into the same accumulator
+// ("wide"), so the codes of a block are converted once for all heads.
 //
 // Codes become fp16 values without a table: for 1-bit codes (stored in
 // fragment order) a rotated bit lands on an exponent bit (value 2^e), for
@@ -55,10 +55,7 @@ constexpr int kWarps = KVQ_ATTN_WARPS;            // warps per CTA
 constexpr int kThreads = 32 * kWarps;
 constexpr int kCtasPerSm = kWarps <= 8 ? 2 : 1;   // resident CTAs per SM
 constexpr int kRingBudget = (kCtasPerSm == 2 ? 96 : 192) * 1024;  // staged page bytes per CTA
-constexpr int kHeads = 4;  // query heads per CTA (the head columns of the MMAs)
-
-// Head groups per kv-head: its query heads in runs of at most kHeads.
-__host__ __device__ inline int head_groups(const Dims& d) { return (d.gq + kHeads - 1) / kHeads; }
+constexpr int kHeads = kMaxGq;  // query heads per CTA (the wide layout's head columns)
 constexpr long long kWaitCycles = 4000000000LL;  // bounded mbarrier waits (~2 s)
 constexpr int kZeroBytes = 512;                   // all-zero metadata rows
 
@@ -66,7 +63,7 @@ struct Ws {
   float* m;       // [B][Hq][S]
   float* l;       // [B][Hq][S]
   float* o;       // [B][Hq][S][128]
-  unsigned* tk;   // [B][Hkv][head groups] (sized [B][Hq])
+  unsigned* tk;   // [B][Hkv] (sized [B][Hq])
 };
 
 __host__ __device__ inline size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -86,7 +83,7 @@ __host__ __device__ inline Ws carve(void* base, int batch, int hq, int hkv, int 
 }
 
 // A warp's final state (row maximum, row sum, unnormalised output row per
-// query head of the CTA's head group), written at the start of the warp's own
+// query head of the kv-head), written at the start of the warp's own
 // ring as soon as it is done.
 struct WarpState {
   float m[kHeads];
@@ -295,12 +292,16 @@ struct TcState {
 };
 
 // Online softmax over NB 32-token blocks (per block 4 token rows x 2 heads
-// per lane; lanes tig and tig^2 hold the same scores), then the
-// probabilities as fp16 high / low parts (columns 0..3 / 4..7) moved to the
+// per lane), then the probabilities as fp16 high / low parts moved to the
 // B-operand layout of the value MMAs with movmatrix.
-template <int NB>
+//   narrow (up to 4 heads): columns 0..3 / 4..7 hold the high / low parts of
+//     heads 0..3 (lanes tig and tig^2 hold the same scores); pt is one
+//     operand whose columns carry both parts;
+//   wide (5..8 heads): column = head; pt holds the high parts, pl the low
+//     parts, each one operand of its own MMA.
+template <int NB, bool kWide>
 __device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, const Lane& ln,
-                                           uint32_t (&pt)[NB][2][2]) {
+                                           uint32_t (&pt)[NB][2][2], uint32_t (&pl)[NB][2][2]) {
   float mx[2];
 #pragma unroll
   for (int hh = 0; hh < 2; ++hh) {
@@ -346,15 +347,24 @@ __device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, c
         const float p1 = fast_exp2(sc[bi][j][1] - st.m[1]);
         st.l[0] += p0;
         st.l[1] += p1;
-        const float2 hf = __half22float2(__floats2half2_rn(p0, p1));
-        const __half2 r = __floats2half2_rn(fmaf(-ln.p_lo, hf.x, p0), fmaf(-ln.p_lo, hf.y, p1));
-        pt[bi][mt][rh] = movmatrix_t(h2u(r));
+        const __half2 h = __floats2half2_rn(p0, p1);
+        const float2 hf = __half22float2(h);
+        if constexpr (kWide) {
+          pt[bi][mt][rh] = movmatrix_t(h2u(h));
+          pl[bi][mt][rh] = movmatrix_t(h2u(__floats2half2_rn(p0 - hf.x, p1 - hf.y)));
+        } else {
+          const __half2 r =
+              __floats2half2_rn(fmaf(-ln.p_lo, hf.x, p0), fmaf(-ln.p_lo, hf.y, p1));
+          pt[bi][mt][rh] = movmatrix_t(h2u(r));
+        }
       }
 }
 
 // NB packed 32-token blocks (pages in shared memory) for one warp: scores of
-// all blocks, one softmax update, then the value MMAs.
-template <int BK, int BV, int NB>
+// all blocks, one softmax update, then the value MMAs.  Narrow: one MMA per
+// operand pair, B columns = (head, part); wide: B column = head, and the
+// high and low parts of B are two MMAs into the same accumulator.
+template <int BK, int BV, int NB, bool kWide>
 __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char* zero,
                                         const uint32_t (&qb)[16], const Lane& ln,
                                         float scale_log2, TcState& st) {
@@ -384,7 +394,7 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
       const char* kmeta = pg[bi] + page_off_kmeta(BK);
       // scales of channels c..c+3 (two fp16 per word)
       const uint2 sw = *reinterpret_cast<const uint2*>(kmeta + 2 * c);
-      uint32_t a0[4], a1[4], b[2];
+      uint32_t a0[4], a1[4], b[2], bl[2];
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         uint32_t v[4];
@@ -400,17 +410,28 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
         a1[2 * half] = v[2];
         a1[2 * half + 1] = v[3];
         const uint32_t s2 = half ? sw.y : sw.x;
-        // q*s as fp16 high part (columns 0..3) or its exact residual (4..7)
         const __half2 hi = __hmul2(u2h(qb[2 * ks + half]), u2h(s2));
-        b[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hmul2(hi, u2h(ln.neg_lo))));
+        if constexpr (kWide) {
+          // q*s as its fp16 high part and exact residual, two operands
+          b[half] = h2u(hi);
+          bl[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hneg2(hi)));
+        } else {
+          // q*s as fp16 high part (columns 0..3) or its exact residual (4..7)
+          b[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hmul2(hi, u2h(ln.neg_lo))));
+        }
       }
       mma16816(dk[bi][0], a0[0], a0[1], a0[2], a0[3], b[0], b[1]);
       mma16816(dk[bi][1], a1[0], a1[1], a1[2], a1[3], b[0], b[1]);
+      if constexpr (kWide) {
+        mma16816(dk[bi][0], a0[0], a0[1], a0[2], a0[3], bl[0], bl[1]);
+        mma16816(dk[bi][1], a1[0], a1[1], a1[2], a1[3], bl[0], bl[1]);
+      }
     }
     const uint2 zw = *reinterpret_cast<const uint2*>(zrow + 2 * (kHeadDim + c));
     mma16816(dz, zw.x, 0u, zw.y, 0u, qb[2 * ks], qb[2 * ks + 1]);
   }
-  // Scores in the log2 domain.  Lanes tig and tig^2 hold the two parts.
+  // Scores in the log2 domain.  Narrow: lanes tig and tig^2 hold the two
+  // parts; wide: the accumulator holds the whole score.
   float sc[NB][4][2];
 #pragma unroll
   for (int bi = 0; bi < NB; ++bi) {
@@ -424,13 +445,13 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
         for (int hh = 0; hh < 2; ++hh) {
           const int j = 2 * mt + rh;
           const float d = dk[bi][mt][2 * rh + hh];
-          const float full = d + __shfl_xor_sync(0xffffffffu, d, 2);
+          const float full = kWide ? d : d + __shfl_xor_sync(0xffffffffu, d, 2);
           sc[bi][j][hh] = fmaf(full, Codes<BK>::inv(j) * scale_log2, hh ? z1 : z0);
         }
   }
 
-  uint32_t pt[NB][2][2];
-  tc_softmax<NB>(sc, st, ln, pt);
+  uint32_t pt[NB][2][2], pl[NB][2][2];
+  tc_softmax<NB, kWide>(sc, st, ln, pt, pl);
 
   // ---- values: o^T[c][h] ----
   // Value scales and zeros are stored in token pairs (t, t + 4), so the
@@ -444,18 +465,28 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
     const uint4 z8 = *reinterpret_cast<const uint4*>(vzrow + 2 * (kHeadDim + 32 * (gid & 3) + 8 * tig));
     mma16816(st.zv, z8.x, 0u, z8.y, 0u, pt[bi][0][0], pt[bi][0][1]);
     mma16816(st.zv, z8.z, 0u, z8.w, 0u, pt[bi][1][0], pt[bi][1][1]);
-    // B = p * s in two fp16 parts, columns 0..3 and 4..7: the high part is
-    // RN16(p_hi s); the low part RN16(p_lo s + (p_hi s - RN16(p_hi s))), so
-    // rounding the product costs no accuracy.  Lanes of columns 4..7 hold p_lo
-    // after movmatrix and fetch p_hi from lane - 16.
+    if constexpr (kWide) {
+      mma16816(st.zv, z8.x, 0u, z8.y, 0u, pl[bi][0][0], pl[bi][0][1]);
+      mma16816(st.zv, z8.z, 0u, z8.w, 0u, pl[bi][1][0], pl[bi][1][1]);
+    }
+    // B = p * s in two fp16 parts: the high part is RN16(p_hi s); the low
+    // part RN16(p_lo s + (p_hi s - RN16(p_hi s))), so rounding the product
+    // costs no accuracy.  Narrow: columns 0..3 / 4..7, lanes of columns 4..7
+    // hold p_lo after movmatrix and fetch p_hi from lane - 16; wide: every
+    // lane has both parts of its head.
     uint32_t pa[2][2], pb[2][2];
 #pragma unroll
     for (int ks = 0; ks < 2; ++ks)
 #pragma unroll
       for (int dl = 0; dl < 2; ++dl) {
-        const uint32_t other = __shfl_xor_sync(0xffffffffu, pt[bi][ks][dl], 16);
-        pa[ks][dl] = lane < 16 ? pt[bi][ks][dl] : other;
-        pb[ks][dl] = lane < 16 ? 0u : pt[bi][ks][dl];
+        if constexpr (kWide) {
+          pa[ks][dl] = pt[bi][ks][dl];
+          pb[ks][dl] = pl[bi][ks][dl];
+        } else {
+          const uint32_t other = __shfl_xor_sync(0xffffffffu, pt[bi][ks][dl], 16);
+          pa[ks][dl] = lane < 16 ? pt[bi][ks][dl] : other;
+          pb[ks][dl] = lane < 16 ? 0u : pt[bi][ks][dl];
+        }
       }
     uint4 vw1;
     if constexpr (BV == 1) vw1 = *reinterpret_cast<const uint4*>(vc + 16 * lane);
@@ -471,7 +502,7 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
       }
 #pragma unroll
       for (int ks = 0; ks < 2; ++ks) {
-        uint32_t am0[4], am1[4], bv[2];
+        uint32_t am0[4], am1[4], bv[2], bw[2];
 #pragma unroll
         for (int dl = 0; dl < 2; ++dl) {
           const int ia = 2 * ks + dl, ib = ia + 4;  // tokens 8tig + ia, 8tig + ib
@@ -484,11 +515,21 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
           am1[2 * dl + 1] = v[3];
           const __half2 sc = u2h(mw[ia]);
           const __half2 t = __hmul2(u2h(pa[ks][dl]), sc);
-          const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hmul2(t, u2h(ln.neg_lo)));
-          bv[dl] = h2u(__hfma2(u2h(pb[ks][dl]), sc, err));
+          if constexpr (kWide) {
+            const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hneg2(t));
+            bv[dl] = h2u(t);
+            bw[dl] = h2u(__hfma2(u2h(pb[ks][dl]), sc, err));
+          } else {
+            const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hmul2(t, u2h(ln.neg_lo)));
+            bv[dl] = h2u(__hfma2(u2h(pb[ks][dl]), sc, err));
+          }
         }
         mma16816(st.acc[2 * g], am0[0], am0[1], am0[2], am0[3], bv[0], bv[1]);
         mma16816(st.acc[2 * g + 1], am1[0], am1[1], am1[2], am1[3], bv[0], bv[1]);
+        if constexpr (kWide) {
+          mma16816(st.acc[2 * g], am0[0], am0[1], am0[2], am0[3], bw[0], bw[1]);
+          mma16816(st.acc[2 * g + 1], am1[0], am1[1], am1[2], am1[3], bw[0], bw[1]);
+        }
       }
     }
   }
@@ -508,13 +549,14 @@ __device__ __forceinline__ Lane make_lane(int lane) {
   return ln;
 }
 
-// q of head gid & 3 in the B layout (exact fp16), zero beyond the group.
-// kPermuted: the packed path's K-slot order (four contiguous channels per
-// lane); otherwise slot k of a k-step is channel 16 ks + k.
-template <bool kPermuted>
+// q of head gid & 3 (narrow) or gid (wide) in the B layout (exact fp16),
+// zero beyond the group.  kPermuted: the packed path's K-slot order (four
+// contiguous channels per lane); otherwise slot k of a k-step is channel
+// 16 ks + k.
+template <bool kPermuted, bool kWide>
 __device__ __forceinline__ void load_qb(uint32_t (&qb)[16], const __half* qh, int gq,
                                         const Lane& ln) {
-  const int head = ln.gid & 3;
+  const int head = kWide ? ln.gid : ln.gid & 3;
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks)
 #pragma unroll
@@ -537,10 +579,11 @@ __device__ __forceinline__ void init_state(TcState& st) {
 }
 
 // A warp's running state to the merge area: row maximum, row sum and the
-// unnormalised output row of heads 0..3.  kPacked: channel rows follow the
+// unnormalised output row of heads 0..3 (narrow: the two parts in columns
+// tig and tig^2 are added) or 0..7 (wide).  kPacked: channel rows follow the
 // packed layout (nibble of a group, power-of-two factors, zero-point term);
 // otherwise channel = 16 * m-tile + row.
-template <bool kPacked, int BV>
+template <bool kPacked, int BV, bool kWide>
 __device__ __forceinline__ void tc_write_state(const TcState& st, WarpState& ws, int lane) {
   const int gid = lane >> 2, tig = lane & 3;
   float l0 = st.l[0], l1 = st.l[1];
@@ -550,9 +593,9 @@ __device__ __forceinline__ void tc_write_state(const TcState& st, WarpState& ws,
     l1 += __shfl_xor_sync(0xffffffffu, l1, o);
   }
   float zsum[2];
-  zsum[0] = st.zv[0] + __shfl_xor_sync(0xffffffffu, st.zv[0], 2);
-  zsum[1] = st.zv[1] + __shfl_xor_sync(0xffffffffu, st.zv[1], 2);
-  if (gid == 0 && tig < 2) {
+  zsum[0] = kWide ? st.zv[0] : st.zv[0] + __shfl_xor_sync(0xffffffffu, st.zv[0], 2);
+  zsum[1] = kWide ? st.zv[1] : st.zv[1] + __shfl_xor_sync(0xffffffffu, st.zv[1], 2);
+  if (gid == 0 && (kWide || tig < 2)) {
     ws.m[2 * tig] = st.m[0];
     ws.m[2 * tig + 1] = st.m[1];
     ws.l[2 * tig] = l0;
@@ -573,8 +616,8 @@ __device__ __forceinline__ void tc_write_state(const TcState& st, WarpState& ws,
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
           const float a = st.acc[mtp][2 * rh + hh];
-          const float full_v = a + __shfl_xor_sync(0xffffffffu, a, 2);
-          if (tig < 2) ws.o[2 * tig + hh][cch] = fmaf(full_v, inv, hh ? zg1 : zg0);
+          const float full_v = kWide ? a : a + __shfl_xor_sync(0xffffffffu, a, 2);
+          if (kWide || tig < 2) ws.o[2 * tig + hh][cch] = fmaf(full_v, inv, hh ? zg1 : zg0);
         }
       }
     }
@@ -610,10 +653,11 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t 
                : "memory");
 }
 
+template <bool kWide>
 __device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
                                                 const uint32_t (&qb)[16], const Lane& ln,
                                                 float scale_log2, TcState& st,
-                                                uint32_t (&pt)[1][2][2]) {
+                                                uint32_t (&pt)[1][2][2], uint32_t (&pl)[1][2][2]) {
   const int lane = threadIdx.x & 31;
   const int mi = lane >> 3, r8 = lane & 7;
   float dk[2][4] = {};
@@ -635,11 +679,12 @@ __device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
       for (int hh = 0; hh < 2; ++hh)
         sc[0][2 * mt + rh][hh] = ok ? dk[mt][2 * rh + hh] * scale_log2 : -INFINITY;
     }
-  tc_softmax<1>(sc, st, ln, pt);
+  tc_softmax<1, kWide>(sc, st, ln, pt, pl);
 }
 
+template <bool kWide>
 __device__ __forceinline__ void tc_resid_values(const __half* vs_s, const uint32_t (&pt)[1][2][2],
-                                                TcState& st) {
+                                                const uint32_t (&pl)[1][2][2], TcState& st) {
   const int lane = threadIdx.x & 31;
   const int mi = lane >> 3, r8 = lane & 7;
 #pragma unroll
@@ -649,6 +694,7 @@ __device__ __forceinline__ void tc_resid_values(const __half* vs_s, const uint32
       uint32_t a[4];
       ldsm_x4_t(a, vs_s + (16 * ks + 8 * (mi >> 1) + r8) * kResRow + 16 * mtp + 8 * (mi & 1));
       mma16816(st.acc[mtp], a[0], a[1], a[2], a[3], pt[0][ks][0], pt[0][ks][1]);
+      if constexpr (kWide) mma16816(st.acc[mtp], a[0], a[1], a[2], a[3], pl[0][ks][0], pl[0][ks][1]);
     }
 }
 
@@ -741,8 +787,8 @@ __device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int 
 // Decode step with a flush: the 32-token block of positions [p0, p0 + 32),
 // still fp16 in the ring, leaves the window.  One warp quantizes it exactly as
 // kvq_pack does (same quantizer, same page layout) into a page image in
-// `image` (shared memory) and, if `page_out` is set, writes the page there
-// (other head groups of the kv-head build the same image); the caller folds
+// `image` (shared memory) and, if `page_out` is set, writes the page there;
+// the caller folds
 // the image into its state like any streamed block.  Kept out of line: it is
 // rare and its registers would otherwise crowd the streaming loop.
 template <int BK, int BV>
@@ -816,11 +862,11 @@ __device__ __noinline__ void flush_block(const __half* ring_k, const __half* rin
 
 // Fold blocks [lo, hi) into st; `pre` slots holding blocks [lo_h, pre_end)
 // were streamed early.
-template <int BK, int BV>
+template <int BK, int BV, bool kWide>
 __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_end, int lo, int hi_all,
                                char* ring, uint64_t* full, int R, const char* zero,
                                const __half* qh, int gq, float scale_log2, unsigned* flag,
-                               TcState& st, int flush_blk, bool write_page, const __half* ring_k,
+                               TcState& st, int flush_blk, const __half* ring_k,
                                const __half* ring_v, int ring_size) {
   constexpr int page = page_bytes_c(BK, BV);
   constexpr int NB = ring_blocks(page);
@@ -846,7 +892,7 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
 
   const Lane ln = make_lane<BK, BV>(lane);
   uint32_t qb[16];
-  load_qb<true>(qb, qh, gq, ln);
+  load_qb<true, kWide>(qb, qh, gq, ln);
   int consumed = 0;
   for (int s = 0; s < total; ++s) {
     const int slot = s % R;
@@ -863,10 +909,10 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
         const char* pg[NB];
 #pragma unroll
         for (int i = 0; i < NB; ++i) pg[i] = base + i * page;
-        tc_unit<BK, BV, NB>(pg, zero, qb, ln, scale_log2, st);
+        tc_unit<BK, BV, NB, kWide>(pg, zero, qb, ln, scale_log2, st);
       } else {
         const char* pg[1] = {base};
-        tc_unit<BK, BV, 1>(pg, zero, qb, ln, scale_log2, st);
+        tc_unit<BK, BV, 1, kWide>(pg, zero, qb, ln, scale_log2, st);
       }
     }
     __syncwarp();
@@ -883,10 +929,9 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
   __syncwarp();
   if (flush) {
     flush_block<BK, BV>(ring_k, ring_v, flush_blk * kGroup, ring_size, ring,
-                        write_page ? const_cast<char*>(pages_bh) + (long long)flush_blk * page
-                                   : nullptr);
+                        const_cast<char*>(pages_bh) + (long long)flush_blk * page);
     const char* pg[1] = {ring};
-    tc_unit<BK, BV, 1>(pg, zero, qb, ln, scale_log2, st);
+    tc_unit<BK, BV, 1, kWide>(pg, zero, qb, ln, scale_log2, st);
   }
 }
 
@@ -935,7 +980,7 @@ __device__ __forceinline__ void prefetch_rows_l2(const __half* ring_base, int p0
 }
 
 // Window warp: chunks c0, c0 + stride, ... of the fp16 window.
-template <int BK, int BV>
+template <int BK, int BV, bool kWide>
 __device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half* ring_v,
                                const Plan& p, int L, int c0, int stride, char* area,
                                const __half* qh, int gq, float scale_log2, TcState& st,
@@ -944,24 +989,24 @@ __device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half
   const int lane = threadIdx.x & 31;
   const Lane ln = make_lane<BK, BV>(lane);
   uint32_t qb[16];
-  load_qb<false>(qb, qh, gq, ln);
+  load_qb<false, kWide>(qb, qh, gq, ln);
   __half* rows = reinterpret_cast<__half*>(area);
   uint32_t phase = 0u;
   for (int u = c0; u < p.n_res; u += stride) {
     const int p0 = p.Lq + u * kGroup;
     const int n_tok = min(kGroup, L - p0);
-    uint32_t pt[1][2][2];
+    uint32_t pt[1][2][2], pl[1][2][2];
     if (!stage_rows_bulk(rows, ring_k, p0, n_tok, d.ring, p_new, k_row, bar, phase++ & 1u)) {
       if ((threadIdx.x & 31) == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
       return;
     }
-    tc_resid_scores(rows, n_tok, qb, ln, scale_log2, st, pt);
+    tc_resid_scores<kWide>(rows, n_tok, qb, ln, scale_log2, st, pt, pl);
     __syncwarp();
     if (!stage_rows_bulk(rows, ring_v, p0, n_tok, d.ring, p_new, v_row, bar, phase++ & 1u)) {
       if ((threadIdx.x & 31) == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
       return;
     }
-    tc_resid_values(rows, pt, st);
+    tc_resid_values<kWide>(rows, pt, pl, st);
     __syncwarp();
   }
 }
@@ -976,7 +1021,7 @@ __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
 // The kernel
 // ---------------------------------------------------------------------------
 
-template <int BK, int BV>
+template <int BK, int BV, bool kWide>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     decode_attn_kernel(Dims d, kvq_cache c, const __half* __restrict__ q, float* __restrict__ out,
                        float scale_log2, int S, unsigned smem_size, Ws ws,
@@ -987,26 +1032,22 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   __shared__ __align__(16) __half q_s[kHeads * kHeadDim];  // the CTA's query heads
   __shared__ __align__(8) uint64_t wbar[kWarps];      // a window warp's staging barrier
 
-  // head group hg of kv-head h: query heads h * group + 4 hg + [0, gq)
-  const int n_hg = head_groups(d);
-  const int h = blockIdx.y / n_hg, hg = blockIdx.y - h * n_hg, b = blockIdx.z;
-  const int gq = min(kHeads, d.gq - kHeads * hg);
+  const int h = blockIdx.y, b = blockIdx.z;
+  const int gq = d.gq;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int NV = gridDim.x * kWarps;     // warps per (sequence, kv-head, head group)
+  const int NV = gridDim.x * kWarps;     // warps per (sequence, kv-head)
   const int v = blockIdx.x * kWarps + warp;
   pdl_launch_dependents();
   const long long bh = (long long)b * d.hkv + h;
   const char* pages = static_cast<const char*>(c.pages) + bh * d.max_blocks * d.page_bytes;
   const __half* ring_k = reinterpret_cast<const __half*>(c.k_resid) + bh * d.ring * kHeadDim;
   const __half* ring_v = reinterpret_cast<const __half*>(c.v_resid) + bh * d.ring * kHeadDim;
-  const long long head0 = (long long)b * d.hq + (long long)h * d.gq + kHeads * hg;
+  const long long head0 = (long long)b * d.hq + (long long)h * gq;
   const __half* qh = q + head0 * kHeadDim;
   unsigned* flag = reinterpret_cast<unsigned*>(c.seq_len) + d.batch;
   // Decode step (k_new given): this kernel appends one token per sequence
   // before attending.  seq_len[b] is read once per CTA; the last CTA of the
-  // sequence to have read it (ticket) publishes L0 + 1.  Head group 0 writes
-  // the new ring row and flushed pages; the other groups compute the same
-  // values for their own use.
+  // sequence to have read it (ticket) publishes L0 + 1.
   const bool append = k_new != nullptr;
   unsigned seq_ticket = 0u;
 
@@ -1074,7 +1115,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       seq_ticket = atomicAdd(reinterpret_cast<unsigned*>(c.seq_len) + d.batch + 2 + b, 1u);
     const __half* k_row = grew ? k_new + bh * kHeadDim : nullptr;
     const __half* v_row = grew ? v_new + bh * kHeadDim : nullptr;
-    if (grew && blockIdx.x == 0 && hg == 0 && warp == 0) {  // the new token into its ring slot
+    if (grew && blockIdx.x == 0 && warp == 0) {  // the new token into its ring slot
       const long long slot = (long long)(L0 % d.ring) * kHeadDim;
       __half* rk = const_cast<__half*>(ring_k) + slot;
       __half* rv = const_cast<__half*>(ring_v) + slot;
@@ -1094,17 +1135,17 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         lo = hi = 0;
         if (packed) block_range(p, v, lo, hi);
       }
-      tc_packed_warp<BK, BV>(pages, lo_h, pre, pre_end, lo, hi, ring, full, R,
+      tc_packed_warp<BK, BV, kWide>(pages, lo_h, pre, pre_end, lo, hi, ring, full, R,
                              reinterpret_cast<const char*>(zero), q_s, gq, scale_log2, flag, st,
-                             flush_blk, hg == 0, ring_k, ring_v, d.ring);
+                             flush_blk, ring_k, ring_v, d.ring);
     }
     if (!packed)
-      tc_window_warp<BK, BV>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, q_s, gq,
+      tc_window_warp<BK, BV, kWide>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, q_s, gq,
                              scale_log2, st, grew ? L0 : -1, k_row, v_row, &wbar[warp], flag);
     // the warp's ring is idle now: its state goes to the start of it
     WarpState& mine = *reinterpret_cast<WarpState*>(ring);
-    if (packed) tc_write_state<true, BV>(st, mine, lane);
-    else tc_write_state<false, BV>(st, mine, lane);
+    if (packed) tc_write_state<true, BV, kWide>(st, mine, lane);
+    else tc_write_state<false, BV, kWide>(st, mine, lane);
   }
   __syncthreads();
 
@@ -1153,13 +1194,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   }
   if (S == 1) return;
 
-  // ---- the last CTA of this (sequence, kv-head, head group) merges the S partials ----
-  const long long bhg = (long long)b * gridDim.y + blockIdx.y;
+  // ---- the last CTA of this (sequence, kv-head) merges the S partials ----
   __syncthreads();
-  if (threadIdx.x == 0) ms.last = atom_add_acq_rel(&ws.tk[bhg], 1u) == (unsigned)S - 1;
+  if (threadIdx.x == 0) ms.last = atom_add_acq_rel(&ws.tk[bh], 1u) == (unsigned)S - 1;
   __syncthreads();
   if (!ms.last) return;
-  // The partial rows of this head group are one contiguous range: a
+  // The partial rows of this (sequence, kv-head) are one contiguous range: a
   // bulk copy brings them into shared memory (when they fit) while the maxima
   // and sums are loaded and turned into weights.
   const size_t o_bytes = (size_t)gq * S * kHeadDim * sizeof(float);
@@ -1215,7 +1255,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     const float Ls = lsum[g];
     out[(head0 + g) * kHeadDim + ch] = Ls > 0.0f ? o / Ls : 0.0f;
   }
-  if (threadIdx.x == 0) ws.tk[bhg] = 0u;
+  if (threadIdx.x == 0) ws.tk[bh] = 0u;
 }
 
 size_t smem_bytes(const Dims& d) {
@@ -1226,19 +1266,25 @@ size_t smem_bytes(const Dims& d) {
   return (rings + kZeroBytes + 16 + 127) / 128 * 128;
 }
 
-template <int BK, int BV>
+template <int BK, int BV, bool kWide>
 cudaError_t prepare(const Dims& d) {
-  return cudaFuncSetAttribute(decode_attn_kernel<BK, BV>,
+  return cudaFuncSetAttribute(decode_attn_kernel<BK, BV, kWide>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes(d));
 }
 
+// Kernel instance for (bits_k, bits_v, query-group width): groups of up to 4
+// heads take the narrow MMA layout, 5..8 heads the wide one.
+template <int BK, int BV, typename Op>
+cudaError_t dispatch_width(const Dims& d, const Op& op) {
+  return d.gq <= 4 ? op.template run<BK, BV, false>() : op.template run<BK, BV, true>();
+}
 template <int BK, typename Op>
 cudaError_t dispatch_bv(const Dims& d, const Op& op) {
   switch (d.bits_v) {
-    case 1: return op.template run<BK, 1>();
-    case 2: return op.template run<BK, 2>();
-    case 4: return op.template run<BK, 4>();
-    default: return op.template run<BK, 8>();
+    case 1: return dispatch_width<BK, 1>(d, op);
+    case 2: return dispatch_width<BK, 2>(d, op);
+    case 4: return dispatch_width<BK, 4>(d, op);
+    default: return dispatch_width<BK, 8>(d, op);
   }
 }
 template <typename Op>
@@ -1262,12 +1308,12 @@ struct LaunchOp {
   cudaStream_t st;
   const __half* k_new = nullptr;
   const __half* v_new = nullptr;
-  template <int BK, int BV>
+  template <int BK, int BV, bool kWide>
   cudaError_t run() const {
-    cudaError_t e = prepare<BK, BV>(d);
+    cudaError_t e = prepare<BK, BV, kWide>(d);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(S, d.hkv * head_groups(d), d.batch);
+    cfg.gridDim = dim3(S, d.hkv, d.batch);
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem_bytes(d);
     cfg.stream = st;
@@ -1276,7 +1322,7 @@ struct LaunchOp {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV>, d, c, q, out, sl2, S,
+    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV, kWide>, d, c, q, out, sl2, S,
                            (unsigned)smem_bytes(d), ws, k_new, v_new);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
@@ -1285,9 +1331,8 @@ struct LaunchOp {
 
 }  // namespace
 
-// n_splits = CTAs per (sequence, kv-head, head group); workspace rows for up
-// to n_splits.  Tickets: one per (sequence, kv-head, head group), at most one
-// per query head.
+// n_splits = CTAs per (sequence, kv-head); workspace rows for up to
+// n_splits.  Tickets: one per (sequence, kv-head), sized one per query head.
 size_t attn_workspace_bytes(const Dims& d, int n_splits) {
   const int S = n_splits + 1;
   const size_t nml = (size_t)d.batch * d.hq * S;
@@ -1311,10 +1356,10 @@ cudaError_t launch_decode_step(const Dims& d, const kvq_cache& c, const __half* 
   return dispatch(d, op);
 }
 
-// CTAs per (sequence, kv-head, head group): enough for every resident CTA
+// CTAs per (sequence, kv-head): enough for every resident CTA
 // slot of the GPU to hold one, with at least a few blocks per CTA.
 int attn_default_splits(const Dims& d, int sm_count) {
-  const int bh = d.batch * d.hkv * head_groups(d);
+  const int bh = d.batch * d.hkv;
   int n = kCtasPerSm * sm_count / bh;
   const int cap = (d.max_blocks + 3) / 4;
   if (n > cap) n = cap;
@@ -1323,12 +1368,12 @@ int attn_default_splits(const Dims& d, int sm_count) {
 }
 
 // Split count from the sequence lengths, known to the caller on the host.
-// Up to half the SMs' worth of (sequence, kv-head, head group) triples: one
+// Up to half the SMs' worth of (sequence, kv-head) pairs: one
 // wave, as attn_default_splits.  More: one split each for lengths within 15%
 // of their mean; for a ragged batch about four waves of CTAs, so the
 // scheduler's dynamic fill evens out the long and short sequences.
 int attn_splits_for_lengths(const Dims& d, int sm_count, const int32_t* lengths) {
-  const int bh = d.batch * d.hkv * head_groups(d);
+  const int bh = d.batch * d.hkv;
   if (2 * bh <= sm_count) return attn_default_splits(d, sm_count);
   long long sum = 0;
   int mx = 0;

@@ -48,8 +48,8 @@ def test_gqa_group_sizes(kvq_lib, gq):
 @pytest.mark.parametrize("gq", [1, 2, 3, 5, 6, 7])
 @pytest.mark.parametrize("n_splits", [3, 5, 19])
 def test_group_widths_with_odd_split_counts(kvq_lib, gq, n_splits):
-    # head groups of 1..4 query heads (5 = 4 + 1, 6 = 4 + 2, 7 = 4 + 3) and an
-    # odd number of splits: the final merge stages gq * S partial rows
+    # narrow (1..3) and wide (5..7) query groups with an odd number of
+    # splits: the final merge stages gq * S partial rows
     cfg = kvq.CacheConfig(batch=2, n_q_heads=2 * gq, n_kv_heads=2, bits_k=2, bits_v=1,
                           max_len=4096)
     errs, _ = _run(cfg, [4000, 1111], seed=60 + gq, n_splits=n_splits)

@@ -66,9 +66,9 @@ def test_steps_equal_pack_then_attention(kvq_lib, bk, bv):
 
 
 @pytest.mark.parametrize("gq", [5, 8])
-def test_wide_query_groups_two_head_groups(kvq_lib, gq):
-    # two head groups per kv-head: both read the pages, group 0 writes the
-    # ring row and the flushed page (lengths cross the flush at 160)
+def test_wide_query_groups(kvq_lib, gq):
+    # groups of 5..8 heads take the wide MMA layout; the lengths cross the
+    # flush at 160
     cfg = kvq.CacheConfig(batch=3, n_q_heads=2 * gq, n_kv_heads=2, bits_k=1, bits_v=2,
                           max_len=1024)
     pair, oracle = _steps(cfg, [158, 400, 159], 5, seed=21 + gq, check_oracle_every=5)
