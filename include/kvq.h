@@ -334,6 +334,17 @@ kvq_status dgap_restore(const dgap_params* params, float* logits,
                         size_t ws_bytes, void* stream);
 
 /*
+ * kvq_selftest_wait_timeout — checks on the device that a bounded wait gives
+ * up instead of hanging.  One warp waits, with a limit of ~10 ms, on an
+ * mbarrier armed for 16 bytes that no copy delivers (the loop the attention
+ * kernels use for their copy waits, whose limit is ~2 s); the wait runs out
+ * and the kernel sets KVQ_FLAG_WAIT_TIMEOUT in *flag and returns, leaving
+ * the context usable.
+ *   flag  device uint32, 4-byte aligned; the bit is OR-ed in.
+ */
+kvq_status kvq_selftest_wait_timeout(uint32_t* flag, void* stream);
+
+/*
  * Offline drift metrics (Sec. 4.1 "Adaptive recovery-window selection",
  * Sec. 4.2 "Offline supervision and calibration").  Tooling for paired
  * traces: each row holds one decode step's FP16-cache logits z_fp and

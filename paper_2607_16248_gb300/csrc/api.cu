@@ -400,6 +400,15 @@ kvq_status dgap_restore(const dgap_params* p, float* logits, int32_t batch, int3
                      "dgap_restore launch");
 }
 
+kvq_status kvq_selftest_wait_timeout(uint32_t* flag, void* stream) {
+  if (!flag) return fail(KVQ_ERR_ARG, "flag is NULL");
+  if ((reinterpret_cast<uintptr_t>(flag) & 3u) != 0) return fail(KVQ_ERR_ALIGN, "flag must be 4-byte aligned");
+  // about 10 ms at the SM clock: the copy waits' loop with a short limit
+  return cuda_status(launch_wait_selftest(reinterpret_cast<unsigned*>(flag), 20000000LL,
+                                          static_cast<cudaStream_t>(stream)),
+                     "kvq_selftest_wait_timeout launch");
+}
+
 int32_t kvq_drift_max_vocab(void) { return drift_max_vocab(); }
 
 kvq_status kvq_drift_metrics(const float* z_fp, const float* z_q, int32_t rows, int32_t vocab,

@@ -136,12 +136,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 // Wait for the phase with the given parity to complete; false after ~2 s.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity))
-    if (clock64() - t0 > kWaitCycles) return false;
+    if (clock64() - t0 > limit) return false;
   return true;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  return mbar_wait_for(bar, parity, kWaitCycles);
 }
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
   asm volatile(
@@ -1329,7 +1332,28 @@ struct LaunchOp {
   }
 };
 
+// Bounded-wait self-test: one warp arms an mbarrier for 16 bytes that no copy
+// delivers and waits on it with the given cycle limit, the same loop the
+// attention kernel's copy waits use.  The wait gives up, the kernel sets
+// KVQ_FLAG_WAIT_TIMEOUT in *flag and returns (no copy is in flight).
+__global__ void __launch_bounds__(32) wait_selftest_kernel(unsigned* flag, long long limit) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    mbar_expect_tx(&bar, 16u);  // the arrival; 16 bytes stay pending
+  }
+  __syncwarp();
+  const bool ok = __all_sync(0xffffffffu, mbar_wait_for(&bar, 0u, limit));
+  if (!ok && threadIdx.x == 0) atomicOr(flag, (unsigned)KVQ_FLAG_WAIT_TIMEOUT);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(unsigned* flag, long long limit_cycles, cudaStream_t st) {
+  wait_selftest_kernel<<<1, 32, 0, st>>>(flag, limit_cycles);
+  return cudaGetLastError();
+}
 
 // n_splits = CTAs per (sequence, kv-head); workspace rows for up to
 // n_splits.  Tickets: one per (sequence, kv-head), sized one per query head.

@@ -135,6 +135,7 @@ cudaError_t launch_decode_step(const Dims& d, const kvq_cache& cache, const __ha
                                cudaStream_t stream);
 size_t attn_workspace_bytes(const Dims& d, int n_splits);
 int attn_default_splits(const Dims& d, int sm_count);
+cudaError_t launch_wait_selftest(unsigned* flag, long long limit_cycles, cudaStream_t st);
 int attn_splits_for_lengths(const Dims& d, int sm_count, const int32_t* lengths);
 size_t attn_static_scratch_bytes();
 cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& cache, const __half* q,

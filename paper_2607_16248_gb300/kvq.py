@@ -29,6 +29,7 @@ EXPORTS = (
     "kvq_workspace_init",
     "kvq_decode_attn", "kvq_decode_step", "kvq_decode_attn_noalloc", "dgap_workspace_bytes",
     "dgap_restore", "kvq_drift_max_vocab", "kvq_drift_metrics", "kvq_drift_window",
+    "kvq_selftest_wait_timeout",
 )
 NOALLOC_SCRATCH_BYTES = 4 << 20
 
@@ -92,6 +93,7 @@ def lib():
             "dgap_workspace_bytes": (SZ, [I32, I32, par_p]),
             "dgap_restore": (I32, [par_p, P, I32, I32, P, P, P, P, P, P, P, SZ, P]),
             "kvq_drift_max_vocab": (I32, []),
+            "kvq_selftest_wait_timeout": (I32, [P, P]),
             "kvq_drift_metrics": (I32, [P, P, I32, I32, ctypes.POINTER(_DriftParams),
                                         P, P, P, P, P, P]),
             "kvq_drift_window": (I32, [P, I32, I32, F32, P, P, P]),
@@ -448,3 +450,11 @@ def drift_window(cov, rho_k, stream=None):
                                   _dev(mean, torch.float32, "mean_cov"),
                                   _dev(kb, torch.int32, "k_b"), _stream(stream)))
     return kb, mean
+
+
+def selftest_wait_timeout(stream=None):
+    """kvq_selftest_wait_timeout: the device flag word after a bounded wait on
+    a copy that never arrives ran out (KVQ_FLAG_WAIT_TIMEOUT expected)."""
+    flag = torch.zeros(1, dtype=torch.int32, device="cuda")
+    _check(lib().kvq_selftest_wait_timeout(_dev(flag, torch.int32, "flag"), _stream(stream)))
+    return flag
