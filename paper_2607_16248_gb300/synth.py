@@ -80,6 +80,20 @@ def dgap_weights(seed, K=32, hidden=256):
     }
 
 
+def save_weights(path, w):
+    """Write a weight dict (detector and corrector tensors) to an .npz file,
+    so a run's seeded parameters can be kept and reloaded."""
+    import numpy as np
+    np.savez(path, **{k: v.cpu().numpy() for k, v in w.items()})
+
+
+def load_weights(path):
+    """The weight dict written by save_weights (fp32 CPU tensors)."""
+    import numpy as np
+    with np.load(path) as f:
+        return {k: torch.from_numpy(f[k].copy()) for k in f.files}
+
+
 def split_weights(w):
     """(detector, corrector) dicts of float64 numpy arrays, w2 as [out][in]."""
     def a(t):

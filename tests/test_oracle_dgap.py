@@ -7,6 +7,7 @@ from math import log
 import numpy as np
 import pytest
 import scipy.stats
+import torch
 
 from oracle import dgap
 from paper_2607_16248_gb300 import synth
@@ -142,3 +143,17 @@ def test_next_token_is_argmax_of_merged_row():
         out = dgap.restore_row(z, 8, -1.0, det, cor)
         zt = out["z_tilde"]
         assert out["next_token"] == int(np.flatnonzero(zt == zt.max())[0])
+
+
+def test_weights_round_trip_through_npz(tmp_path):
+    w = synth.dgap_weights(7, K=8, hidden=32)
+    path = tmp_path / "dgap_weights.npz"
+    synth.save_weights(path, w)
+    back = synth.load_weights(path)
+    assert sorted(back) == sorted(w)
+    for k in w:
+        assert back[k].dtype == w[k].dtype and torch.equal(back[k], w[k])
+    z = synth.logits(3, 1, 500)[0].numpy().astype(np.float64)
+    a = dgap.restore_row(z, 8, -1.0, *synth.split_weights(w))
+    b = dgap.restore_row(z, 8, -1.0, *synth.split_weights(back))
+    assert np.array_equal(a["val"], b["val"]) and a["r"] == b["r"]
