@@ -413,14 +413,17 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
         a1[2 * half] = v[2];
         a1[2 * half + 1] = v[3];
         const uint32_t s2 = half ? sw.y : sw.x;
-        const __half2 hi = __hmul2(u2h(qb[2 * ks + half]), u2h(s2));
         if constexpr (kWide) {
           // q*s as its fp16 high part and exact residual, two operands
+          const __half2 hi = __hmul2(u2h(qb[2 * ks + half]), u2h(s2));
           b[half] = h2u(hi);
           bl[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hneg2(hi)));
         } else {
-          // q*s as fp16 high part (columns 0..3) or its exact residual (4..7)
-          b[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hmul2(hi, u2h(ln.neg_lo))));
+          // q*s as fp16 high part (columns 0..3) or its exact residual (4..7):
+          // qn = -q on the lanes of columns 4..7 and 0 elsewhere (the same
+          // for every block), RN16(qn s) = -RN16(q s) there
+          const __half2 qn = __hmul2(u2h(qb[2 * ks + half]), u2h(ln.neg_lo));
+          b[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hmul2(qn, u2h(s2))));
         }
       }
       mma16816(dk[bi][0], a0[0], a0[1], a0[2], a0[3], b[0], b[1]);
@@ -477,7 +480,10 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
     // costs no accuracy.  Narrow: columns 0..3 / 4..7, lanes of columns 4..7
     // hold p_lo after movmatrix and fetch p_hi from lane - 16; wide: every
     // lane has both parts of its head.
-    uint32_t pa[2][2], pb[2][2];
+    // Narrow: pn = -p_hi on lanes of columns 4..7 and 0 elsewhere, so
+    // RN16(pn s) is -RN16(p_hi s) there (rounding is symmetric) and the
+    // residual fma needs no separate product.
+    uint32_t pa[2][2], pb[2][2], pn[2][2];
 #pragma unroll
     for (int ks = 0; ks < 2; ++ks)
 #pragma unroll
@@ -489,6 +495,7 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
           const uint32_t other = __shfl_xor_sync(0xffffffffu, pt[bi][ks][dl], 16);
           pa[ks][dl] = lane < 16 ? pt[bi][ks][dl] : other;
           pb[ks][dl] = lane < 16 ? 0u : pt[bi][ks][dl];
+          pn[ks][dl] = h2u(__hmul2(u2h(pa[ks][dl]), u2h(ln.neg_lo)));
         }
       }
     uint4 vw1;
@@ -517,13 +524,14 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
           am1[2 * dl] = v[2];
           am1[2 * dl + 1] = v[3];
           const __half2 sc = u2h(mw[ia]);
-          const __half2 t = __hmul2(u2h(pa[ks][dl]), sc);
           if constexpr (kWide) {
+            const __half2 t = __hmul2(u2h(pa[ks][dl]), sc);
             const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hneg2(t));
             bv[dl] = h2u(t);
             bw[dl] = h2u(__hfma2(u2h(pb[ks][dl]), sc, err));
           } else {
-            const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hmul2(t, u2h(ln.neg_lo)));
+            // columns 0..3: RN16(p_hi s); 4..7: RN16(p_lo s + exact residual)
+            const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hmul2(u2h(pn[ks][dl]), sc));
             bv[dl] = h2u(__hfma2(u2h(pb[ks][dl]), sc, err));
           }
         }
