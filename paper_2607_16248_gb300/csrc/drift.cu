@@ -70,6 +70,7 @@ struct Sm {
   uint32_t rc[kBins / kCl];
   u64 rm[kBins / kCl];
   u64 xin[kCl][kXw];                // values loaded from the eight CTAs
+  u64 xin8[kCl][2 * kXw];           // the same for a two-slot exchange
   u64 wsel[kMaxKcov];               // coverage terms of the TopK list
   float bc[4];                      // broadcast scalars
   uint32_t ru[kW];
@@ -274,6 +275,23 @@ __device__ void cluster_gather(Sm& s, int slot, u64 a, u64 b, u64 c = 0ull, u64 
   if (threadIdx.x < kXw * kCl)
     s.xin[threadIdx.x / kXw][threadIdx.x % kXw] =
         ld_peer_u64(peer_addr(&s.xd[slot][threadIdx.x % kXw], threadIdx.x / kXw));
+  __syncthreads();
+}
+// Six words in slots `slot` and `slot + 1`, one barrier; s.xin8[rank][word].
+__device__ void cluster_gather2x(Sm& s, int slot, u64 a, u64 b, u64 c, u64 d, u64 e, u64 f) {
+  if (threadIdx.x == 0) {
+    s.xd[slot][0] = a;
+    s.xd[slot][1] = b;
+    s.xd[slot][2] = c;
+    s.xd[slot][3] = d;
+    s.xd[slot + 1][0] = e;
+    s.xd[slot + 1][1] = f;
+  }
+  cluster_sync();
+  if (threadIdx.x < 2 * kXw * kCl) {
+    const int r = threadIdx.x / (2 * kXw), w = threadIdx.x % (2 * kXw);
+    s.xin8[r][w] = ld_peer_u64(peer_addr(&s.xd[slot + w / kXw][w % kXw], (uint32_t)r));
+  }
   __syncthreads();
 }
 __device__ __forceinline__ void cluster_gather2(Sm& s, int slot, u64 a, u64 b) {
@@ -504,6 +522,41 @@ __device__ uint32_t nth_tie(Sm& s, const Ctx& cx, const float* a, uint32_t key, 
   return ans_s;
 }
 
+// The elements i of this CTA's slice with hit(i), as packed (key(i), index)
+// words, appended to rank 0's buf: compacted in this CTA's histogram area
+// (free once a selection's bin is known), then one remote reservation on
+// rank 0's fill count and parallel remote stores.  Rank 0's nbuf must be
+// zero, and visible through a cluster barrier, before the call.
+template <typename Hit, typename Key>
+__device__ void gather_to_rank0(Sm& s, const Ctx& cx, const Hit& hit, const Key& key) {
+  __shared__ uint32_t lcount, lbase;
+  u64* loc = reinterpret_cast<u64*>(&s.hm[0][0]);  // 3 * kBins u32 >= kCap u64
+  if (threadIdx.x == 0) lcount = 0u;
+  __syncthreads();
+  const int l = threadIdx.x & 31;
+  for (int t0 = 0; t0 < cx.n; t0 += kT) {
+    const int i = t0 + threadIdx.x;
+    const bool h = i < cx.n && hit(i);
+    const uint32_t bal = __ballot_sync(0xffffffffu, h);
+    if (bal == 0u) continue;
+    uint32_t base = 0u;
+    if (l == 0) base = atomicAdd(&lcount, (uint32_t)__popc(bal));
+    base = __shfl_sync(0xffffffffu, base, 0);
+    if (h) {
+      const uint32_t pos = base + __popc(bal & ((1u << l) - 1u));
+      if (pos < (uint32_t)kCap) loc[pos] = pack(key(i), cx.i0 + (uint32_t)i);
+    }
+  }
+  __syncthreads();
+  const uint32_t n = min(lcount, (uint32_t)kCap);
+  if (threadIdx.x == 0) lbase = n ? atom_add_peer(peer_addr(&s.nbuf, 0), n) : 0u;
+  __syncthreads();
+  for (uint32_t j = threadIdx.x; j < n; j += kT) {
+    const uint32_t pos = lbase + j;
+    if (pos < (uint32_t)kCap) st_peer_u64(peer_addr(&s.buf[pos], 0), loc[j]);
+  }
+}
+
 __device__ void clear_hist(Sm& s) {
   for (int i = threadIdx.x; i < kBins; i += kT) {
     s.hc[i] = 0u;
@@ -651,22 +704,7 @@ __device__ Pick select(Sm& s, const Ctx& cx, const float* a, float m, bool weigh
   // ---- gather the set into rank 0, sort, scan ----
   if (cx.rank == 0 && threadIdx.x == 0) s.nbuf = 0u;
   cluster_sync();
-  const uint32_t nb0 = peer_addr(&s.nbuf, 0);
-  for (int t0 = 0; t0 < cx.n; t0 += kT) {
-    const int i = t0 + threadIdx.x;
-    const bool hit = i < cx.n && in_set(a[i]);
-    const uint32_t bal = __ballot_sync(0xffffffffu, hit);
-    if (bal == 0u) continue;
-    const int l = threadIdx.x & 31;
-    uint32_t base = 0u;
-    if (l == 0) base = atom_add_peer(nb0, __popc(bal));
-    base = __shfl_sync(0xffffffffu, base, 0);
-    if (hit) {
-      const uint32_t pos = base + __popc(bal & ((1u << l) - 1u));
-      if (pos < (uint32_t)kCap)
-        st_peer_u64(peer_addr(&s.buf[pos], 0), pack(fkey(a[i]), cx.i0 + (uint32_t)i));
-    }
-  }
+  gather_to_rank0(s, cx, [&](int i) { return in_set(a[i]); }, [&](int i) { return fkey(a[i]); });
   cluster_sync();
   if (cx.rank == 0) {
     const int n = (int)min(s.nbuf, (uint32_t)kCap);
@@ -774,24 +812,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kT, 1)
   // ---- the k_max best of z_q, sorted, in rank 0 ----
   if (cx.rank == 0 && threadIdx.x == 0) s.nbuf = 0u;
   cluster_sync();
-  {
-    const uint32_t nb0 = peer_addr(&s.nbuf, 0);
-    for (int t0 = 0; t0 < cx.n; t0 += kT) {
-      const int i = t0 + threadIdx.x;
-      const bool hit = i < cx.n && ranks_in(fkey(s.zq[i]), cx.i0 + (uint32_t)i, pq);
-      const uint32_t bal = __ballot_sync(0xffffffffu, hit);
-      if (bal == 0u) continue;
-      const int l = threadIdx.x & 31;
-      uint32_t base = 0u;
-      if (l == 0) base = atom_add_peer(nb0, __popc(bal));
-      base = __shfl_sync(0xffffffffu, base, 0);
-      if (hit) {
-        const uint32_t pos = base + __popc(bal & ((1u << l) - 1u));
-        if (pos < (uint32_t)kCap)
-          st_peer_u64(peer_addr(&s.buf[pos], 0), pack(fkey(s.zq[i]), cx.i0 + (uint32_t)i));
-      }
-    }
-  }
+  gather_to_rank0(
+      s, cx, [&](int i) { return ranks_in(fkey(s.zq[i]), cx.i0 + (uint32_t)i, pq); },
+      [&](int i) { return fkey(s.zq[i]); });
   cluster_sync();
   if (cx.rank == 0) {
     sort_desc(s, (int)min(s.nbuf, (uint32_t)kCap));
@@ -815,48 +838,114 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kT, 1)
   // masses A = e_fp(U), B = e_q(U), c = e_fp(C and S) in fixed point; the
   // sums of e_fp^2, e_fp e_q, e_q^2 in double-float for
   //   d_loc^2 = Saa / A^2 - 2 Sab / (A B) + Sbb / B^2.
+  // U is sparse: each warp queues its members (local index, bit 31 = in C
+  // and S) in its own 64 entries of buf past the TopK list and works on them
+  // 32 at a time, so the exponentials and products run on full warps.
   u64 A = 0ull, B = 0ull, Cs = 0ull;
   Df saa, sab, sbb;
-  for (int i = threadIdx.x; i < cx.n; i += kT) {
-    const uint32_t gi = cx.i0 + (uint32_t)i;
-    const bool inc = ranks_in(fkey(s.zf[i]), gi, pf);
-    const bool ins = ranks_in(fkey(s.zq[i]), gi, ps);
-    if (inc || ins) {
+  {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint32_t* uq = reinterpret_cast<uint32_t*>(&s.buf[kMaxKcov]) + warp * 64;
+    auto member = [&](uint32_t e) {
+      const int i = (int)(e & 0x7fffffffu);
       const float a = expf(s.zf[i] - mf), b = expf(s.zq[i] - mq);
       const u64 qa = fix40(a);
       A += qa;
       B += fix40(b);
-      if (inc && ins) Cs += qa;
+      if (e >> 31) Cs += qa;
       saa.add_prod(a, a);
       sab.add_prod(a, b);
       sbb.add_prod(b, b);
+    };
+    int qn = 0;
+    for (int t0 = warp * 32; t0 < cx.n; t0 += kT) {
+      const int i = t0 + lane;
+      bool inc = false, ins = false;
+      if (i < cx.n) {
+        const uint32_t gi = cx.i0 + (uint32_t)i;
+        inc = ranks_in(fkey(s.zf[i]), gi, pf);
+        ins = ranks_in(fkey(s.zq[i]), gi, ps);
+      }
+      const bool mem = inc || ins;
+      const uint32_t bal = __ballot_sync(0xffffffffu, mem);
+      if (mem) uq[qn + __popc(bal & ((1u << lane) - 1u))] = (uint32_t)i | (inc && ins ? 0x80000000u : 0u);
+      qn += __popc(bal);
+      __syncwarp();
+      if (qn >= 32) {
+        member(uq[lane]);
+        __syncwarp();
+        if (lane < qn - 32) uq[lane] = uq[32 + lane];  // the rest (< 32) to the front
+        qn -= 32;
+        __syncwarp();
+      }
     }
+    if (lane < qn) member(uq[lane]);
   }
-  A = block_sum_q(A, s);
-  B = block_sum_q(B, s);
-  Cs = block_sum_q(Cs, s);
-  saa = block_sum_df(saa, s);
-  sab = block_sum_df(sab, s);
-  sbb = block_sum_df(sbb, s);
-  cluster_gather(s, slot++, A, B, Cs);
+  // per-warp sums (a fixed pairing order), then thread 0 adds the warps
+  {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      A += __shfl_xor_sync(0xffffffffu, A, o);
+      B += __shfl_xor_sync(0xffffffffu, B, o);
+      Cs += __shfl_xor_sync(0xffffffffu, Cs, o);
+      Df* acc[3] = {&saa, &sab, &sbb};
+#pragma unroll
+      for (int k = 0; k < 3; ++k) {
+        Df w;
+        w.hi = __shfl_xor_sync(0xffffffffu, acc[k]->hi, o);
+        w.lo = __shfl_xor_sync(0xffffffffu, acc[k]->lo, o);
+        if ((threadIdx.x & o) == 0) {
+          acc[k]->add(w);
+        } else {
+          w.add(*acc[k]);
+          *acc[k] = w;
+        }
+      }
+    }
+    u64* wpart = reinterpret_cast<u64*>(s.wsel);  // [kW][6] (wsel is free until the outputs)
+    if ((threadIdx.x & 31) == 0) {
+      u64* w = wpart + (threadIdx.x >> 5) * 6;
+      w[0] = A;
+      w[1] = B;
+      w[2] = Cs;
+      w[3] = saa.pack();
+      w[4] = sab.pack();
+      w[5] = sbb.pack();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      A = B = Cs = 0ull;
+      Df ta, tb, tc;
+      for (int w = 0; w < kW; ++w) {
+        A += wpart[w * 6];
+        B += wpart[w * 6 + 1];
+        Cs += wpart[w * 6 + 2];
+        ta.add(Df::unpack(wpart[w * 6 + 3]));
+        tb.add(Df::unpack(wpart[w * 6 + 4]));
+        tc.add(Df::unpack(wpart[w * 6 + 5]));
+      }
+      saa = ta;
+      sab = tb;
+      sbb = tc;
+    }
+    __syncthreads();
+  }
+  // one exchange of the six CTA totals (thread 0's values are published)
+  cluster_gather2x(s, slot, A, B, Cs, saa.pack(), sab.pack(), sbb.pack());
+  slot += 2;
   u64 c_sum = 0ull;
-  A = B = 0ull;
-  for (int r = 0; r < kCl; ++r) {
-    A += s.xin[r][0];
-    B += s.xin[r][1];
-    c_sum += s.xin[r][2];
-  }
-  __syncthreads();
-  cluster_gather(s, slot++, saa.pack(), sab.pack(), sbb.pack());
-  Df taa, tab, tbb;
-  for (int r = 0; r < kCl; ++r) {
-    taa.add(Df::unpack(s.xin[r][0]));
-    tab.add(Df::unpack(s.xin[r][1]));
-    tbb.add(Df::unpack(s.xin[r][2]));
-  }
-  __syncthreads();
   double Dsum = 0.0;
   if (threadIdx.x == 0) {
+    A = B = 0ull;
+    Df taa, tab, tbb;
+    for (int r = 0; r < kCl; ++r) {
+      A += s.xin8[r][0];
+      B += s.xin8[r][1];
+      c_sum += s.xin8[r][2];
+      taa.add(Df::unpack(s.xin8[r][3]));
+      tab.add(Df::unpack(s.xin8[r][4]));
+      tbb.add(Df::unpack(s.xin8[r][5]));
+    }
     const double ia = kFix / (double)A, ib = kFix / (double)B;
     Dsum = taa.value() * ia * ia - 2.0 * tab.value() * ia * ib + tbb.value() * ib * ib;
     if (Dsum < 0.0) Dsum = 0.0;  // rounding of an exact zero
