@@ -758,6 +758,8 @@ __host__ __device__ constexpr int warp_ring_bytes(int page) {
           127) / 128 * 128;
 }
 static_assert(kWarps * warp_ring_bytes(page_bytes_c(4, 8)) <= kRingBudget + 8 * 1024, "rings fit");
+// Shared-memory page image of a block that leaves the window (decode step).
+__host__ __device__ constexpr int image_bytes(int page) { return (page + 127) / 128 * 128; }
 
 // Packed warps stream their blocks through a private ring of slots.  A page
 // is written once, when its group leaves the window, and never changes
@@ -795,16 +797,24 @@ __device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int 
   return n;
 }
 
+__device__ __forceinline__ bool stage_rows_bulk(__half* rows, const __half* ring_base, int p0,
+                                                int n_tok, int ring, int p_new,
+                                                const __half* new_row, uint64_t* bar,
+                                                uint32_t parity);
+
 // Decode step with a flush: the 32-token block of positions [p0, p0 + 32),
 // still fp16 in the ring, leaves the window.  One warp quantizes it exactly as
 // kvq_pack does (same quantizer, same page layout) into a page image in
-// `image` (shared memory) and, if `page_out` is set, writes the page there;
-// the caller folds
-// the image into its state like any streamed block.  Kept out of line: it is
-// rare and its registers would otherwise crowd the streaming loop.
+// `image` (shared memory) and writes the page to `page_out`; the caller folds
+// the image into its state like any streamed block.  The block's K rows, then
+// its V rows, are staged in `rows` (the warp's idle ring) by one bulk copy per
+// row on `bar` (phases 0 and 1).  Returns false if a bounded wait gave up.
+// Kept out of line: it is rare and its registers would otherwise crowd the
+// streaming loop.
 template <int BK, int BV>
-__device__ __noinline__ void flush_block(const __half* ring_k, const __half* ring_v, int p0,
-                                         int ring, char* image, char* page_out) {
+__device__ __noinline__ bool flush_block(const __half* ring_k, const __half* ring_v, int p0,
+                                         int ring, __half* rows, uint64_t* bar, char* image,
+                                         char* page_out) {
   constexpr int page = page_bytes_c(BK, BV);
   const int lane = threadIdx.x & 31;
   uint32_t* kcodes = reinterpret_cast<uint32_t*>(image);
@@ -815,14 +825,13 @@ __device__ __noinline__ void flush_block(const __half* ring_k, const __half* rin
     for (int i = lane; i < kHeadDim; i += 32) kcodes[i] = 0u;
   if (BV == 1)
     for (int i = lane; i < kHeadDim; i += 32) vcodes[i] = 0u;
-  __syncwarp();
+  if (!stage_rows_bulk(rows, ring_k, p0, kGroup, ring, -1, nullptr, bar, 0u)) return false;
   // keys: lane l quantizes channels 4l .. 4l+3 over the block's 32 tokens
   for (int cc = 0; cc < 4; ++cc) {
     const int c = 4 * lane + cc;
     float x[kGroup];
 #pragma unroll
-    for (int t = 0; t < kGroup; ++t)
-      x[t] = __half2float(ring_k[(long long)((p0 + t) % ring) * kHeadDim + c]);
+    for (int t = 0; t < kGroup; ++t) x[t] = __half2float(rows[t * kResRow + c]);
     uint32_t w[BK];
     __half sc, z;
     quantize_group<BK>(x, w, sc, z);
@@ -839,14 +848,25 @@ __device__ __noinline__ void flush_block(const __half* ring_k, const __half* rin
     kmeta[c] = sc;
     kmeta[kHeadDim + c] = z;
   }
+  __syncwarp();
+  if (!stage_rows_bulk(rows, ring_v, p0, kGroup, ring, -1, nullptr, bar, 1u)) return false;
   // values: lane t quantizes the four 32-channel groups of token t
   {
     const int t = lane;
-    const __half* row = ring_v + (long long)((p0 + t) % ring) * kHeadDim;
+    const uint4* row = reinterpret_cast<const uint4*>(rows + t * kResRow);
     for (int g = 0; g < 4; ++g) {
       float x[kGroup];
 #pragma unroll
-      for (int i = 0; i < kGroup; ++i) x[i] = __half2float(row[g * kGroup + i]);
+      for (int k = 0; k < 4; ++k) {
+        const uint4 u = row[4 * g + k];
+        const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __half22float2(u2h(wd[e]));
+          x[8 * k + 2 * e] = f.x;
+          x[8 * k + 2 * e + 1] = f.y;
+        }
+      }
       uint32_t w[BV];
       __half sc, z;
       quantize_group<BV>(x, w, sc, z);
@@ -865,10 +885,10 @@ __device__ __noinline__ void flush_block(const __half* ring_k, const __half* rin
     }
   }
   __syncwarp();
-  if (page_out)
-    for (int i = lane; i < page / 16; i += 32)
-      reinterpret_cast<uint4*>(page_out)[i] = reinterpret_cast<const uint4*>(image)[i];
+  for (int i = lane; i < page / 16; i += 32)
+    reinterpret_cast<uint4*>(page_out)[i] = reinterpret_cast<const uint4*>(image)[i];
   __syncwarp();
+  return true;
 }
 
 // Fold blocks [lo, hi) into st; `pre` slots holding blocks [lo_h, pre_end)
@@ -878,7 +898,8 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
                                char* ring, uint64_t* full, int R, const char* zero,
                                const __half* qh, int gq, float scale_log2, unsigned* flag,
                                TcState& st, int flush_blk, const __half* ring_k,
-                               const __half* ring_v, int ring_size) {
+                               const __half* ring_v, int ring_size, uint64_t* fbar,
+                               char* image) {
   constexpr int page = page_bytes_c(BK, BV);
   constexpr int NB = ring_blocks(page);
   const int lane = threadIdx.x & 31;
@@ -939,10 +960,14 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
     for (int s = max(consumed, issued - R); s < issued; ++s) mbar_wait(full + s % R, (s / R) & 1);
   __syncwarp();
   if (flush) {
-    flush_block<BK, BV>(ring_k, ring_v, flush_blk * kGroup, ring_size, ring,
-                        const_cast<char*>(pages_bh) + (long long)flush_blk * page);
-    const char* pg[1] = {ring};
-    tc_unit<BK, BV, 1, kWide>(pg, zero, qb, ln, scale_log2, st);
+    if (flush_block<BK, BV>(ring_k, ring_v, flush_blk * kGroup, ring_size,
+                            reinterpret_cast<__half*>(ring), fbar, image,
+                            const_cast<char*>(pages_bh) + (long long)flush_blk * page)) {
+      const char* pg[1] = {image};
+      tc_unit<BK, BV, 1, kWide>(pg, zero, qb, ln, scale_log2, st);
+    } else if (lane == 0) {
+      atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
+    }
   }
 }
 
@@ -1088,6 +1113,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       block_range(ph, v, lo_h, hi_h);
       // the newest block may be the one the previous kernel is writing
       pre = tc_pre_issue<BK, BV>(pages, lo_h, hi_h, ph.nb - 1, ring, full, R, pre_end);
+      // a decode step that pushes a group out of the window: its owner brings
+      // the group's ring rows (old, unchanging) into L2 for the flush
+      if (append && lane == 0 && hi_h == ph.nb && ph.nb > 0 &&
+          ph.Lq > packed_len(hint - 1, d.residual)) {
+        prefetch_rows_l2(ring_k, ph.Lq - kGroup, kGroup, d.ring);
+        prefetch_rows_l2(ring_v, ph.Lq - kGroup, kGroup, d.ring);
+      }
     } else if (lane == 0) {
       // window rows of the length read before the wait into L2 (rows below
       // the newest token do not change; this is a hint, nothing waits on it)
@@ -1148,7 +1180,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       }
       tc_packed_warp<BK, BV, kWide>(pages, lo_h, pre, pre_end, lo, hi, ring, full, R,
                              reinterpret_cast<const char*>(zero), q_s, gq, scale_log2, flag, st,
-                             flush_blk, ring_k, ring_v, d.ring);
+                             flush_blk, ring_k, ring_v, d.ring, &wbar[warp],
+                             reinterpret_cast<char*>(smem + smem_size - 16 - kZeroBytes -
+                                                     image_bytes(page)));
     }
     if (!packed)
       tc_window_warp<BK, BV, kWide>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, q_s, gq,
@@ -1273,8 +1307,9 @@ size_t smem_bytes(const Dims& d) {
   const int page = (int)d.page_bytes;
   const size_t rings = (size_t)kWarps * warp_ring_bytes(page) +
                        (size_t)kWarps * ring_slots(page) * sizeof(uint64_t);
-  // + the zero rows of the packed warps and the final merge's mbarrier
-  return (rings + kZeroBytes + 16 + 127) / 128 * 128;
+  // + a flushed block's page image, the zero rows of the packed warps and
+  // the final merge's mbarrier
+  return (rings + image_bytes(page) + kZeroBytes + 16 + 127) / 128 * 128;
 }
 
 template <int BK, int BV, bool kWide>
