@@ -797,98 +797,108 @@ __device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int 
   return n;
 }
 
-__device__ __forceinline__ bool stage_rows_bulk(__half* rows, const __half* ring_base, int p0,
-                                                int n_tok, int ring, int p_new,
-                                                const __half* new_row, uint64_t* bar,
-                                                uint32_t parity);
-
 // Decode step with a flush: the 32-token block of positions [p0, p0 + 32),
-// still fp16 in the ring, leaves the window.  One warp quantizes it exactly as
+// still fp16 in the ring, leaves the window and is quantized exactly as
 // kvq_pack does (same quantizer, same page layout) into a page image in
-// `image` (shared memory) and writes the page to `page_out`; the caller folds
-// the image into its state like any streamed block.  The block's K rows, then
-// its V rows, are staged in `rows` (the warp's idle ring) by one bulk copy per
-// row on `bar` (phases 0 and 1).  Returns false if a bounded wait gave up.
-// Kept out of line: it is rare and its registers would otherwise crowd the
-// streaming loop.
+// shared memory.  The work comes in four quarters: quarter qi is the key
+// groups of channels 32 qi .. 32 qi + 31 (lane = channel) and value group qi
+// of the 32 tokens (lane = token).  The quarters write disjoint words of the
+// image (1-bit codes: words 4 l + qi, l = 0..31), so different warps can
+// take them.  Rows are read straight from global memory (L2); nothing in
+// this kernel writes them.  Kept out of line: it is rare and its registers
+// would otherwise crowd the streaming loop.
 template <int BK, int BV>
-__device__ __noinline__ bool flush_block(const __half* ring_k, const __half* ring_v, int p0,
-                                         int ring, __half* rows, uint64_t* bar, char* image,
-                                         char* page_out) {
-  constexpr int page = page_bytes_c(BK, BV);
+__device__ __noinline__ void flush_quarter(const __half* ring_k, const __half* ring_v, int p0,
+                                           int ring, int qi, char* image) {
   const int lane = threadIdx.x & 31;
   uint32_t* kcodes = reinterpret_cast<uint32_t*>(image);
   uint32_t* vcodes = reinterpret_cast<uint32_t*>(image + page_off_vcodes(BK));
   __half* kmeta = reinterpret_cast<__half*>(image + page_off_kmeta(BK));
   __half* vmeta = reinterpret_cast<__half*>(image + page_off_vmeta(BK, BV));
-  if (BK == 1)
-    for (int i = lane; i < kHeadDim; i += 32) kcodes[i] = 0u;
-  if (BV == 1)
-    for (int i = lane; i < kHeadDim; i += 32) vcodes[i] = 0u;
-  if (!stage_rows_bulk(rows, ring_k, p0, kGroup, ring, -1, nullptr, bar, 0u)) return false;
-  // keys: lane l quantizes channels 4l .. 4l+3 over the block's 32 tokens
-  for (int cc = 0; cc < 4; ++cc) {
-    const int c = 4 * lane + cc;
-    float x[kGroup];
+  const int s0 = p0 % ring;
+  const int c = kGroup * qi + lane;  // this lane's key channel
+  float xk[kGroup], xv[kGroup];
 #pragma unroll
-    for (int t = 0; t < kGroup; ++t) x[t] = __half2float(rows[t * kResRow + c]);
-    uint32_t w[BK];
-    __half sc, z;
-    quantize_group<BK>(x, w, sc, z);
-    if (BK == 1) {
-#pragma unroll 4
-      for (int t = 0; t < kGroup; ++t) {
-        const int bit = key1_bit(t, c);
-        if ((w[0] >> t) & 1u) atomicOr(&kcodes[bit >> 5], 1u << (bit & 31));
-      }
-    } else {
-#pragma unroll
-      for (int j = 0; j < BK; ++j) kcodes[c * BK + j] = w[j];
-    }
-    kmeta[c] = sc;
-    kmeta[kHeadDim + c] = z;
+  for (int t = 0; t < kGroup; ++t) {
+    const int s = s0 + t < ring ? s0 + t : s0 + t - ring;
+    xk[t] = __half2float(ring_k[(long long)s * kHeadDim + c]);
   }
-  __syncwarp();
-  if (!stage_rows_bulk(rows, ring_v, p0, kGroup, ring, -1, nullptr, bar, 1u)) return false;
-  // values: lane t quantizes the four 32-channel groups of token t
   {
-    const int t = lane;
-    const uint4* row = reinterpret_cast<const uint4*>(rows + t * kResRow);
-    for (int g = 0; g < 4; ++g) {
-      float x[kGroup];
+    const int s = s0 + lane < ring ? s0 + lane : s0 + lane - ring;
+    const uint4* row = reinterpret_cast<const uint4*>(ring_v + (long long)s * kHeadDim + kGroup * qi);
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const uint4 u = row[4 * g + k];
-        const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
+    for (int k = 0; k < 4; ++k) {
+      const uint4 u = row[k];
+      const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 f = __half22float2(u2h(wd[e]));
-          x[8 * k + 2 * e] = f.x;
-          x[8 * k + 2 * e + 1] = f.y;
-        }
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __half22float2(u2h(wd[e]));
+        xv[8 * k + 2 * e] = f.x;
+        xv[8 * k + 2 * e + 1] = f.y;
       }
-      uint32_t w[BV];
-      __half sc, z;
-      quantize_group<BV>(x, w, sc, z);
-      if (BV == 1) {
-#pragma unroll 4
-        for (int i = 0; i < kGroup; ++i) {
-          const int bit = val1_bit(t, g * kGroup + i);
-          if ((w[0] >> i) & 1u) atomicOr(&vcodes[bit >> 5], 1u << (bit & 31));
-        }
-      } else {
-#pragma unroll
-        for (int j = 0; j < BV; ++j) vcodes[(g * kGroup + t) * BV + j] = w[j];
-      }
-      vmeta[vmeta_index(g, t)] = sc;
-      vmeta[kHeadDim + vmeta_index(g, t)] = z;
     }
   }
-  __syncwarp();
-  for (int i = lane; i < page / 16; i += 32)
-    reinterpret_cast<uint4*>(page_out)[i] = reinterpret_cast<const uint4*>(image)[i];
-  __syncwarp();
-  return true;
+  uint32_t wk[BK], wv[BV];
+  __half sk, zk, sv, zv;
+  quantize_group<BK>(xk, wk, sk, zk);
+  quantize_group<BV>(xv, wv, sv, zv);
+  kmeta[c] = sk;
+  kmeta[kHeadDim + c] = zk;
+  vmeta[vmeta_index(qi, lane)] = sv;
+  vmeta[kHeadDim + vmeta_index(qi, lane)] = zv;
+  // 1-bit codes: lane l = 4 gid + tig assembles word 4 l + qi from ballots
+  // (bit positions of key1_bit / val1_bit)
+  const int gid = lane >> 2, tig = lane & 3;
+  if constexpr (BK == 1) {
+    uint32_t mine[4] = {0u, 0u, 0u, 0u};  // ballots of tokens 4 gid + j over channels
+#pragma unroll
+    for (int t = 0; t < kGroup; ++t) {
+      const uint32_t bt = __ballot_sync(0xffffffffu, (wk[0] >> t) & 1u);
+      if ((t >> 2) == gid) mine[t & 3] = bt;
+    }
+    uint32_t word = 0u;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t m = mine[j] >> (4 * tig);
+#pragma unroll
+      for (int ks1 = 0; ks1 < 2; ++ks1)
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int e = 0; e < 2; ++e)
+            word |= ((m >> (16 * ks1 + 2 * h + e)) & 1u) << ((10 + 16 * e + j - 4 * (2 * ks1 + h)) & 31);
+    }
+    kcodes[4 * lane + qi] = word;
+  } else {
+#pragma unroll
+    for (int j = 0; j < BK; ++j) kcodes[c * BK + j] = wk[j];
+  }
+  if constexpr (BV == 1) {
+    uint32_t mine[4] = {0u, 0u, 0u, 0u};  // ballots of channels 4 gid + j over tokens
+#pragma unroll
+    for (int ci = 0; ci < kGroup; ++ci) {
+      const uint32_t bc = __ballot_sync(0xffffffffu, (wv[0] >> ci) & 1u);
+      if ((ci >> 2) == gid) mine[ci & 3] = bc;
+    }
+    uint32_t word = 0u;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t m = mine[j] >> (8 * tig);
+#pragma unroll
+      for (int e = 0; e < 2; ++e)
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          word |= ((m >> (4 * e + r)) & 1u) << ((10 + 16 * e + j - 4 * r) & 31);
+    }
+    vcodes[4 * lane + qi] = word;
+  } else {
+#pragma unroll
+    for (int j = 0; j < BV; ++j) vcodes[(qi * kGroup + lane) * BV + j] = wv[j];
+  }
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 
 // Fold blocks [lo, hi) into st; `pre` slots holding blocks [lo_h, pre_end)
@@ -897,9 +907,8 @@ template <int BK, int BV, bool kWide>
 __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_end, int lo, int hi_all,
                                char* ring, uint64_t* full, int R, const char* zero,
                                const __half* qh, int gq, float scale_log2, unsigned* flag,
-                               TcState& st, int flush_blk, const __half* ring_k,
-                               const __half* ring_v, int ring_size, uint64_t* fbar,
-                               char* image) {
+                               TcState& st, int flush_blk,
+                               uint64_t* fl_bar, char* image) {
   constexpr int page = page_bytes_c(BK, BV);
   constexpr int NB = ring_blocks(page);
   const int lane = threadIdx.x & 31;
@@ -960,9 +969,11 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
     for (int s = max(consumed, issued - R); s < issued; ++s) mbar_wait(full + s % R, (s / R) & 1);
   __syncwarp();
   if (flush) {
-    if (flush_block<BK, BV>(ring_k, ring_v, flush_blk * kGroup, ring_size,
-                            reinterpret_cast<__half*>(ring), fbar, image,
-                            const_cast<char*>(pages_bh) + (long long)flush_blk * page)) {
+    // the page image is complete once its four quarters have arrived
+    if (__all_sync(0xffffffffu, mbar_wait(fl_bar, 0u))) {
+      uint4* dst =
+          reinterpret_cast<uint4*>(const_cast<char*>(pages_bh) + (long long)flush_blk * page);
+      for (int i = lane; i < page / 16; i += 32) dst[i] = reinterpret_cast<const uint4*>(image)[i];
       const char* pg[1] = {image};
       tc_unit<BK, BV, 1, kWide>(pg, zero, qb, ln, scale_log2, st);
     } else if (lane == 0) {
@@ -1067,6 +1078,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   __shared__ int len_s[2];  // length attended, length before the append
   __shared__ __align__(16) __half q_s[kHeads * kHeadDim];  // the CTA's query heads
   __shared__ __align__(8) uint64_t wbar[kWarps];      // a window warp's staging barrier
+  __shared__ __align__(8) uint64_t fl_bar;            // page image of a flush complete
 
   const int h = blockIdx.y, b = blockIdx.z;
   const int gq = d.gq;
@@ -1101,6 +1113,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     if (lane == 0) {
       for (int i = 0; i < R; ++i) mbar_init(full + i, 1);
       mbar_init(&wbar[warp], 1);
+      if (warp == 0) mbar_init(&fl_bar, 4 * 32);
       fence_mbar_init();
       hint = read_len(c.seq_len + b);
     }
@@ -1169,6 +1182,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     const Plan p = same ? ph : make_plan(L, d.residual, NV);
     const int flush_blk = grew && p.Lq > packed_len(L0, d.residual) ? p.nb - 1 : -1;
     const bool packed = v < p.np;
+    // A flush is folded in by the packed warp np - 1 (it owns the last
+    // block).  The window warps of its CTA quantize the block's four quarters
+    // into the image while it streams; with no window warp in that CTA it
+    // does them itself, before streaming.
+    char* image = reinterpret_cast<char*>(smem + smem_size - 16 - kZeroBytes - image_bytes(page));
+    const int cta_f = (p.np - 1) / kWarps;
+    const int n_help = (cta_f + 1) * kWarps - p.np;  // window warps in CTA cta_f
+    if (flush_blk >= 0 && (int)blockIdx.x == cta_f && (n_help > 0 ? !packed : v == p.np - 1)) {
+      const int nw = n_help > 0 ? n_help : 1;
+      for (int qi = n_help > 0 ? v - p.np : 0; qi < 4; qi += nw) {
+        flush_quarter<BK, BV>(ring_k, ring_v, flush_blk * kGroup, d.ring, qi, image);
+        mbar_arrive(&fl_bar);
+      }
+    }
     TcState st;
     init_state(st);
     if (packed || pre > 0) {
@@ -1180,9 +1207,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       }
       tc_packed_warp<BK, BV, kWide>(pages, lo_h, pre, pre_end, lo, hi, ring, full, R,
                              reinterpret_cast<const char*>(zero), q_s, gq, scale_log2, flag, st,
-                             flush_blk, ring_k, ring_v, d.ring, &wbar[warp],
-                             reinterpret_cast<char*>(smem + smem_size - 16 - kZeroBytes -
-                                                     image_bytes(page)));
+                             flush_blk, &fl_bar, image);
     }
     if (!packed)
       tc_window_warp<BK, BV, kWide>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, q_s, gq,

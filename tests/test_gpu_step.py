@@ -20,7 +20,7 @@ def _cache_state(cache, lengths):
             for b, L in enumerate(lengths)]
 
 
-def _steps(cfg, lengths, n_steps, seed, check_oracle_every=0):
+def _steps(cfg, lengths, n_steps, seed, check_oracle_every=0, n_splits=0):
     a, kv = _util.make_cache(cfg, lengths, seed)
     b_, _ = _util.make_cache(cfg, lengths, seed)
     g = synth.generator(seed + 5)
@@ -31,7 +31,7 @@ def _steps(cfg, lengths, n_steps, seed, check_oracle_every=0):
         kn = torch.randn(cfg.batch, cfg.n_kv_heads, 128, generator=g).half()
         vn = torch.randn(cfg.batch, cfg.n_kv_heads, 128, generator=g).half()
         q = torch.randn(cfg.batch, cfg.n_q_heads, 128, generator=g).half()
-        out_a = kvq.kvq_decode_step(a, kn.cuda(), vn.cuda(), q.cuda())
+        out_a = kvq.kvq_decode_step(a, kn.cuda(), vn.cuda(), q.cuda(), n_splits=n_splits)
         kvq.kvq_pack(b_, kn[:, :, None].cuda(), vn[:, :, None].cuda())
         out_b = kvq.kvq_decode_attn(b_, q.cuda())
         torch.cuda.synchronize()
@@ -72,6 +72,22 @@ def test_wide_query_groups(kvq_lib, gq):
     cfg = kvq.CacheConfig(batch=3, n_q_heads=2 * gq, n_kv_heads=2, bits_k=1, bits_v=2,
                           max_len=1024)
     pair, oracle = _steps(cfg, [158, 400, 159], 5, seed=21 + gq, check_oracle_every=5)
+    assert pair <= 1e-5, pair
+    assert oracle <= _util.ATTN_TOL, oracle
+
+
+@pytest.mark.parametrize("residual,n_splits,bk,bv", [(32, 1, 1, 2), (96, 2, 2, 1), (160, 2, 1, 1),
+                                                    (512, 4, 1, 1), (512, 3, 4, 2)])
+def test_flush_workers_for_window_sizes(kvq_lib, residual, n_splits, bk, bv):
+    # The group leaving the window is quantized by the window warps of the
+    # CTA that folds it in: 1, 3, 5 and 12 of them here, and none for a
+    # 512-token window over 4 splits, where the folding warp does it alone.
+    R = residual
+    lengths = [R - 1, R + 30, R + 63, 3 * R + 5]
+    cfg = kvq.CacheConfig(batch=len(lengths), n_q_heads=8, n_kv_heads=2, bits_k=bk, bits_v=bv,
+                          max_len=4 * R + 128, residual=R)
+    pair, oracle = _steps(cfg, lengths, 34, seed=R + n_splits, check_oracle_every=17,
+                          n_splits=n_splits)
     assert pair <= 1e-5, pair
     assert oracle <= _util.ATTN_TOL, oracle
 
