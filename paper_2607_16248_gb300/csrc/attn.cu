@@ -1460,18 +1460,46 @@ int attn_default_splits(const Dims& d, int sm_count) {
 }
 
 // Split count from the sequence lengths, known to the caller on the host.
-// Up to half the SMs' worth of (sequence, kv-head) pairs: one
-// wave, as attn_default_splits.  More: one split each for lengths within 15%
-// of their mean; for a ragged batch about four waves of CTAs, so the
-// scheduler's dynamic fill evens out the long and short sequences.
+// Up to half the SMs' worth of (sequence, kv-head) pairs: one wave, as
+// attn_default_splits, unless a few waves of shorter splits fill the SMs
+// that one wave leaves idle (the pair count does not divide the SM count).
+// The estimate of a count n, in units of one packed block's compute, is
+// waves(n) x (blocks per split + kCtaFixedBlocks): measured on GB300, a
+// CTA's fixed cost (start, warp and split merges) is ~6.4 us, ~46 blocks
+// (64 pairs of 64k-token K1V1 sequences: 7 splits in 2.95 waves take 140.6
+// us per layer against 156.7 for 2 splits in one wave).  A count is taken
+// only if it is estimated 2% faster, and at most four waves.  More pairs:
+// one split each for lengths within 15% of their mean; for a ragged batch
+// about four waves of CTAs, so the scheduler's dynamic fill evens out the
+// long and short sequences.
+constexpr int kCtaFixedBlocks = 46;
 int attn_splits_for_lengths(const Dims& d, int sm_count, const int32_t* lengths) {
   const int bh = d.batch * d.hkv;
-  if (2 * bh <= sm_count) return attn_default_splits(d, sm_count);
   long long sum = 0;
   int mx = 0;
   for (int b = 0; b < d.batch; ++b) {
     sum += lengths[b];
     mx = lengths[b] > mx ? lengths[b] : mx;
+  }
+  if (2 * bh <= sm_count) {
+    const int n1 = attn_default_splits(d, sm_count);
+    const double nb = (double)(packed_len(mx, d.residual) / kGroup);
+    const int slots = kCtasPerSm * sm_count;
+    const int cap = min((d.max_blocks + 3) / 4, kMaxSplits - 1);
+    auto estimate = [&](int n) {
+      const long long waves = ((long long)bh * n + slots - 1) / slots;
+      return (double)waves * (nb / n + kCtaFixedBlocks);
+    };
+    int best = n1;
+    double best_t = estimate(n1);
+    for (int n = n1 + 1; n <= cap && (long long)bh * n <= 4LL * slots; ++n) {
+      const double t = estimate(n);
+      if (t < 0.98 * best_t) {
+        best = n;
+        best_t = t;
+      }
+    }
+    return best;
   }
   if ((double)mx <= 1.15 * (double)sum / d.batch) return attn_default_splits(d, sm_count);
   int n = (4 * sm_count + bh / 2) / bh;

@@ -99,6 +99,13 @@ def test_splits_for_lengths(L):
     assert 3 <= n(big, ragged) <= 8 and n(big, ragged) > d  # about four waves
     one = kvq.CacheConfig(batch=1, n_q_heads=32, n_kv_heads=8, bits_k=1, bits_v=1, max_len=32800)
     assert n(one, [32768]) == L.kvq_attn_default_splits(ctypes.byref(one.c()))
+    # 64 pairs (Qwen-14B shape, batch 8): one wave of 2 splits leaves 24 of
+    # 152 SMs idle; at 64k tokens 7 splits in 2.95 waves are faster, at 4k
+    # the fixed cost of each wave outweighs the fill
+    qwen = kvq.CacheConfig(batch=8, n_q_heads=40, n_kv_heads=8, bits_k=1, bits_v=1, max_len=65664)
+    assert L.kvq_attn_default_splits(ctypes.byref(qwen.c())) == 2
+    assert n(qwen, [65536] * 8) == 7
+    assert n(qwen, [4096] * 8) == 2
     assert n(big, [20000] * 15 + [40000]) == 0  # beyond max_len
     assert n(big, [-1] + [20000] * 15) == 0
 
