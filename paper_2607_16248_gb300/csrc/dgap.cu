@@ -237,28 +237,16 @@ __device__ __forceinline__ uint32_t warp_kth_key(uint32_t k, int q) {
 
 constexpr int kSurvivors = 1024;  // candidates kept for the exact ranking
 
-// The n best (n <= 72) of the elements the CTA's threads hold in registers
-// (E per thread; key 0 marks padding), sorted best first into ok / oi.
-// Every warp's q = ceil(n / 8)-th largest per-thread maximum bounds the n-th
-// best key from below (8 q >= n elements reach it), so the elements at or
-// above the smallest of those bounds contain the n best.  They are packed
-// into sv as (key, ~index) words, whose order is the ranking order, and
-// ranked exactly.  With more than kSurvivors of them (heavy ties) every
-// thread calls fallback() instead.
+// The n best of the elements held in registers whose key is at least T0, a
+// lower bound on the n-th best key (so they contain the n best), sorted best
+// first into ok / oi: packed into sv as (key, ~index) words, whose order is
+// the ranking order, and ranked exactly.  With more than kSurvivors of them
+// (heavy ties) every thread calls fallback() instead.
 template <int E, typename Fallback>
-__device__ void select_top(const uint32_t (&k)[E], const int (&x)[E], int n, Sel& ss,
-                           unsigned long long* sv, uint32_t* ok, int* oi,
-                           const Fallback& fallback) {
+__device__ void select_above(const uint32_t (&k)[E], const int (&x)[E], int n, uint32_t T0,
+                             Sel& ss, unsigned long long* sv, uint32_t* ok, int* oi,
+                             const Fallback& fallback) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  uint32_t mk = 0u;
-#pragma unroll
-  for (int i = 0; i < E; ++i) mk = max(mk, k[i]);
-  const uint32_t wq = warp_kth_key(mk, (n + kWarpsD - 1) / kWarpsD);
-  if (lane == 0) ss.hist[warp] = wq;
-  __syncthreads();
-  uint32_t T0 = ss.hist[0];
-#pragma unroll
-  for (int w = 1; w < kWarpsD; ++w) T0 = min(T0, ss.hist[w]);
   int c = 0;
 #pragma unroll
   for (int i = 0; i < E; ++i) c += k[i] >= T0;
@@ -302,6 +290,28 @@ __device__ void select_top(const uint32_t (&k)[E], const int (&x)[E], int n, Sel
   __syncthreads();
 }
 
+// The n best (n <= 72) of the elements the CTA's threads hold in registers
+// (E per thread; key 0 marks padding), sorted best first into ok / oi.
+// Every warp's q = ceil(n / 8)-th largest per-thread maximum bounds the n-th
+// best key from below (8 q >= n elements reach it); select_above does the
+// rest.
+template <int E, typename Fallback>
+__device__ void select_top(const uint32_t (&k)[E], const int (&x)[E], int n, Sel& ss,
+                           unsigned long long* sv, uint32_t* ok, int* oi,
+                           const Fallback& fallback) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t mk = 0u;
+#pragma unroll
+  for (int i = 0; i < E; ++i) mk = max(mk, k[i]);
+  const uint32_t wq = warp_kth_key(mk, (n + kWarpsD - 1) / kWarpsD);
+  if (lane == 0) ss.hist[warp] = wq;
+  __syncthreads();
+  uint32_t T0 = ss.hist[0];
+#pragma unroll
+  for (int w = 1; w < kWarpsD; ++w) T0 = min(T0, ss.hist[w]);
+  select_above(k, x, n, T0, ss, sv, ok, oi, fallback);
+}
+
 constexpr int kCandReg = 16;                // candidates of a row per thread (finalize)
 constexpr size_t kW1StageMax = 168 * 1024;  // largest staged corrector W1 (256 x 168)
 
@@ -316,6 +326,8 @@ struct Smem {
   uint64_t w1_bar;
   Sel sel;
   unsigned long long sv[kSurvivors];    // select_top: candidates above the bound
+  unsigned long long su[kMaxK + 1 + kMaxChunks];  // finalize: leaders of every list
+  uint32_t t0;                          // finalize: lower bound on the window's keys
   uint32_t wk[kWarpsD][kMaxK + 1];
   int wi[kWarpsD][kMaxK + 1];
   uint32_t fk[kMaxK + 1];
@@ -352,6 +364,7 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
   const bool w1s = stage_w1(d, p);
   const uint32_t w1_bytes = (uint32_t)((size_t)d.hidden * nin * sizeof(float));
   if (w1s && tid == 0) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // chunk-phase writes first
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&sm.w1_bar)) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(&sm.w1_bar)),
@@ -373,6 +386,22 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     dw2 = __ldg(p.det_w2 + tid);
   }
 
+  // The corrector's output-layer weights of this thread (output k = tid / 8,
+  // every eighth hidden unit from tid mod 8), when that layer is one pass of
+  // at most 256 units, and its hidden bias: fetched with the first round of
+  // loads, used only if the row is gated.
+  constexpr int kW2Reg = 32;
+  const bool w2r = K <= kT / 8 && d.hidden <= 8 * kW2Reg;
+  float w2v[kW2Reg];
+  if (w2r) {
+    const int k = tid >> 3, s8 = tid & 7;
+#pragma unroll
+    for (int i = 0; i < kW2Reg; ++i) {
+      const int j = s8 + 8 * i;
+      w2v[i] = (k < K && j < d.hidden) ? __ldg(p.cor_w2 + (size_t)k * d.hidden + j) : 0.0f;
+    }
+  }
+  const float cb1 = tid < d.hidden ? __ldg(p.cor_b1 + tid) : 0.0f;
   // Chunk statistics and candidate lists in one round of loads.
   const uint2* cand = ws.cand + (size_t)row * nc * K1;
   const int n_cand = nc * K1;
@@ -385,15 +414,51 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     ck[e] = v.x;
     cx[e] = (int)v.y;
   }
-  float mloc = -INFINITY;
+  // The lists are sorted best first, so the first r0 = ceil(K1 / nc)
+  // entries of every list (r0 nc >= K1 of them, all at or above their own
+  // K1-th best) bound the K1-th best overall from below by their K1-th best.
+  // On lists of leaders this bound is far tighter than select_top's per-warp
+  // one, and few candidates are left to rank.
+  const int r0 = (K1 + nc - 1) / nc, m_u = r0 * nc;  // m_u <= K1 + nc - 1 <= 2 kT
+  uint2 uv[2];
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const int t = tid + e * kT;
+    uv[e] = t < m_u ? __ldcg(&cand[(t / r0) * K1 + t % r0]) : make_uint2(0u, 0u);
+  }
   float4 sv[(kMaxChunks + kT - 1) / kT];
 #pragma unroll
   for (int j = 0; j < (kMaxChunks + kT - 1) / kT; ++j) {
     const int c = tid + j * kT;
     sv[j] = c < nc ? __ldcg(&st[c]) : make_float4(-INFINITY, 0.0f, 0.0f, 0.0f);
-    mloc = fmaxf(mloc, sv[j].x);
   }
-  const float M = block_max(mloc, sm.red);
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const int t = tid + e * kT;
+    if (t < m_u) sm.su[t] = ((unsigned long long)uv[e].x << 32) | (uint32_t)~uv[e].y;
+  }
+  float mloc = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < (kMaxChunks + kT - 1) / kT; ++j) mloc = fmaxf(mloc, sv[j].x);
+  const float M = block_max(mloc, sm.red);  // also publishes su
+  {
+    // rank of each leader, P = 8, 4, 2 or 1 consecutive lanes per leader
+    // (each over every P-th other leader, summed by shuffles); the one of
+    // rank K1 - 1 gives the bound
+    const int P = m_u <= kT / 8 ? 8 : m_u <= kT / 4 ? 4 : m_u <= kT / 2 ? 2 : 1;
+    for (int base = 0; base < m_u * P; base += kT) {
+      const int w = base + tid, t = w / P, part = w % P;
+      const unsigned long long me = t < m_u ? sm.su[t] : 0ull;
+      int r = 0;
+      if (t < m_u)
+        for (int j = part; j < m_u; j += P) {
+          const unsigned long long o = sm.su[j];
+          r += (o > me) || (o == me && j < t);
+        }
+      for (int o = 1; o < P; o <<= 1) r += __shfl_xor_sync(0xffffffffu, r, o);
+      if (t < m_u && part == 0 && r == K1 - 1) sm.t0 = (uint32_t)(me >> 32);
+    }
+  }
   float s1 = 0.0f, s2 = 0.0f;
 #pragma unroll
   for (int j = 0; j < (kMaxChunks + kT - 1) / kT; ++j) {
@@ -417,7 +482,7 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     }, sm.sel, sm.fk, sm.fi, &sm.wk[0][0], &sm.wi[0][0]);
   };
   if (n_cand > kCandReg * kT) from_global();
-  else select_top(ck, cx, K1, sm.sel, sm.sv, sm.fk, sm.fi, from_global);
+  else select_above(ck, cx, K1, sm.t0, sm.sel, sm.sv, sm.fk, sm.fi, from_global);
 
   // Features phi (Sec. 4.2): warp 0, lanes over the window.
   if (warp == 0) {
@@ -507,42 +572,32 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     }
     if (tid < 8) sm.x[5 * K + tid] = sm.phi[tid];
     __syncthreads();
-    // The output layer's weights of this thread (output k = tid / 8, every
-    // eighth hidden unit from tid mod 8) into registers meanwhile, when the
-    // layer is one pass of at most 256 units.
-    constexpr int kW2Reg = 32;
-    const bool w2r = K <= kT / 8 && d.hidden <= 8 * kW2Reg;
-    float w2v[kW2Reg];
-    if (w2r) {
-      const int k = tid >> 3, s8 = tid & 7;
-#pragma unroll
-      for (int i = 0; i < kW2Reg; ++i) {
-        const int j = s8 + 8 * i;
-        w2v[i] = (k < K && j < d.hidden) ? __ldg(p.cor_w2 + (size_t)k * d.hidden + j) : 0.0f;
-      }
-    }
     // Hidden layer: one thread per hidden unit (W1 from shared memory when
-    // staged); thread j starts at input j mod nin so that a warp's reads of
-    // its 32 rows fall in different banks.
+    // staged).
     const float* w1 = (w1s && w1_ok) ? sm.u.w1 : p.cor_w1;
     if (w1s && w1_ok && (nin & 3) == 0) {
-      // staged rows of 16-byte multiples: float4 reads, four accumulators
+      // staged rows of float4s, four accumulators.  With an even number n4
+      // of float4s per row, thread j starts at column j mod 8: the float4 at
+      // column c of row j lies in 16-byte bank group (j n4 + c) mod 8, so the
+      // eight rows a quarter-warp reads fall in groups j (n4 + 1) mod 8, all
+      // different (n4 + 1 odd), and so do the eight inputs it reads.
       const float4* xv = reinterpret_cast<const float4*>(sm.x);
       const int n4 = nin / 4;
       for (int j = tid; j < d.hidden; j += kT) {
         const float4* wr = reinterpret_cast<const float4*>(sm.u.w1 + (size_t)j * nin);
         float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-        int c = j % n4;  // skewed start: the eight rows of a phase hit different banks
+        int c = (n4 & 1) ? 0 : (j & 7) % n4;
 #pragma unroll 6
         for (int t = 0; t < n4; ++t) {
           const float4 w = wr[c], xx = xv[c];
+          c = c + 1 == n4 ? 0 : c + 1;
           a.x = fmaf(w.x, xx.x, a.x);
           a.y = fmaf(w.y, xx.y, a.y);
           a.z = fmaf(w.z, xx.z, a.z);
           a.w = fmaf(w.w, xx.w, a.w);
-          c = c + 1 == n4 ? 0 : c + 1;
         }
-        sm.hb[j] = fmaxf((a.x + a.y) + (a.z + a.w) + p.cor_b1[j], 0.0f);
+        const float b1 = j == tid ? cb1 : __ldg(p.cor_b1 + j);
+        sm.hb[j] = fmaxf((a.x + a.y) + (a.z + a.w) + b1, 0.0f);
       }
     } else
     for (int j = tid; j < d.hidden; j += kT) {
@@ -594,17 +649,28 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
   if (tid == 0) {
     risk[row] = 1.0f / (1.0f + expf(-f));
     gate[row] = gated ? 1 : 0;
-    if (next_token) {
-      float bv = key_value(sm.fk[K]);
-      int bi = sm.fi[K];
-      for (int k = 0; k < K; ++k)
-        if (sm.zt[k] > bv || (sm.zt[k] == bv && sm.fi[k] < bi)) {
-          bv = sm.zt[k];
-          bi = sm.fi[k];
-        }
-      next_token[row] = bi;
-    }
     ws.tk[row] = 0u;
+  }
+  if (next_token && warp == 0) {
+    // greedy token: the best of the corrected window and z_(K+1), the lower
+    // index on ties (a total order, so the lanes' partial bests reduce)
+    float bv = lane == 0 ? key_value(sm.fk[K]) : -INFINITY;
+    int bi = lane == 0 ? sm.fi[K] : INT_MAX;
+    for (int k = lane; k < K; k += 32)
+      if (sm.zt[k] > bv || (sm.zt[k] == bv && sm.fi[k] < bi)) {
+        bv = sm.zt[k];
+        bi = sm.fi[k];
+      }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (ov > bv || (ov == bv && oi < bi)) {
+        bv = ov;
+        bi = oi;
+      }
+    }
+    if (lane == 0) next_token[row] = bi;
   }
 }
 

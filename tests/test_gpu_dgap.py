@@ -118,6 +118,23 @@ def test_ties_and_signed_zeros(kvq_lib):
     _compare(zin, out, zout, K, -1.0, det, cor)
 
 
+def test_ties_across_chunk_lists(kvq_lib):
+    # 32 chunk lists of a 128256-token row whose leaders tie: every list all
+    # one key (more survivors than the exact ranking holds: the radix
+    # fallback), a few lists tied at the bound, and keys rounded to a coarse
+    # grid
+    B, V, K = 3, 128256, 32
+    g = synth.generator(19)
+    z = torch.empty(B, V)
+    z[0] = torch.randint(0, 40, (V,), generator=g).float()
+    z[1] = torch.randint(0, 6000, (V,), generator=g).float() / 8.0
+    z[2] = torch.round(torch.randn(V, generator=g) * 12.0) / 4.0
+    zin, out, zout, det, cor = _run(B, V, K, -1.0, seed=19, logits=z)
+    idx = out["topk_idx"].cpu().numpy()
+    assert idx[0].tolist() == np.flatnonzero(z[0].numpy() == 39.0)[:K].tolist()
+    _compare(zin, out, zout, K, -1.0, det, cor)
+
+
 def test_shift_invariance_on_gpu(kvq_lib):
     B, V, K = 4, 10000, 32
     z = synth.logits(12, B, V)

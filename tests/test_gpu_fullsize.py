@@ -1,6 +1,7 @@
 """Parity at the benchmark workloads' full sizes, in the launch configuration
-bench.py times (kvq_decode_step with the default split count, one layer of
-each shape; dgap_restore on the full logit rows).  The oracle recomputes
+bench.py times (kvq_decode_step with the split count kvq.splits_for_lengths
+gives for the prefill lengths, one layer of each shape; dgap_restore on the
+full logit rows).  The oracle recomputes
 sampled (sequence, kv-head) pairs one by one; DGAP rows are all checked.
 
 Workloads: Llama-8B K1V1 at 32768 tokens; the bit-width sweep (K1V1..K8V8) at
@@ -34,7 +35,10 @@ def _one_layer(cfg, lengths, seed, samples):
     kn = torch.randn(cfg.batch, cfg.n_kv_heads, 128, generator=g).half()
     vn = torch.randn(cfg.batch, cfg.n_kv_heads, 128, generator=g).half()
     q = torch.randn(cfg.batch, cfg.n_q_heads, 128, generator=g).half()
-    out = kvq.kvq_decode_step(cache, kn.cuda(), vn.cuda(), q.cuda()).cpu().numpy()
+    ns = kvq.splits_for_lengths(cfg, lengths)
+    ws = kvq.attn_workspace(cfg, ns)
+    out = kvq.kvq_decode_step(cache, kn.cuda(), vn.cuda(), q.cuda(), n_splits=ns,
+                              workspace=ws).cpu().numpy()
     assert cache.seq_lens().cpu().tolist() == [L + 1 for L in lengths]
     assert cache.flags() == 0
     gq = cfg.n_q_heads // cfg.n_kv_heads
