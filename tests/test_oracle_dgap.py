@@ -135,6 +135,31 @@ def test_mlp_closed_forms():
     assert np.allclose(out["val"], 2 * zs[:K] - zs[1:], rtol=0, atol=1e-14)
 
 
+def test_mlp_orientation_with_permuted_first_layer():
+    # A square first layer that is a permutation: hidden unit j reads input
+    # perm[j] (W1[j, perm[j]] = 1).  Output k reads the hidden unit that
+    # holds xi[k, 4] = z_(k) - z_(k+1) >= 0, so Delta_k equals that gap; a
+    # transposed W1 (unit j reading the input whose image is j) picks other
+    # inputs and fails.
+    K = 4
+    nin = 5 * K + 8
+    perm = np.random.default_rng(9).permutation(nin)
+    inv = np.argsort(perm)
+    cor = dict(w1=np.zeros((nin, nin)), b1=np.zeros(nin), w2=np.zeros((K, nin)), b2=np.zeros(K))
+    cor["w1"][np.arange(nin), perm] = 1.0
+    for k in range(K):
+        cor["w2"][k, inv[5 * k + 4]] = 1.0
+    det = dict(w1=np.zeros((2, 8)), b1=np.zeros(2), w2=np.zeros((1, 2)), b2=np.array([1.0]))
+    z = np.random.default_rng(10).standard_normal(300) * 2
+    out = dgap.restore_row(z, K, 0.5, det, cor)  # r = sigmoid(1) > 0.5: gated
+    assert out["gate"]
+    zs = z[dgap.topk_window(z, K)]
+    assert np.allclose(out["delta"], zs[:K] - zs[1:], rtol=0, atol=1e-14)
+    # the same weights transposed read other inputs
+    cor_t = dict(cor, w1=cor["w1"].T.copy())
+    assert not np.allclose(dgap.restore_row(z, K, 0.5, det, cor_t)["delta"], zs[:K] - zs[1:])
+
+
 def test_next_token_is_argmax_of_merged_row():
     det, cor = _weights(6, K=8, hidden=32)
     rng = np.random.default_rng(5)
