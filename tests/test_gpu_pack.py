@@ -107,3 +107,63 @@ def test_constant_and_grid_groups_reach_exact_codes(kvq_lib):
     assert np.all(got["k_scale"][:, :64] == 0)
     assert np.all(got["k_scale"][:, 64:] == 1)
     assert np.all(got["v_scale"].astype(np.float64) == 0.25)
+
+
+@pytest.mark.parametrize("bits", [1, 2, 4, 8])
+def test_exact_ties_round_to_even(kvq_lib, bits):
+    # Every group holds 0, 3 * levels and values 1.5 (2m + 1): scale 3 (not a
+    # power of two), so (x - zero) / scale = m + 0.5 exactly and each code is
+    # a tie that rounds to even.  RN32(1 / 3) times such an x lands just off
+    # the half-integer, so only the exact quotient gives these codes.
+    levels = (1 << bits) - 1
+
+    def pattern(i, c):
+        if i == 0:
+            return 0.0
+        if i == 1:
+            return 3.0 * levels
+        return 1.5 * (2 * ((7 * i + c) % levels) + 1)
+
+    L = 160
+    k = torch.empty(1, L, 128, dtype=torch.float16)
+    v = torch.empty(1, L, 128, dtype=torch.float16)
+    for t in range(L):
+        for c in range(128):
+            k[0, t, c] = pattern(t % 32, c)
+            v[0, t, c] = pattern(c % 32, t + c // 32)
+    cfg = kvq.CacheConfig(batch=1, n_q_heads=1, n_kv_heads=1, bits_k=bits, bits_v=bits,
+                          max_len=256)
+    cache = kvq.QuantKVCache(cfg)
+    kvq.kvq_pack(cache, k[None].cuda(), v[None].cuda())
+    torch.cuda.synchronize()
+    got = _util.head_arrays(cache, 0, 0, L)
+    want = quant.quantize_head(k[0].numpy(), v[0].numpy(), bits, bits, 128)
+    assert np.all(want["k_scale"].astype(np.float64) == 3.0)
+    assert np.all(want["v_scale"].astype(np.float64) == 3.0)
+    _util.assert_head_equal(got, want)
+
+
+def test_tie_where_a_reciprocal_product_misrounds(kvq_lib):
+    # 2-bit groups of range 0.6650390625 = 3 x 0.2216796875 (scale
+    # 0.2216796875): 0.33251953125 / scale is exactly 1.5 (code 2), while
+    # 0.33251953125 * RN32(1 / scale) rounds to 1.4999999 (code 1).
+    pat = [0.0, 0.6650390625, 0.11083984375, 0.33251953125, 0.55419921875]
+
+    def pattern(i, c):
+        return pat[i] if i < 2 else pat[2 + (i + c) % 3]
+
+    L = 160
+    k = torch.empty(1, L, 128, dtype=torch.float16)
+    v = torch.empty(1, L, 128, dtype=torch.float16)
+    for t in range(L):
+        for c in range(128):
+            k[0, t, c] = pattern(t % 32, c)
+            v[0, t, c] = pattern(c % 32, t)
+    cfg = kvq.CacheConfig(batch=1, n_q_heads=1, n_kv_heads=1, bits_k=2, bits_v=2, max_len=256)
+    cache = kvq.QuantKVCache(cfg)
+    kvq.kvq_pack(cache, k[None].cuda(), v[None].cuda())
+    torch.cuda.synchronize()
+    got = _util.head_arrays(cache, 0, 0, L)
+    want = quant.quantize_head(k[0].numpy(), v[0].numpy(), 2, 2, 128)
+    assert np.all(want["k_scale"].astype(np.float64) == 0.2216796875)
+    _util.assert_head_equal(got, want)
