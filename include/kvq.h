@@ -185,11 +185,16 @@ int32_t kvq_attn_default_splits(const kvq_config* cfg);
 /*
  * A split count for kvq_decode_attn / kvq_decode_step from the sequence
  * lengths, which the caller knows on the host (the library keeps them on the
- * device).  lengths: host int32 [batch], each in [0, max_len].  Equals
- * kvq_attn_default_splits unless the (sequence, kv-head) pairs fill more
- * than half the SMs and the longest length exceeds the mean by
- * more than 15%: then about four waves of CTAs (a ragged batch is balanced
- * by the CTA scheduler).  Returns 0 on an invalid argument.
+ * device).  lengths: host int32 [batch], each in [0, max_len].
+ *   Pairs (sequence, kv-head) filling at most half the SMs: one wave of
+ *   kvq_attn_default_splits, unless up to four waves of shorter splits fill
+ *   the SMs that one wave leaves idle and are estimated at least 2% faster
+ *   (waves x (32-token blocks per split + 46), 46 blocks being a CTA's
+ *   measured fixed cost).
+ *   More pairs: kvq_attn_default_splits when the longest length is within
+ *   15% of the mean, else about four waves of CTAs (a ragged batch is
+ *   balanced by the CTA scheduler).
+ * Returns 0 on an invalid argument.
  */
 int32_t kvq_attn_splits_for_lengths(const kvq_config* cfg, const int32_t* lengths);
 
