@@ -417,8 +417,9 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
   // The lists are sorted best first, so the first r0 = ceil(K1 / nc)
   // entries of every list (r0 nc >= K1 of them, all at or above their own
   // K1-th best) bound the K1-th best overall from below by their K1-th best.
-  // On lists of leaders this bound is far tighter than select_top's per-warp
-  // one, and few candidates are left to rank.
+  // They are loaded with this round and ranked directly, which spares
+  // select_top's shuffle network and one barrier; either bound leaves a few
+  // dozen candidates on such lists.
   const int r0 = (K1 + nc - 1) / nc, m_u = r0 * nc;  // m_u <= K1 + nc - 1 <= 2 kT
   uint2 uv[2];
 #pragma unroll
