@@ -2,17 +2,18 @@
 """Decode-step benchmark of the packed low-bit KV cache + DGAP epilogue.
 
 A step is one pass of the whole hot path over one batch: for every layer,
-kvq_pack appends the step's token and kvq_decode_attn attends over the cache;
-then dgap_restore runs once on the step's logits.  Default workload:
-Llama-3.1-8B-shaped K1V1 decode (batch 1, 32 q / 8 kv heads, head_dim 128,
-context 32768, 32 layers with distinct seeded caches, logits [1, 128256],
-K = 32, hidden 256, tau 0.60).  The per-step packed KV (~552 MB) is larger
-than L2, so every step streams it from HBM.
+kvq_decode_step appends the step's token and attends over the cache; then
+dgap_restore runs once on the step's logits.  Default workload:
+Qwen2.5-14B-shaped K1V1 decode (batch 8, 40 q / 8 kv heads, head_dim 128,
+context 65536, 48 layers with distinct seeded caches, logits [8, 152064],
+K = 32, hidden 256, tau 0.60), the largest configuration, and the model of
+the paper's latency table (Sec. 5.4).  The per-step packed KV (~13 GB) is
+far larger than L2, so every step streams it from HBM.
 
-The step runs as three CUDA graphs (packs, attentions, epilogue) replayed
-back to back, with CUDA events between them on the launching stream; the
-attention events give the dominant kernel's average launch duration for the
-roofline.  One JSON line is printed by rank 0.
+The whole step is one CUDA graph, replayed with a CUDA event between steps
+(total, median and p95 per step); the layers' decode-step launches alone
+form a second graph, whose events give the dominant kernel's average launch
+duration for the roofline.  One JSON line is printed by rank 0.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the CPU oracle on the same config
@@ -39,12 +40,12 @@ from pathlib import Path
 ROOT = Path(__file__).resolve().parent
 sys.path.insert(0, str(ROOT))
 
-DEFAULT_WORKLOAD = "llama8b-k1v1-32k"
+DEFAULT_WORKLOAD = "qwen14b-k1v1-64k"
 METRIC = "packed-KV decode attn HBM GB/s (% of GB300 peak); DGAP epilogue µs/step"
 FALLBACK_HBM_GBS = 6800.0
 DGAP_K, DGAP_HIDDEN, DGAP_TAU = 32, 256, 0.60
-ATTN_PROFILE = ROOT / "profiles" / "attn_llama8b_k1v1_32k.md"
-DRIFT_PROFILE = ROOT / "profiles" / "drift_paired_128k.md"
+PROFILES = ROOT / "profiles"
+DRIFT_PROFILE = PROFILES / "drift_paired_128k.md"
 DRIFT_METRIC = "drift metrics on paired logits: HBM GB/s (% of GB300 peak)"
 # Offline drift tooling: 256 decode steps of paired Llama-vocabulary logits.
 DRIFT_WORKLOADS = {
@@ -56,7 +57,7 @@ DRIFT_WORKLOADS = {
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=2000)
+    p.add_argument("--steps", type=int, default=500)
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", default="kvq", choices=["kvq", "reference"])
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
@@ -94,10 +95,10 @@ def packed_len(L, R=128):
 def attn_bytes(L, hkv, hq, bk, bv, R=128):
     """Algorithmic HBM bytes of one sequence's attention for one layer:
     packed codes + scale/zero of Lq tokens, fp16 residual tokens, q (fp16 in)
-    and out (fp32)."""
+    and out (fp16)."""
     Lq = packed_len(L, R)
     per_tok = 16 * (bk + bv) + 32
-    return hkv * (Lq * per_tok + (L - Lq) * 512) + hq * 128 * (2 + 4)
+    return hkv * (Lq * per_tok + (L - Lq) * 512) + hq * 128 * (2 + 2)
 
 
 def source_digest(*names):
@@ -107,8 +108,12 @@ def source_digest(*names):
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(path=ATTN_PROFILE, sources=("attn.cu", "common.cuh"),
-                     sha_key="attn_source_sha"):
+def attn_profile(workload):
+    """The committed ncu summary of the attention kernel on this workload."""
+    return PROFILES / f"attn_{workload.replace('-', '_')}.md"
+
+
+def profiled_traffic(path, sources=("attn.cu", "common.cuh"), sha_key="attn_source_sha"):
     """DRAM bytes per launch of the profiled kernel from its committed ncu
     summary, if it was taken on the current source."""
     if not path.exists():
@@ -199,13 +204,15 @@ class Clocks:
 # ---------------------------------------------------------------------------
 
 
-def cpu_worker(spec_json, budget_s, mode):
-    """Run the oracle on a bounded sample of the workload; print JSON."""
+def _oracle_unit(spec):
+    """One unit of oracle work on the workload: the float64 dequantization
+    and softmax attention of one (layer, kv-head) of one sequence at the
+    workload's context.  Returns (run, unit_bytes, epilogue), each a call
+    without arguments; the inputs are built here, outside any timing."""
     import numpy as np
     from oracle import attention, dgap, quant
     from paper_2607_16248_gb300 import synth
 
-    spec = json.loads(spec_json)
     hkv, hq, b = spec["n_kv_heads"], spec["n_q_heads"], spec["bits"]
     gq = hq // hkv
     L = spec["context"] if isinstance(spec["context"], int) else spec["context"][1]
@@ -215,42 +222,95 @@ def cpu_worker(spec_json, budget_s, mode):
     w = synth.dgap_weights(spec["seed"], K=DGAP_K, hidden=DGAP_HIDDEN)
     det, cor = synth.split_weights(w)
     z = synth.logits(spec["seed"], 1, spec["vocab"])[0].numpy().astype(np.float64)
-    unit_bytes = attn_bytes(L, 1, gq, b, b)
 
-    def unit():
+    def run():
         khat, vhat = quant.dequantize_head(qh)
         attention.attend_head(q, khat, vhat, 1 / math.sqrt(128))
 
+    def epilogue():
+        dgap.restore_row(z, DGAP_K, DGAP_TAU, det, cor)
+
+    return run, attn_bytes(L, 1, gq, b, b), epilogue
+
+
+def _pool_member(spec_json, seconds, n_units, warmup, barrier, results, index):
+    """One host core of the all-cores oracle run: build the inputs, run
+    `warmup` untimed units, wait for every member, then run units for
+    `seconds` (or exactly n_units)."""
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[var] = "1"
+    sys.path.insert(0, str(ROOT))
+    run, _, _ = _oracle_unit(json.loads(spec_json))
+    for _ in range(warmup):
+        run()
+    barrier.wait()
     t0 = time.perf_counter()
-    unit()
+    n = 0
+    while (n_units is None and (time.perf_counter() - t0 < seconds or n == 0)) or \
+            (n_units is not None and n < n_units):
+        run()
+        n += 1
+    results.put((index, n, time.perf_counter() - t0))
+
+
+def oracle_all_cores(spec, seconds=None, n_units=None, cores=None, warmup=0):
+    """The oracle on every host core at once: one spawned process per core,
+    each running whole units on its own (one thread each).  Returns
+    (units done, wall seconds of the slowest member, cores)."""
+    import multiprocessing as mp
+    cores = cores or os.cpu_count() or 1
+    ctx = mp.get_context("spawn")
+    barrier = ctx.Barrier(cores)
+    results = ctx.Queue()
+    procs = [ctx.Process(target=_pool_member,
+                         args=(json.dumps(spec), seconds, n_units, warmup, barrier, results, i))
+             for i in range(cores)]
+    for p in procs:
+        p.start()
+    got = [results.get(timeout=1800) for _ in procs]
+    for p in procs:
+        p.join(timeout=60)
+    return sum(n for _, n, _ in got), max(t for _, _, t in got), cores
+
+
+def cpu_worker(spec_json, budget_s, mode):
+    """Run the oracle on a bounded sample of the workload; print JSON."""
+    spec = json.loads(spec_json)
+    hkv, b = spec["n_kv_heads"], spec["bits"]
+    L = spec["context"] if isinstance(spec["context"], int) else spec["context"][1]
+    run, unit_bytes, epilogue = _oracle_unit(spec)
+    t0 = time.perf_counter()
+    run()
     t_unit = time.perf_counter() - t0
     t0 = time.perf_counter()
-    dgap.restore_row(z, DGAP_K, DGAP_TAU, det, cor)
+    epilogue()
     t_epi = time.perf_counter() - t0
+    what = (f"one (layer, kv-head) of {hkv * spec['layers']} per step, context {L}, K{b}V{b}: "
+            f"float64 dequant + softmax attention (numpy)")
     if mode == "baseline":
-        n = max(1, int(budget_s / max(t_unit, 1e-6)))
+        # one thread for half the budget, then every host core for the other half
+        n1 = max(1, int(0.5 * budget_s / max(t_unit, 1e-6)))
         t0 = time.perf_counter()
-        for _ in range(n):
-            unit()
-        t = time.perf_counter() - t0
-        out = {"value": unit_bytes * n / t / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
-               "epilogue_ms_per_row": t_epi * 1e3,
-               "sample": f"{n} x one (layer, kv-head) of {hkv * spec['layers']} per step, "
-                         f"context {L}, K{b}V{b}: float64 dequant + softmax attention "
-                         f"(numpy, 1 thread); DGAP restore of one [{spec['vocab']}] row "
-                         f"timed once"}
-    else:  # reference arm: W + K steps of one sampled unit each
+        for _ in range(n1):
+            run()
+        t1 = time.perf_counter() - t0
+        n_all, t_all, cores = oracle_all_cores(spec, seconds=0.5 * budget_s)
+        out = {"value": unit_bytes * n_all / t_all / 1e9, "unit": "GB/s", "cores": cores,
+               "kind": "oracle", "epilogue_ms_per_row": t_epi * 1e3,
+               "single_thread": {"value": unit_bytes * n1 / t1 / 1e9, "unit": "GB/s",
+                                 "cores": 1, "units": n1},
+               "sample": f"{n_all} units on {cores} host cores at once (one process each) and "
+                         f"{n1} on one thread; a unit is {what}; DGAP restore of one "
+                         f"[{spec['vocab']}] row timed once"}
+    else:  # reference arm: W + K steps, a step = one unit on every host core at once
         steps, warmup = spec["_steps"], spec["_warmup"]
-        for _ in range(warmup):
-            unit()
-        t0 = time.perf_counter()
-        for _ in range(steps):
-            unit()
-        t = time.perf_counter() - t0
-        out = {"value": unit_bytes * steps / t / 1e9, "unit": "GB/s", "cores": 1,
-               "ms_per_step": t / steps * 1e3, "kind": "oracle",
-               "sample": f"each step: one (layer, kv-head) of {hkv * spec['layers']}, "
-                         f"context {L}, K{b}V{b}, float64 numpy, 1 thread"}
+        cores = spec.get("_cores") or os.cpu_count() or 1
+        n_all, t_all, cores = oracle_all_cores(spec, n_units=steps, cores=cores, warmup=warmup)
+        per_step = t_all / steps
+        out = {"value": unit_bytes * cores / per_step / 1e9, "unit": "GB/s", "cores": cores,
+               "ms_per_step": per_step * 1e3, "kind": "oracle",
+               "sample": f"each step: {cores} units at once, one per host core; a unit is "
+                         f"{what}; {warmup} untimed warm-up units per core first"}
     print(json.dumps(out))
 
 
@@ -262,7 +322,7 @@ def run_cpu_worker(spec, budget_s, mode):
     cmd = [sys.executable, str(ROOT / "bench.py"), "--cpu-worker", mode,
            "--workload", "x"]
     res = subprocess.run(cmd + ["--", json.dumps(spec), str(budget_s)], env=env,
-                         stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True, timeout=900)
+                         stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True, timeout=1800)
     if res.returncode != 0:
         raise RuntimeError(f"cpu worker failed: {res.stderr[-2000:]}")
     return json.loads(res.stdout.strip().splitlines()[-1])
@@ -303,6 +363,18 @@ def reduce_max(x, world):
     t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def percentile(xs, q):
+    """The q-th percentile of xs by linear interpolation between order
+    statistics (numpy's default rule)."""
+    v = sorted(xs)
+    if not v:
+        return float("nan")
+    pos = (len(v) - 1) * q / 100.0
+    lo = int(math.floor(pos))
+    hi = min(lo + 1, len(v) - 1)
+    return v[lo] + (v[hi] - v[lo]) * (pos - lo)
 
 
 def job_gbs(world, bytes_per_rank, ms_max):
@@ -346,7 +418,7 @@ class Step:
         self.q = torch.randn(layers, B, hq, 128, generator=g, device=device).half()
         self.k_new = torch.randn(layers, B, hkv, 128, generator=g, device=device).half()
         self.v_new = torch.randn(layers, B, hkv, 128, generator=g, device=device).half()
-        self.out = torch.empty(layers, B, hq, 128, dtype=torch.float32, device=device)
+        self.out = torch.empty(layers, B, hq, 128, dtype=torch.float16, device=device)
         self.n_splits = kvq.splits_for_lengths(self.cfg, self.lengths0)
         self.ws_attn = kvq.attn_workspace(self.cfg, self.n_splits, device)
         self.dgap = kvq.DGAP(synth.dgap_weights(seed, K=DGAP_K, hidden=DGAP_HIDDEN), K=DGAP_K,
@@ -473,9 +545,23 @@ def run_gpu(args, spec):
     time.sleep(0.25)  # let the sampler come up before the timed region
     torch.cuda.synchronize()
     wall0 = time.perf_counter()
-    total_ms = timed(st.g_step.replay, 0, K)
+    # one event between consecutive steps: the total and the per-step times
+    # (median and p95, the paper reports p95 latency) come from the same run
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+    torch.cuda.synchronize()
+    barrier(world)
+    evs[0].record()
+    for i in range(K):
+        st.g_step.replay()
+        evs[i + 1].record()
+    torch.cuda.synchronize()
+    done += K
+    per_step = [evs[i].elapsed_time(evs[i + 1]) for i in range(K)]
+    total_ms = reduce_max(evs[0].elapsed_time(evs[K]), world)
     wall = time.perf_counter() - wall0
     clk = clocks.stop()
+    step_ms_median = reduce_max(statistics.median(per_step), world)
+    step_ms_p95 = reduce_max(percentile(per_step, 95.0), world)
     step_bytes = [st.bytes_for_step(step0 + i) for i in range(K)]
     bytes_total = sum(step_bytes)
 
@@ -503,6 +589,8 @@ def run_gpu(args, spec):
     ph_step0 = done + W
     attn_ms = timed(st.g_attn.replay, W, K)
     attn_bytes_total = sum(st.bytes_for_step(ph_step0 + i) for i in range(K))
+
+    single = single_layer_times(st, device) if rank == 0 else None
 
     value = job_gbs(world, bytes_total, total_ms)
     launches = K * st.launches_per_step()
@@ -533,6 +621,8 @@ def run_gpu(args, spec):
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": round(total_ms / K, 5),
+        "ms_per_step_median": round(step_ms_median, 5),
+        "ms_per_step_p95": round(step_ms_p95, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded N(0,1) q/k/v with 4 x10 key outlier channels per head; "
                 "N(0,3^2) logits; random-init DGAP MLPs)",
@@ -541,6 +631,7 @@ def run_gpu(args, spec):
         "attn_frac_of_peak": round(achieved / peak, 4),
         "attn_us_per_layer": round(attn_ms / attn_launches * 1e3, 3),
         "epilogue_us_per_step": round(epi_ms / K * 1e3, 3),
+        "single_layer": single,
         "epilogue_frac_of_step_attn": round(epi_ms / attn_ms, 5),
         "breakdown": "attn_us_per_layer: the step's kvq_decode_step launches (append + "
                      "attention) alone in one graph; epilogue_us_per_step: a graph of 10 x (logits "
@@ -549,7 +640,7 @@ def run_gpu(args, spec):
         "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "peak_source": f"{peak_kind} hbm_gbs (copy)",
-                     "traffic": profiled_traffic(),
+                     "traffic": profiled_traffic(attn_profile(args.workload)),
                      "algorithmic_bytes_per_launch": round(attn_bytes_total / attn_launches)},
         "gpu_launches": launches,
         "wall_s_timed": round(wall, 4),
@@ -566,6 +657,51 @@ def run_gpu(args, spec):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def single_layer_times(st, device, reps=50, warm=5):
+    """One layer's kvq_decode_attn (layer 0's cache, no append, so every
+    repetition sees the same input) timed alone, warm (back-to-back
+    repetitions: a layer smaller than L2 stays there) and cold (a buffer of
+    twice the L2 size written before each repetition), median and p95 in us.
+    Only for layers whose packed cache fits in half the L2: larger layers are
+    cold by construction and their time is attn_us_per_layer."""
+    import torch
+    from paper_2607_16248_gb300 import kvq
+    s = st.spec
+    st.rewind()
+    layer_bytes = sum(attn_bytes(L, s["n_kv_heads"], s["n_q_heads"], s["bits"], s["bits"])
+                      for L in st.lengths0)
+    l2 = torch.cuda.get_device_properties(device).L2_cache_size
+    if layer_bytes > l2 // 2:
+        return None
+    flush = torch.empty(2 * l2 // 4, dtype=torch.float32, device=device)
+    ws = kvq.attn_workspace(st.cfg, st.n_splits, device)
+    out = torch.empty_like(st.q[0])
+
+    def one():
+        kvq.kvq_decode_attn(st.caches[0], st.q[0], out=out, n_splits=st.n_splits, workspace=ws)
+
+    res = {}
+    for mode in ("warm", "cold"):
+        times = []
+        for i in range(warm + reps):
+            if mode == "cold":
+                flush.fill_(float(i))
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            one()
+            b.record()
+            b.synchronize()
+            if i >= warm:
+                times.append(a.elapsed_time(b) * 1e3)
+        res[f"{mode}_us_median"] = round(statistics.median(times), 3)
+        res[f"{mode}_us_p95"] = round(percentile(times, 95.0), 3)
+    res["reps"] = reps
+    res["bytes"] = layer_bytes
+    res["note"] = ("latency-bound single layer (no 70% claim): one kvq_decode_attn launch, "
+                   "events around the launch alone")
+    return res
 
 
 def run_e2e(st, W, K, world, done):

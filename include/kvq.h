@@ -168,10 +168,11 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache,
                     void* stream);
 
 /*
- * Split-K workspace for kvq_decode_attn: per (sequence, query head, split)
- * partial max, sum and fp32 output row for up to n_splits + 1 splits, plus
- * one ticket per (sequence, kv-head) (the size allows one per query head).
- * n_splits = 0 means the library's choice.  Returns 0 on an invalid config.
+ * Split-K workspace for kvq_decode_attn / kvq_decode_step: per (sequence,
+ * query head, split) partial max, sum and fp32 output row for the n_splits
+ * CTAs of one call, plus one ticket per (sequence, kv-head) (the size allows
+ * one per query head).  n_splits = 0 means the library's choice.  Returns 0
+ * on an invalid config.
  */
 size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits);
 
@@ -210,11 +211,10 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream);
  *   out[b, i] = softmax(q[b, i] . K_hat[b, g(i)]^T * softmax_scale) V_hat[b, g(i)]
  * over all L = seq_len[b] cached tokens (Sec. 1 gives softmax(QK^T/sqrt(d_k))V;
  * g(i) = i / (n_q_heads / n_kv_heads)).  K_hat, V_hat are the dequantized
- * blocks plus the fp16 residual window.
+ * blocks plus the fp16 residual window.  Accumulation is fp32; the result is
+ * rounded once to fp16 (round to nearest even) when it is stored.
  *   q              device fp16 [batch][n_q_heads][128], 16-byte aligned.
- *   out            device fp32 [batch][n_q_heads][128], 16-byte aligned (the
- *                  fp32 accumulation result; rounding it to fp16 is left to
- *                  the caller).
+ *   out            device fp16 [batch][n_q_heads][128], 16-byte aligned.
  *   softmax_scale  0 selects 1/sqrt(128).
  *   n_splits       CTAs per (sequence, kv-head) that share its 32-token
  *                  blocks and window chunks; 0 = kvq_attn_default_splits(cfg);
@@ -227,9 +227,19 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream);
  * must not overlap on the GPU.
  */
 kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache,
-                           const uint16_t* q, float* out,
+                           const uint16_t* q, uint16_t* out,
                            float softmax_scale, int32_t n_splits,
                            void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * kvq_decode_attn_f32 — kvq_decode_attn with the fp32 accumulation result
+ * stored unrounded: out is device fp32 [batch][n_q_heads][128].  Rounding it
+ * to fp16 to nearest even gives kvq_decode_attn's output bit for bit.
+ */
+kvq_status kvq_decode_attn_f32(const kvq_config* cfg, const kvq_cache* cache,
+                               const uint16_t* q, float* out,
+                               float softmax_scale, int32_t n_splits,
+                               void* workspace, size_t ws_bytes, void* stream);
 
 /*
  * kvq_decode_step — one decode step of one layer: kvq_pack of one token per
@@ -240,19 +250,28 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache,
  * kvq_pack) into its page and attended in quantized form; seq_len[b] becomes
  * L + 1 when the kernel ends.
  *   k_new, v_new   device fp16 [batch][n_kv_heads][128], 16-byte aligned.
- *   q, out, softmax_scale, n_splits, workspace, ws_bytes: as kvq_decode_attn.
+ *   q, out, softmax_scale, n_splits, workspace, ws_bytes: as kvq_decode_attn
+ *                  (out fp16).
  * A sequence at max_len is not appended (KVQ_FLAG_OVERFLOW is set) and
  * attends over its L tokens.  Results equal kvq_pack(n_new = 1) then
  * kvq_decode_attn on the same inputs.
  */
 kvq_status kvq_decode_step(const kvq_config* cfg, const kvq_cache* cache,
                            const uint16_t* k_new, const uint16_t* v_new,
-                           const uint16_t* q, float* out, float softmax_scale,
+                           const uint16_t* q, uint16_t* out, float softmax_scale,
                            int32_t n_splits, void* workspace, size_t ws_bytes,
                            void* stream);
 
+/* kvq_decode_step_f32 — kvq_decode_step with an fp32 out, as
+ * kvq_decode_attn_f32. */
+kvq_status kvq_decode_step_f32(const kvq_config* cfg, const kvq_cache* cache,
+                               const uint16_t* k_new, const uint16_t* v_new,
+                               const uint16_t* q, float* out, float softmax_scale,
+                               int32_t n_splits, void* workspace, size_t ws_bytes,
+                               void* stream);
+
 /*
- * kvq_decode_attn_noalloc — kvq_decode_attn without a caller workspace.
+ * kvq_decode_attn_noalloc — kvq_decode_attn_f32 without a caller workspace.
  * The paper has no counterpart; this serves callers that cannot allocate
  * device memory where they run a decode step: code inside a framework whose
  * memory pool owns the whole GPU (a raw allocation would fail or fragment
@@ -260,7 +279,8 @@ kvq_status kvq_decode_step(const kvq_config* cfg, const kvq_cache* cache,
  * partials and tickets live in one built-in device array of
  * KVQ_NOALLOC_SCRATCH_BYTES, which every GPU that loads this library holds
  * until the process exits.
- *   Arguments and results: those of kvq_decode_attn, without workspace.
+ *   Arguments and results: those of kvq_decode_attn_f32 (fp32 out), without
+ *   workspace.
  *   Returns KVQ_ERR_CAPACITY, with nothing enqueued, when
  *   kvq_attn_workspace_bytes(cfg, n_splits) > KVQ_NOALLOC_SCRATCH_BYTES.
  *   The first call on a device looks up the array's device address (once

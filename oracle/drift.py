@@ -57,10 +57,18 @@ def step_metrics(z_fp, z_q, alpha, K, eps, rho_c, k_max=None):
     """c_t, d_loc and y_t of Sec. 4.2 for one step, plus M_t and the coverage
     curve cov(K') for K' = 1 .. k_max (Sec. 4.1)."""
     z_fp = np.asarray(z_fp, dtype=np.float64)
+    C, _ = candidate_set(softmax(z_fp), order_desc(z_fp), alpha)
+    return metrics_given_candidates(z_fp, z_q, C, K, eps, rho_c, k_max)
+
+
+def metrics_given_candidates(z_fp, z_q, C, K, eps, rho_c, k_max=None):
+    """Steps 3-7 for a given FP16 candidate set C (Sec. 4.1-4.2): c_t, d_loc,
+    y_t and the coverage curve with C fixed rather than found from alpha;
+    M_t is |C|."""
+    z_fp = np.asarray(z_fp, dtype=np.float64)
     z_q = np.asarray(z_q, dtype=np.float64)
     V = z_fp.shape[0]
     p_fp, p_q = softmax(z_fp), softmax(z_q)
-    C, m = candidate_set(p_fp, order_desc(z_fp), alpha)
     in_c = np.zeros(V, bool)
     in_c[C] = True
     order_q = order_desc(z_q)
@@ -73,7 +81,7 @@ def step_metrics(z_fp, z_q, alpha, K, eps, rho_c, k_max=None):
     b = p_q[U] / p_q[U].sum()
     d = float(np.sqrt(((a - b) ** 2).sum()))
     y = bool(d > eps and c >= rho_c)
-    out = {"M": m, "c": c, "d_loc": d, "y": y, "C": C, "S": S}
+    out = {"M": len(C), "c": c, "d_loc": d, "y": y, "C": C, "S": S}
     if k_max is not None:
         top = order_q[:k_max]
         out["cov"] = np.cumsum(np.where(in_c[top], p_fp[top], 0.0))

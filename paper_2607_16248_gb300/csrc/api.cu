@@ -251,9 +251,17 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream) {
                      "kvq_workspace_init");
 }
 
-kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const uint16_t* q,
-                           float* out, float softmax_scale, int32_t n_splits,
-                           void* workspace, size_t ws_bytes, void* stream) {
+}  // extern "C"
+
+namespace kvq {
+
+// Shared host validation of the decode-attention calls; on success *scale_log2
+// holds softmax_scale (0 -> 1/sqrt(128)) times log2(e) and *n_splits the
+// split count to launch.
+static kvq_status check_attn_call(const kvq_config* cfg, const kvq_cache* cache,
+                                  const void* q, const void* out, float softmax_scale,
+                                  int32_t* n_splits, void* workspace, size_t ws_bytes,
+                                  float* scale_log2) {
   kvq_status s = check_config(cfg);
   if (s != KVQ_OK) return s;
   if ((s = check_cache(*cfg, cache)) != KVQ_OK) return s;
@@ -261,59 +269,88 @@ kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const 
   if (!aligned16(q) || !aligned16(out)) return fail(KVQ_ERR_ALIGN, "q / out must be 16-byte aligned");
   if (!(softmax_scale >= 0.0f) || isinf(softmax_scale))
     return fail(KVQ_ERR_ARG, "softmax_scale must be finite and >= 0");
-  if (n_splits == 0) n_splits = default_splits(*cfg);
-  if (n_splits < 1 || n_splits > kMaxSplits - 1)
-    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, n_splits);
-  Dims d = make_dims(*cfg);
-  const size_t need = attn_workspace_bytes(d, n_splits);
+  if (*n_splits == 0) *n_splits = default_splits(*cfg);
+  if (*n_splits < 1 || *n_splits > kMaxSplits - 1)
+    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, *n_splits);
+  const size_t need = attn_workspace_bytes(make_dims(*cfg), *n_splits);
   if (!workspace) return fail(KVQ_ERR_ARG, "workspace is NULL");
   if (!aligned16(workspace)) return fail(KVQ_ERR_ALIGN, "workspace must be 16-byte aligned");
   if (ws_bytes < need)
     return fail(KVQ_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", ws_bytes, need);
   const float scale = softmax_scale == 0.0f ? 1.0f / sqrtf((float)kHeadDim) : softmax_scale;
-  const float scale_log2 = scale * 1.4426950408889634f;
-  trace("kvq_decode_attn batch %d heads %d/%d bits K%dV%d grid (%d, %d, %d) x 512, %d splits",
-        d.batch, d.hq, d.hkv, d.bits_k, d.bits_v, n_splits, d.hkv * ((d.gq + 3) / 4), d.batch,
-        n_splits);
-  return cuda_status(launch_decode_attn(d, *cache, reinterpret_cast<const __half*>(q),
-                                        out, scale_log2, n_splits,
-                                        workspace, static_cast<cudaStream_t>(stream)),
+  *scale_log2 = scale * 1.4426950408889634f;
+  return KVQ_OK;
+}
+
+static kvq_status decode_attn(const kvq_config* cfg, const kvq_cache* cache, const uint16_t* q,
+                              void* out, int out_f16, float softmax_scale, int32_t n_splits,
+                              void* workspace, size_t ws_bytes, void* stream) {
+  float sl2 = 0.0f;
+  kvq_status s = check_attn_call(cfg, cache, q, out, softmax_scale, &n_splits, workspace,
+                                 ws_bytes, &sl2);
+  if (s != KVQ_OK) return s;
+  Dims d = make_dims(*cfg);
+  trace("kvq_decode_attn%s batch %d heads %d/%d bits K%dV%d grid (%d, %d, %d) x 512, %d splits",
+        out_f16 ? "" : "_f32", d.batch, d.hq, d.hkv, d.bits_k, d.bits_v, n_splits, d.hkv,
+        d.batch, n_splits);
+  return cuda_status(launch_decode_attn(d, *cache, reinterpret_cast<const __half*>(q), out,
+                                        out_f16, sl2, n_splits, workspace,
+                                        static_cast<cudaStream_t>(stream)),
                      "kvq_decode_attn launch");
 }
 
+static kvq_status decode_step(const kvq_config* cfg, const kvq_cache* cache,
+                              const uint16_t* k_new, const uint16_t* v_new, const uint16_t* q,
+                              void* out, int out_f16, float softmax_scale, int32_t n_splits,
+                              void* workspace, size_t ws_bytes, void* stream) {
+  if (!k_new || !v_new) return fail(KVQ_ERR_ARG, "k_new / v_new is NULL");
+  if (!aligned16(k_new) || !aligned16(v_new))
+    return fail(KVQ_ERR_ALIGN, "k_new / v_new must be 16-byte aligned");
+  float sl2 = 0.0f;
+  kvq_status s = check_attn_call(cfg, cache, q, out, softmax_scale, &n_splits, workspace,
+                                 ws_bytes, &sl2);
+  if (s != KVQ_OK) return s;
+  Dims d = make_dims(*cfg);
+  trace("kvq_decode_step%s batch %d heads %d/%d bits K%dV%d grid (%d, %d, %d) x 512, %d splits",
+        out_f16 ? "" : "_f32", d.batch, d.hq, d.hkv, d.bits_k, d.bits_v, n_splits, d.hkv,
+        d.batch, n_splits);
+  return cuda_status(launch_decode_step(d, *cache, reinterpret_cast<const __half*>(k_new),
+                                        reinterpret_cast<const __half*>(v_new),
+                                        reinterpret_cast<const __half*>(q), out, out_f16, sl2,
+                                        n_splits, workspace, static_cast<cudaStream_t>(stream)),
+                     "kvq_decode_step launch");
+}
+
+}  // namespace kvq
+
+extern "C" {
+
+kvq_status kvq_decode_attn(const kvq_config* cfg, const kvq_cache* cache, const uint16_t* q,
+                           uint16_t* out, float softmax_scale, int32_t n_splits,
+                           void* workspace, size_t ws_bytes, void* stream) {
+  return decode_attn(cfg, cache, q, out, 1, softmax_scale, n_splits, workspace, ws_bytes, stream);
+}
+
+kvq_status kvq_decode_attn_f32(const kvq_config* cfg, const kvq_cache* cache, const uint16_t* q,
+                               float* out, float softmax_scale, int32_t n_splits,
+                               void* workspace, size_t ws_bytes, void* stream) {
+  return decode_attn(cfg, cache, q, out, 0, softmax_scale, n_splits, workspace, ws_bytes, stream);
+}
+
 kvq_status kvq_decode_step(const kvq_config* cfg, const kvq_cache* cache, const uint16_t* k_new,
-                           const uint16_t* v_new, const uint16_t* q, float* out,
+                           const uint16_t* v_new, const uint16_t* q, uint16_t* out,
                            float softmax_scale, int32_t n_splits, void* workspace,
                            size_t ws_bytes, void* stream) {
-  kvq_status s = check_config(cfg);
-  if (s != KVQ_OK) return s;
-  if ((s = check_cache(*cfg, cache)) != KVQ_OK) return s;
-  if (!k_new || !v_new || !q || !out) return fail(KVQ_ERR_ARG, "k_new / v_new / q / out is NULL");
-  if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(q) || !aligned16(out))
-    return fail(KVQ_ERR_ALIGN, "k_new / v_new / q / out must be 16-byte aligned");
-  if (!(softmax_scale >= 0.0f) || isinf(softmax_scale))
-    return fail(KVQ_ERR_ARG, "softmax_scale must be finite and >= 0");
-  if (n_splits == 0) n_splits = default_splits(*cfg);
-  if (n_splits < 1 || n_splits > kMaxSplits - 1)
-    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, n_splits);
-  Dims d = make_dims(*cfg);
-  const size_t need = attn_workspace_bytes(d, n_splits);
-  if (!workspace) return fail(KVQ_ERR_ARG, "workspace is NULL");
-  if (!aligned16(workspace)) return fail(KVQ_ERR_ALIGN, "workspace must be 16-byte aligned");
-  if (ws_bytes < need)
-    return fail(KVQ_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", ws_bytes, need);
-  const float scale = softmax_scale == 0.0f ? 1.0f / sqrtf((float)kHeadDim) : softmax_scale;
-  const float scale_log2 = scale * 1.4426950408889634f;
-  const cudaStream_t st = static_cast<cudaStream_t>(stream);
-  const __half* kn = reinterpret_cast<const __half*>(k_new);
-  const __half* vn = reinterpret_cast<const __half*>(v_new);
-  const __half* qh = reinterpret_cast<const __half*>(q);
-  trace("kvq_decode_step batch %d heads %d/%d bits K%dV%d grid (%d, %d, %d) x 512, %d splits",
-        d.batch, d.hq, d.hkv, d.bits_k, d.bits_v, n_splits, d.hkv * ((d.gq + 3) / 4), d.batch,
-        n_splits);
-  return cuda_status(launch_decode_step(d, *cache, kn, vn, qh, out, scale_log2, n_splits,
-                                        workspace, st),
-                     "kvq_decode_step launch");
+  return decode_step(cfg, cache, k_new, v_new, q, out, 1, softmax_scale, n_splits, workspace,
+                     ws_bytes, stream);
+}
+
+kvq_status kvq_decode_step_f32(const kvq_config* cfg, const kvq_cache* cache,
+                               const uint16_t* k_new, const uint16_t* v_new, const uint16_t* q,
+                               float* out, float softmax_scale, int32_t n_splits,
+                               void* workspace, size_t ws_bytes, void* stream) {
+  return decode_step(cfg, cache, k_new, v_new, q, out, 0, softmax_scale, n_splits, workspace,
+                     ws_bytes, stream);
 }
 
 kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache,

@@ -1058,6 +1058,13 @@ __device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half
   }
 }
 
+// One element of the attention output: the fp32 result, or its fp16
+// rounding to nearest even.
+__device__ __forceinline__ void store_out(void* out, int out_f16, long long i, float v) {
+  if (out_f16) static_cast<__half*>(out)[i] = __float2half_rn(v);
+  else static_cast<float*>(out)[i] = v;
+}
+
 __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
   unsigned old;
   asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
@@ -1070,8 +1077,8 @@ __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
 
 template <int BK, int BV, bool kWide>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
-    decode_attn_kernel(Dims d, kvq_cache c, const __half* __restrict__ q, float* __restrict__ out,
-                       float scale_log2, int S, unsigned smem_size, Ws ws,
+    decode_attn_kernel(Dims d, kvq_cache c, const __half* __restrict__ q, void* __restrict__ out,
+                       int out_f16, float scale_log2, int S, unsigned smem_size, Ws ws,
                        const __half* __restrict__ k_new, const __half* __restrict__ v_new) {
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ MergeSmall ms;
@@ -1245,7 +1252,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       l = fmaf(w, wstate(i).l[g], l);
     }
     if (S == 1) {
-      out[(head0 + g) * kHeadDim + ch] = l > 0.0f ? o / l : 0.0f;
+      store_out(out, out_f16, (head0 + g) * kHeadDim + ch, l > 0.0f ? o / l : 0.0f);
     } else {
       const long long row = (head0 + g) * S + blockIdx.x;
       ws.o[row * kHeadDim + ch] = o;
@@ -1323,7 +1330,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       for (int k = 0; k < S; ++k) o = fmaf(wv[g * S + k], __ldcg(src + (size_t)k * kHeadDim), o);
     }
     const float Ls = lsum[g];
-    out[(head0 + g) * kHeadDim + ch] = Ls > 0.0f ? o / Ls : 0.0f;
+    store_out(out, out_f16, (head0 + g) * kHeadDim + ch, Ls > 0.0f ? o / Ls : 0.0f);
   }
   if (threadIdx.x == 0) ws.tk[bh] = 0u;
 }
@@ -1372,7 +1379,8 @@ struct LaunchOp {
   const Dims& d;
   const kvq_cache& c;
   const __half* q;
-  float* out;
+  void* out;
+  int out_f16;
   float sl2;
   int S;
   const Ws& ws;
@@ -1393,7 +1401,7 @@ struct LaunchOp {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV, kWide>, d, c, q, out, sl2, S,
+    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV, kWide>, d, c, q, out, out_f16, sl2, S,
                            (unsigned)smem_bytes(d), ws, k_new, v_new);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
@@ -1423,26 +1431,28 @@ cudaError_t launch_wait_selftest(unsigned* flag, long long limit_cycles, cudaStr
   return cudaGetLastError();
 }
 
-// n_splits = CTAs per (sequence, kv-head); workspace rows for up to
-// n_splits.  Tickets: one per (sequence, kv-head), sized one per query head.
+// n_splits = CTAs per (sequence, kv-head); partial rows for exactly the
+// n_splits CTAs of the launch (the same carve the kernel uses).  Tickets: one
+// per (sequence, kv-head), sized one per query head.
 size_t attn_workspace_bytes(const Dims& d, int n_splits) {
-  const int S = n_splits + 1;
+  const int S = n_splits;
   const size_t nml = (size_t)d.batch * d.hq * S;
   return align256(nml * 4) * 2 + align256(nml * kHeadDim * 4) +
          align256((size_t)d.batch * d.hq * 4);
 }
 
-cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& c, const __half* q, float* out,
-                               float scale_log2, int n_splits, void* workspace, cudaStream_t st) {
+cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& c, const __half* q, void* out,
+                               int out_f16, float scale_log2, int n_splits, void* workspace,
+                               cudaStream_t st) {
   const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, n_splits);
-  return dispatch(d, LaunchOp{d, c, q, out, scale_log2, n_splits, ws, st});
+  return dispatch(d, LaunchOp{d, c, q, out, out_f16, scale_log2, n_splits, ws, st});
 }
 
 cudaError_t launch_decode_step(const Dims& d, const kvq_cache& c, const __half* k_new,
-                               const __half* v_new, const __half* q, float* out,
+                               const __half* v_new, const __half* q, void* out, int out_f16,
                                float scale_log2, int n_splits, void* workspace, cudaStream_t st) {
   const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, n_splits);
-  LaunchOp op{d, c, q, out, scale_log2, n_splits, ws, st};
+  LaunchOp op{d, c, q, out, out_f16, scale_log2, n_splits, ws, st};
   op.k_new = k_new;
   op.v_new = v_new;
   return dispatch(d, op);
@@ -1561,7 +1571,7 @@ cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& c, const _
   const Ws w = carve(ws, d.batch, d.hq, d.hkv, n_splits);
   e = cudaMemsetAsync(w.tk, 0, (size_t)d.batch * d.hq * sizeof(unsigned), st);
   if (e != cudaSuccess) return e;
-  return launch_decode_attn(d, c, q, out, scale_log2, n_splits, ws, st);
+  return launch_decode_attn(d, c, q, out, 0, scale_log2, n_splits, ws, st);
 }
 
 }  // namespace kvq

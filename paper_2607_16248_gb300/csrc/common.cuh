@@ -133,13 +133,14 @@ void set_error(const char* fmt, ...);
 cudaError_t launch_pack(const Dims& d, const kvq_cache& cache, const __half* k_new,
                         const __half* v_new, int n_new, int batch_begin,
                         int batch_count, cudaStream_t stream);
+// out is fp16 [batch][n_q_heads][128] when out_f16, else fp32.
 cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& cache, const __half* q,
-                               float* out, float scale_log2, int n_splits,
+                               void* out, int out_f16, float scale_log2, int n_splits,
                                void* workspace, cudaStream_t stream);
 // Append one token per sequence (k_new / v_new [batch][n_kv_heads][128]) and
-// attend in the same kernel (query groups up to 4).
+// attend in the same kernel.
 cudaError_t launch_decode_step(const Dims& d, const kvq_cache& cache, const __half* k_new,
-                               const __half* v_new, const __half* q, float* out,
+                               const __half* v_new, const __half* q, void* out, int out_f16,
                                float scale_log2, int n_splits, void* workspace,
                                cudaStream_t stream);
 size_t attn_workspace_bytes(const Dims& d, int n_splits);

@@ -27,7 +27,8 @@ EXPORTS = (
     "kvq_cache_layout", "kvq_cache_bind", "kvq_cache_reset", "kvq_pack",
     "kvq_attn_workspace_bytes", "kvq_attn_default_splits", "kvq_attn_splits_for_lengths",
     "kvq_workspace_init",
-    "kvq_decode_attn", "kvq_decode_step", "kvq_decode_attn_noalloc", "dgap_workspace_bytes",
+    "kvq_decode_attn", "kvq_decode_attn_f32", "kvq_decode_step", "kvq_decode_step_f32",
+    "kvq_decode_attn_noalloc", "dgap_workspace_bytes",
     "dgap_restore", "kvq_drift_max_vocab", "kvq_drift_metrics", "kvq_drift_window",
     "kvq_selftest_wait_timeout",
 )
@@ -88,7 +89,9 @@ def lib():
             "kvq_attn_splits_for_lengths": (I32, [cfg_p, ctypes.POINTER(I32)]),
             "kvq_workspace_init": (I32, [P, SZ, P]),
             "kvq_decode_attn": (I32, [cfg_p, cache_p, P, P, F32, I32, P, SZ, P]),
+            "kvq_decode_attn_f32": (I32, [cfg_p, cache_p, P, P, F32, I32, P, SZ, P]),
             "kvq_decode_step": (I32, [cfg_p, cache_p, P, P, P, P, F32, I32, P, SZ, P]),
+            "kvq_decode_step_f32": (I32, [cfg_p, cache_p, P, P, P, P, F32, I32, P, SZ, P]),
             "kvq_decode_attn_noalloc": (I32, [cfg_p, cache_p, P, P, F32, I32, P]),
             "dgap_workspace_bytes": (SZ, [I32, I32, par_p]),
             "dgap_restore": (I32, [par_p, P, I32, I32, P, P, P, P, P, P, P, SZ, P]),
@@ -263,62 +266,77 @@ def splits_for_lengths(cfg: CacheConfig, lengths):
     return n
 
 
+def _attn_out(q, out, out_dtype):
+    """The output tensor and the entry-point suffix for its dtype."""
+    if out is None:
+        out = torch.empty(q.shape, dtype=out_dtype, device=q.device)
+    if out.dtype == torch.float16:
+        return out, ""
+    if out.dtype == torch.float32:
+        return out, "_f32"
+    raise TypeError(f"out must be float16 or float32, got {out.dtype}")
+
+
 def kvq_decode_attn(cache: QuantKVCache, q, out=None, softmax_scale=0.0, n_splits=0,
-                    workspace=None, stream=None):
-    """out = softmax(q K^T * scale) V over the cache; q fp16 [batch, n_q_heads, 128],
-    out fp32 of the same shape."""
+                    workspace=None, stream=None, out_dtype=torch.float16):
+    """out = softmax(q K^T * scale) V over the cache; q fp16 [batch, n_q_heads, 128].
+
+    out fp16 (the fp32 result rounded to nearest, kvq_decode_attn) or fp32
+    (kvq_decode_attn_f32), picked by the dtype of ``out`` or ``out_dtype``."""
     cfg = cache.cfg
     if q.shape != (cfg.batch, cfg.n_q_heads, cfg.head_dim):
         raise ValueError(f"q must be [{cfg.batch}, {cfg.n_q_heads}, {cfg.head_dim}]")
-    if out is None:
-        out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+    out, suffix = _attn_out(q, out, out_dtype)
+    if out.shape != q.shape:
+        raise ValueError("out must have the shape of q")
     if workspace is None:
         workspace = attn_workspace(cfg, n_splits, q.device)
     c = cfg.c()
-    _check(lib().kvq_decode_attn(ctypes.byref(c), ctypes.byref(cache._c),
-                                 _dev(q, torch.float16, "q"), _dev(out, torch.float32, "out"),
-                                 float(softmax_scale), n_splits,
-                                 _dev(workspace, torch.uint8, "workspace"), workspace.numel(),
-                                 _stream(stream)))
+    fn = getattr(lib(), "kvq_decode_attn" + suffix)
+    _check(fn(ctypes.byref(c), ctypes.byref(cache._c), _dev(q, torch.float16, "q"),
+              _dev(out, out.dtype, "out"), float(softmax_scale), n_splits,
+              _dev(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)))
     return out
 
 
 def kvq_decode_step(cache: QuantKVCache, k_new, v_new, q, out=None, softmax_scale=0.0,
-                    n_splits=0, workspace=None, stream=None):
+                    n_splits=0, workspace=None, stream=None, out_dtype=torch.float16):
     """Append one token per sequence (k_new / v_new fp16 [batch, n_kv_heads, 128])
-    and attend (q fp16 [batch, n_q_heads, 128] -> out fp32) in one call: the
-    same results as kvq_pack then kvq_decode_attn."""
+    and attend (q fp16 [batch, n_q_heads, 128] -> out fp16, or fp32 as in
+    kvq_decode_attn) in one call: the same results as kvq_pack then
+    kvq_decode_attn."""
     cfg = cache.cfg
     if q.shape != (cfg.batch, cfg.n_q_heads, cfg.head_dim):
         raise ValueError(f"q must be [{cfg.batch}, {cfg.n_q_heads}, {cfg.head_dim}]")
     for name, t in (("k_new", k_new), ("v_new", v_new)):
         if t.shape != (cfg.batch, cfg.n_kv_heads, cfg.head_dim):
             raise ValueError(f"{name} must be [{cfg.batch}, {cfg.n_kv_heads}, {cfg.head_dim}]")
-    if out is None:
-        out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+    out, suffix = _attn_out(q, out, out_dtype)
+    if out.shape != q.shape:
+        raise ValueError("out must have the shape of q")
     if workspace is None:
         workspace = attn_workspace(cfg, n_splits, q.device)
     c = cfg.c()
-    _check(lib().kvq_decode_step(ctypes.byref(c), ctypes.byref(cache._c),
-                                 _dev(k_new, torch.float16, "k_new"),
-                                 _dev(v_new, torch.float16, "v_new"),
-                                 _dev(q, torch.float16, "q"), _dev(out, torch.float32, "out"),
-                                 float(softmax_scale), n_splits,
-                                 _dev(workspace, torch.uint8, "workspace"), workspace.numel(),
-                                 _stream(stream)))
+    fn = getattr(lib(), "kvq_decode_step" + suffix)
+    _check(fn(ctypes.byref(c), ctypes.byref(cache._c), _dev(k_new, torch.float16, "k_new"),
+              _dev(v_new, torch.float16, "v_new"), _dev(q, torch.float16, "q"),
+              _dev(out, out.dtype, "out"), float(softmax_scale), n_splits,
+              _dev(workspace, torch.uint8, "workspace"), workspace.numel(), _stream(stream)))
     return out
 
 
-def kvq_decode_attn_noalloc(cache: QuantKVCache, q, out=None, softmax_scale=0.0, n_splits=0,
+def kvq_decode_attn_noalloc(cache: QuantKVCache, q, out, softmax_scale=0.0, n_splits=0,
                             stream=None):
-    """kvq_decode_attn with the library's built-in scratch array instead of a
-    workspace, for callers that cannot allocate device memory per step.  Calls
-    share the array: do not let two of them overlap on the GPU."""
+    """kvq_decode_attn_f32 with the library's built-in scratch array instead of
+    a workspace, for callers that cannot allocate device memory per step.
+    ``out`` (fp32, the shape of q) is required: this wrapper allocates
+    nothing either.  Calls share the array: do not let two of them overlap on
+    the GPU."""
     cfg = cache.cfg
     if q.shape != (cfg.batch, cfg.n_q_heads, cfg.head_dim):
         raise ValueError(f"q must be [{cfg.batch}, {cfg.n_q_heads}, {cfg.head_dim}]")
-    if out is None:
-        out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+    if out is None or out.shape != q.shape:
+        raise ValueError("out must be a preallocated fp32 tensor of q's shape")
     c = cfg.c()
     _check(lib().kvq_decode_attn_noalloc(ctypes.byref(c), ctypes.byref(cache._c),
                                          _dev(q, torch.float16, "q"),

@@ -46,11 +46,9 @@ def _compare(z_in, out, z_after, K, tau, det, cor, require_gate=None):
         assert np.array_equal(z_after[b][mask].view(np.uint32), z_in[b][mask].view(np.uint32))
         # greedy token: the decision in float32 on the oracle's merged values
         zt = z_after[b].astype(np.float32)
-        cand = np.concatenate([ref["val"], [ref["z_K"]]]) if gate[b] else None
         top = np.sort(np.concatenate([zt[idx[b]], [z_in[b][ref["idx_K"]]]]))[::-1]
         if top.size < 2 or top[0] - top[1] > 2 * _util.LOGIT_TOL:
             assert nxt[b] == ref["next_token"]
-        del cand
     if require_gate is not None:
         assert checked_gate >= require_gate
 
@@ -83,8 +81,29 @@ def test_window_sizes(kvq_lib, K):
 
 
 def test_paper_threshold_mixed_rows(kvq_lib):
+    # tau = 0.60 (Sec. 5.5): the seeded rows must all lie outside the band
+    # |f - logit(tau)| <= GATE_BAND, so the gate is compared on every row
     zin, out, zout, det, cor = _run(16, 32768, 32, 0.60, seed=4)
-    _compare(zin, out, zout, 32, 0.60, det, cor)
+    _compare(zin, out, zout, 32, 0.60, det, cor, require_gate=16)
+
+
+@pytest.mark.parametrize("offset", [-4e-4, -2e-4, 2e-4, 4e-4])
+def test_gate_decided_just_outside_the_band(kvq_lib, offset):
+    # tau placed so that one row's detector output f sits |offset| (2 to 4
+    # band widths) from logit(tau): that row's gate must still match the
+    # oracle exactly, on both sides of the threshold (Eq. 13: r > tau)
+    B, V, K = 4, 32768, 32
+    w = synth.dgap_weights(7, K=K)
+    det, cor = synth.split_weights(w)
+    z = synth.logits(71, B, V)
+    f = [odgap.restore_row(r, K, 2.0, det, cor)["f"] for r in z.numpy().astype(np.float64)]
+    lt = f[1] - offset  # row 1 is gated exactly when offset > 0
+    tau = float(1.0 / (1.0 + np.exp(-lt)))
+    assert abs(kvq.logit(tau) - lt) < 1e-9
+    assert all(abs(x - kvq.logit(tau)) > _util.GATE_BAND for x in f)
+    zin, out, zout, det, cor = _run(B, V, K, tau, seed=7, logits=z)
+    assert bool(out["gate"][1].item()) == (offset > 0)
+    _compare(zin, out, zout, K, tau, det, cor, require_gate=B)
 
 
 def test_quantile_threshold_gates_about_thirty_percent(kvq_lib):

@@ -31,9 +31,10 @@ def _steps(cfg, lengths, n_steps, seed, check_oracle_every=0, n_splits=0):
         kn = torch.randn(cfg.batch, cfg.n_kv_heads, 128, generator=g).half()
         vn = torch.randn(cfg.batch, cfg.n_kv_heads, 128, generator=g).half()
         q = torch.randn(cfg.batch, cfg.n_q_heads, 128, generator=g).half()
-        out_a = kvq.kvq_decode_step(a, kn.cuda(), vn.cuda(), q.cuda(), n_splits=n_splits)
+        out_a = kvq.kvq_decode_step(a, kn.cuda(), vn.cuda(), q.cuda(), n_splits=n_splits,
+                                    out_dtype=torch.float32)
         kvq.kvq_pack(b_, kn[:, :, None].cuda(), vn[:, :, None].cuda())
-        out_b = kvq.kvq_decode_attn(b_, q.cuda())
+        out_b = kvq.kvq_decode_attn(b_, q.cuda(), out_dtype=torch.float32)
         torch.cuda.synchronize()
         oa, ob = out_a.cpu().numpy(), out_b.cpu().numpy()
         for s in range(cfg.batch):

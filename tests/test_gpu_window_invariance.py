@@ -17,7 +17,7 @@ def test_window_token_permutation_invariance(kvq_lib):
     lengths = [300, 150]  # 140 window tokens after 160 packed; an all-window sequence
     cache, _ = _util.make_cache(cfg, lengths, 62)
     q = synth.queries(63, cfg.batch, cfg.n_q_heads).cuda()
-    before = kvq.kvq_decode_attn(cache, q).float().cpu().numpy()
+    before = kvq.kvq_decode_attn(cache, q, out_dtype=torch.float32).cpu().numpy()
     kr, vr = cache.resid()  # views of the cache's fp16 rings
     g = torch.Generator().manual_seed(64)
     for b, L in enumerate(lengths):
@@ -28,6 +28,6 @@ def test_window_token_permutation_invariance(kvq_lib):
         kr[b, :, slots] = kr[b, :, perm]
         vr[b, :, slots] = vr[b, :, perm]
     torch.cuda.synchronize()
-    after = kvq.kvq_decode_attn(cache, q).float().cpu().numpy()
+    after = kvq.kvq_decode_attn(cache, q, out_dtype=torch.float32).cpu().numpy()
     rms = np.sqrt((before ** 2).mean(axis=-1))
     assert (np.abs(after - before).max(axis=-1) / rms).max() <= 1e-4
