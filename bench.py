@@ -65,6 +65,8 @@ def parse():
     p.add_argument("--layers", type=int, default=0, help="override the layer count")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--paged", action="store_true",
+                   help="run the caches on the paged layout (block table, shuffled pool)")
     p.add_argument("--cpu-worker", default="", help=argparse.SUPPRESS)
     return p.parse_args()
 
@@ -85,6 +87,8 @@ def workload_spec(args):
         spec["bits"] = args.bits
     if args.layers:
         spec["layers"] = args.layers
+    if getattr(args, "paged", False):
+        spec["paged"] = True
     return spec
 
 
@@ -404,8 +408,25 @@ class Step:
         self.cfg = kvq.CacheConfig(batch=B, n_q_heads=hq, n_kv_heads=hkv, bits_k=b, bits_v=b,
                                    max_len=max_len)
         self.caches = []
+        self.paged_pages = None
         for l in range(layers):
-            cache = kvq.QuantKVCache(self.cfg, device)
+            if spec.get("paged"):
+                # a pool holding exactly the blocks each sequence reaches in
+                # this run (prefill + every replayed step), mapped in a seeded
+                # shuffled order before the prefill, so the steps' flushes
+                # land in pages the caller assigned
+                need = [packed_len(L + steps_total + 1) // 32 for L in self.lengths0]
+                n_pages = max(1, sum(need))
+                cache = kvq.QuantKVCache(self.cfg, device, n_pages=n_pages)
+                perm = torch.randperm(n_pages, generator=synth.generator(seed + 31 * l)).tolist()
+                at = 0
+                for s_, nb in enumerate(need):
+                    if nb:
+                        cache.map_blocks(s_, range(nb), perm[at:at + nb])
+                    at += nb
+                self.paged_pages = n_pages
+            else:
+                cache = kvq.QuantKVCache(self.cfg, device)
             for s, L in enumerate(self.lengths0):
                 k, v = synth.kv_heads(seed * 100003 + l * 1009 + s, hkv, L, device=device)
                 kvq.kvq_pack(cache, k[None], v[None], batch_begin=s)
@@ -614,6 +635,8 @@ def run_gpu(args, spec):
            "layers": s["layers"], "vocab": s["vocab"], "residual": 128, "group": 32,
            "dgap_K": DGAP_K, "dgap_hidden": DGAP_HIDDEN, "tau": round(st.dgap.tau, 6),
            "n_splits": st.n_splits,
+           "kv_layout": (f"paged: block table over a shuffled pool of {st.paged_pages} page sets "
+                         f"per layer" if st.paged_pages else "contiguous pages per sequence"),
            "l2": f"inputs larger than L2: {step_bytes[0] / 1e6:.0f} MB of packed KV read per "
                  f"step (distinct cache per layer), L2 129 MB",
            "step": f"{s['layers']} x kvq_decode_step (append + attention) + logits copy + "
@@ -684,17 +707,20 @@ def single_layer_times(st, device, reps=50, warm=5):
 
     res = {}
     for mode in ("warm", "cold"):
-        times = []
-        for i in range(warm + reps):
+        # a device-side wait first, so that every repetition is queued before
+        # the GPU reaches it and the events see no host launch latency
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(warm + reps)]
+        torch.cuda.synchronize()
+        torch.cuda._sleep(20_000_000)
+        for i, (a, b) in enumerate(evs):
             if mode == "cold":
                 flush.fill_(float(i))
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record()
             one()
             b.record()
-            b.synchronize()
-            if i >= warm:
-                times.append(a.elapsed_time(b) * 1e3)
+        torch.cuda.synchronize()
+        times = [a.elapsed_time(b) * 1e3 for a, b in evs[warm:]]
         res[f"{mode}_us_median"] = round(statistics.median(times), 3)
         res[f"{mode}_us_p95"] = round(percentile(times, 95.0), 3)
     res["reps"] = reps

@@ -51,6 +51,10 @@ typedef enum kvq_status {
 #define KVQ_FLAG_OVERFLOW 1u /* an append would have passed max_len */
 #define KVQ_FLAG_WAIT_TIMEOUT 2u /* an attention kernel's copy wait gave up (~2 s);
                                     its output for that call is not valid */
+#define KVQ_FLAG_BAD_PAGE 4u /* a paged cache's block table mapped a block that a
+                                call had to read or write outside [0, n_pages):
+                                the write was skipped, and an output that needed
+                                the block is not valid */
 
 /*
  * Cache configuration.  KbVb with b_k = bits_k and b_v = bits_v (Sec. 3.1
@@ -117,7 +121,32 @@ typedef struct kvq_cache {
   uint16_t* k_resid;
   uint16_t* v_resid;
   int32_t* seq_len;
+  const int32_t* block_table; /* NULL: the contiguous page layout above */
+  int32_t n_pages;            /* page sets in the pool (paged layout only) */
 } kvq_cache;
+
+/*
+ * Paged layout (block_table != NULL; Sec. 3.1's 32-token groups as the unit
+ * of a shared page pool, for ragged batches that should not reserve max_len
+ * per sequence):
+ *   pages        device pool [n_pages][n_kv_heads][page_bytes]: one page set
+ *                holds one 32-token block of one sequence for every kv-head;
+ *                16-byte aligned.
+ *   block_table  device int32 [batch][max_len / 32]: entry (b, j) is the page
+ *                set of block j (tokens [32 j, 32 j + 32)) of sequence b.
+ *   n_pages      1 .. 2^31 - 1.
+ * The caller owns both and assigns the entries: every block a call reads
+ * (j < Lq / 32) or writes must be mapped to a page set in [0, n_pages) before
+ * the call is enqueued, and distinct blocks of live sequences must map to
+ * distinct page sets.  kvq_pack of n_new tokens writes blocks
+ * [Lq(L) / 32, Lq(L + n_new) / 32); a kvq_decode_step from L to L + 1 tokens
+ * writes block Lq(L + 1) / 32 - 1 exactly when Lq(L + 1) > Lq(L), i.e. when
+ * L + 1 - R is a positive multiple of 32 (Lq as above; the caller knows the
+ * lengths).  An entry of a block that holds data must not change while a
+ * call that may read it is in flight.  A block mapped outside [0, n_pages)
+ * is never dereferenced: the kernel skips it and sets KVQ_FLAG_BAD_PAGE.
+ * The fp16 window and seq_len keep the layout above (kvq_paged_cache_layout).
+ */
 
 /* Thread-local description of the last failure ("" after success). */
 const char* kvq_last_error(void);
@@ -140,8 +169,30 @@ kvq_status kvq_cache_layout(const kvq_config* cfg, size_t* total_bytes,
                             size_t offsets[4]);
 
 /* Host-only: fill *cache with pointers into `base` (device, >= total_bytes,
- * 256-byte aligned) following kvq_cache_layout. */
+ * 256-byte aligned) following kvq_cache_layout (contiguous pages;
+ * block_table = NULL, n_pages = 0). */
 kvq_status kvq_cache_bind(const kvq_config* cfg, void* base, kvq_cache* cache);
+
+/* Host-only: bytes of a page pool of n_pages page sets (0 if invalid). */
+size_t kvq_page_pool_bytes(const kvq_config* cfg, int32_t n_pages);
+
+/*
+ * Host-only layout query of a paged cache: the fp16 rings and seq_len only
+ * (the pages live in the caller's pool).  offsets[0] is 0 and the page
+ * region is empty; offsets[1..3] as in kvq_cache_layout.
+ */
+kvq_status kvq_paged_cache_layout(const kvq_config* cfg, size_t* total_bytes,
+                                  size_t offsets[4]);
+
+/*
+ * Host-only: a paged cache.  `base` (device, >= the paged total, 256-byte
+ * aligned) holds the rings and seq_len; `pool` (device, 16-byte aligned,
+ * >= kvq_page_pool_bytes(cfg, n_pages)) the page sets; `block_table` (device
+ * int32 [batch][max_len / 32]) the caller's mapping (see the paged layout).
+ */
+kvq_status kvq_paged_cache_bind(const kvq_config* cfg, void* base, void* pool,
+                                int32_t n_pages, const int32_t* block_table,
+                                kvq_cache* cache);
 
 /* Empty every sequence: zero seq_len, the flag word and the tickets. */
 kvq_status kvq_cache_reset(const kvq_config* cfg, const kvq_cache* cache,

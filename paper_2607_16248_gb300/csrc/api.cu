@@ -91,10 +91,12 @@ struct Layout {
   size_t pages, k_resid, v_resid, seq, total;
 };
 
-static Layout layout_of(const kvq_config& c) {
+// paged: the page region is empty (the pages live in the caller's pool).
+static Layout layout_of(const kvq_config& c, bool paged = false) {
   Layout l;
   const size_t bh = (size_t)c.batch * c.n_kv_heads;
-  const size_t pages = bh * (size_t)(c.max_len / kGroup) * page_bytes(c.bits_k, c.bits_v);
+  const size_t pages =
+      paged ? 0 : bh * (size_t)(c.max_len / kGroup) * page_bytes(c.bits_k, c.bits_v);
   const size_t resid = bh * (size_t)(c.residual + kGroup) * kHeadDim * sizeof(__half);
   const size_t seq = (size_t)(c.batch + 2) * 4 + (size_t)c.batch * 4;
   l.pages = 0;
@@ -116,6 +118,11 @@ static kvq_status check_cache(const kvq_config& c, const kvq_cache* cache) {
   if (!aligned16(cache->pages) || !aligned16(cache->k_resid) || !aligned16(cache->v_resid) ||
       (reinterpret_cast<uintptr_t>(cache->seq_len) & 3u))
     return fail(KVQ_ERR_ALIGN, "cache pointers must be 16-byte aligned");
+  if (cache->block_table) {
+    if (reinterpret_cast<uintptr_t>(cache->block_table) & 3u)
+      return fail(KVQ_ERR_ALIGN, "block_table must be 4-byte aligned");
+    if (cache->n_pages < 1) return fail(KVQ_ERR_ARG, "a paged cache needs n_pages >= 1");
+  }
   (void)c;
   return KVQ_OK;
 }
@@ -180,6 +187,54 @@ kvq_status kvq_cache_bind(const kvq_config* cfg, void* base, kvq_cache* cache) {
   cache->k_resid = reinterpret_cast<uint16_t*>(p + l.k_resid);
   cache->v_resid = reinterpret_cast<uint16_t*>(p + l.v_resid);
   cache->seq_len = reinterpret_cast<int32_t*>(p + l.seq);
+  cache->block_table = nullptr;
+  cache->n_pages = 0;
+  return KVQ_OK;
+}
+
+size_t kvq_page_pool_bytes(const kvq_config* cfg, int32_t n_pages) {
+  if (check_config(cfg) != KVQ_OK) return 0;
+  if (n_pages < 1) {
+    set_error("n_pages must be >= 1 (got %d)", n_pages);
+    return 0;
+  }
+  return (size_t)n_pages * cfg->n_kv_heads * page_bytes(cfg->bits_k, cfg->bits_v);
+}
+
+kvq_status kvq_paged_cache_layout(const kvq_config* cfg, size_t* total_bytes,
+                                  size_t offsets[4]) {
+  kvq_status s = check_config(cfg);
+  if (s != KVQ_OK) return s;
+  if (!total_bytes || !offsets) return fail(KVQ_ERR_ARG, "output pointer is NULL");
+  Layout l = layout_of(*cfg, true);
+  *total_bytes = l.total;
+  offsets[0] = l.pages;
+  offsets[1] = l.k_resid;
+  offsets[2] = l.v_resid;
+  offsets[3] = l.seq;
+  return KVQ_OK;
+}
+
+kvq_status kvq_paged_cache_bind(const kvq_config* cfg, void* base, void* pool, int32_t n_pages,
+                                const int32_t* block_table, kvq_cache* cache) {
+  kvq_status s = check_config(cfg);
+  if (s != KVQ_OK) return s;
+  if (!base || !pool || !block_table || !cache)
+    return fail(KVQ_ERR_ARG, "base, pool, block_table or cache is NULL");
+  if (reinterpret_cast<uintptr_t>(base) & 255u)
+    return fail(KVQ_ERR_ALIGN, "cache buffer must be 256-byte aligned");
+  if (!aligned16(pool)) return fail(KVQ_ERR_ALIGN, "page pool must be 16-byte aligned");
+  if (reinterpret_cast<uintptr_t>(block_table) & 3u)
+    return fail(KVQ_ERR_ALIGN, "block_table must be 4-byte aligned");
+  if (n_pages < 1) return fail(KVQ_ERR_ARG, "n_pages must be >= 1 (got %d)", n_pages);
+  Layout l = layout_of(*cfg, true);
+  char* p = static_cast<char*>(base);
+  cache->pages = pool;
+  cache->k_resid = reinterpret_cast<uint16_t*>(p + l.k_resid);
+  cache->v_resid = reinterpret_cast<uint16_t*>(p + l.v_resid);
+  cache->seq_len = reinterpret_cast<int32_t*>(p + l.seq);
+  cache->block_table = block_table;
+  cache->n_pages = n_pages;
   return KVQ_OK;
 }
 

@@ -768,22 +768,74 @@ __host__ __device__ constexpr int image_bytes(int page) { return (page + 127) / 
 // a length read before the wait gives (tc_pre_issue), up to the block before
 // the newest.  If the range after the wait does not begin with exactly those
 // slots they are consumed without use.
+// A warp's window of 32 consecutive block-table entries (paged caches): lane
+// i holds the entry of block wb + i, refreshed (one coalesced load) when a
+// lookup leaves it.  Lookups are warp-uniform and made by all lanes.
+struct TableWin {
+  int wb, v;
+};
+__device__ __forceinline__ void table_win_init(TableWin& w) {
+  w.wb = -(1 << 30);
+  w.v = -1;
+}
+__device__ __forceinline__ const char* block_addr(const PageMap& pm, TableWin& w, int j) {
+  if (!pm.paged()) return pm.base + (long long)j * pm.page;
+  if (j < w.wb || j >= w.wb + 32) {
+    w.wb = j;
+    const int k = j + (int)(threadIdx.x & 31);
+    w.v = k < pm.max_blocks ? __ldg(pm.row + k) : -1;
+  }
+  return pm.at(j, __shfl_sync(0xffffffffu, w.v, j - w.wb));
+}
+
+// Slot s of the ring: blocks [first, first + nblk) (nblk <= blocks per
+// slot).  Called by all lanes; lane 0 issues.  Contiguous pages come in one
+// bulk copy, paged ones in one copy per page; a block mapped outside the
+// pool is not copied (KVQ_FLAG_BAD_PAGE; its slot bytes are stale and the
+// call's output is flagged invalid) and the barrier expects only the bytes
+// copied.  `fence`: the warp's reads of the slot precede the copies that
+// overwrite it.
 template <int BK, int BV>
-__device__ __forceinline__ void issue_slot(const char* pages_bh, char* ring, uint64_t* full, int R,
-                                           int s, int first, int nblk) {
+__device__ __forceinline__ void issue_slot(const PageMap& pm, TableWin& tw, char* ring,
+                                           uint64_t* full, int R, int s, int first, int nblk,
+                                           unsigned* flag, bool fence) {
   constexpr int page = page_bytes_c(BK, BV);
   constexpr int NB = ring_blocks(page);
+  const bool lead = (threadIdx.x & 31) == 0;
   uint64_t* bar = full + s % R;
-  const uint32_t bytes = (uint32_t)(nblk * page);
-  mbar_expect_tx(bar, bytes);
-  bulk_g2s(ring + (size_t)(s % R) * NB * page, pages_bh + (long long)first * page, bytes, bar);
+  char* dst = ring + (size_t)(s % R) * NB * page;
+  if (!pm.paged()) {
+    if (lead) {
+      if (fence) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      const uint32_t bytes = (uint32_t)(nblk * page);
+      mbar_expect_tx(bar, bytes);
+      bulk_g2s(dst, pm.base + (long long)first * page, bytes, bar);
+    }
+    return;
+  }
+  const char* src[NB];
+  uint32_t bytes = 0;
+#pragma unroll
+  for (int i = 0; i < NB; ++i) {
+    src[i] = i < nblk ? block_addr(pm, tw, first + i) : nullptr;
+    if (src[i]) bytes += page;
+  }
+  if (lead) {
+    if (fence) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    if (bytes < (uint32_t)(nblk * page)) atomicOr(flag, (unsigned)KVQ_FLAG_BAD_PAGE);
+    mbar_expect_tx(bar, bytes);
+#pragma unroll
+    for (int i = 0; i < NB; ++i)
+      if (src[i]) bulk_g2s(dst + i * page, src[i], page, bar);
+  }
 }
 
 // Units (slots) of the range [lo_h, hi_h) that end at or before hi_safe:
 // streams them, returns their count and in `end` the block after them.
 template <int BK, int BV>
-__device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int hi_h, int hi_safe,
-                                            char* ring, uint64_t* full, int R, int& end) {
+__device__ __forceinline__ int tc_pre_issue(const PageMap& pm, TableWin& tw, int lo_h, int hi_h,
+                                            int hi_safe, char* ring, uint64_t* full, int R,
+                                            int& end, unsigned* flag) {
   constexpr int NB = ring_blocks(page_bytes_c(BK, BV));
   int n = 0;
   end = lo_h;
@@ -791,7 +843,7 @@ __device__ __forceinline__ int tc_pre_issue(const char* pages_bh, int lo_h, int 
     const int b0 = lo_h + n * NB;
     const int nblk = min(NB, hi_h - b0);
     if (nblk <= 0 || b0 + nblk > hi_safe) break;
-    if ((threadIdx.x & 31) == 0) issue_slot<BK, BV>(pages_bh, ring, full, R, n, b0, nblk);
+    issue_slot<BK, BV>(pm, tw, ring, full, R, n, b0, nblk, flag, false);
     end = b0 + nblk;
   }
   return n;
@@ -903,12 +955,14 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
 
 // Fold blocks [lo, hi) into st; `pre` slots holding blocks [lo_h, pre_end)
 // were streamed early.
+// Fold blocks [lo, hi) into st; `pre` slots holding blocks [lo_h, pre_end)
+// were streamed early.
 template <int BK, int BV, bool kWide>
-__device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_end, int lo, int hi_all,
-                               char* ring, uint64_t* full, int R, const char* zero,
-                               const __half* qh, int gq, float scale_log2, unsigned* flag,
-                               TcState& st, int flush_blk,
-                               uint64_t* fl_bar, char* image) {
+__device__ void tc_packed_warp(const PageMap& pm, TableWin& tw, int lo_h, int pre, int pre_end,
+                               int lo, int hi_all, char* ring, uint64_t* full, int R,
+                               const char* zero, const __half* qh, int gq, float scale_log2,
+                               unsigned* flag, TcState& st, int flush_blk, uint64_t* fl_bar,
+                               char* image) {
   constexpr int page = page_bytes_c(BK, BV);
   constexpr int NB = ring_blocks(page);
   const int lane = threadIdx.x & 31;
@@ -922,14 +976,14 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
   const int skip = reuse ? 0 : pre;
   const int n_units = (hi - lo + NB - 1) / NB;
   const int total = skip + n_units;
-  int issued = pre;  // lane 0's count of issued slots
-  auto real_issue = [&](int s) {
+  int issued = pre;  // slots issued so far
+  auto real_issue = [&](int s, bool fence) {
     const int u = s - skip;
-    issue_slot<BK, BV>(pages_bh, ring, full, R, s, lo + u * NB, min(NB, hi - lo - u * NB));
+    issue_slot<BK, BV>(pm, tw, ring, full, R, s, lo + u * NB, min(NB, hi - lo - u * NB), flag,
+                       fence);
     issued = s + 1;
   };
-  if (lane == 0)
-    for (int s = pre; s < min(total, R); ++s) real_issue(s);
+  for (int s = pre; s < min(total, R); ++s) real_issue(s, false);
 
   const Lane ln = make_lane<BK, BV>(lane);
   uint32_t qb[16];
@@ -957,11 +1011,7 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
       }
     }
     __syncwarp();
-    if (lane == 0 && s + R < total) {
-      // this warp's reads of the slot precede the copy that overwrites it
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      real_issue(s + R);
-    }
+    if (s + R < total) real_issue(s + R, true);
   }
   // Copies issued but not consumed (a wait gave up, or the range shrank) land
   // before the ring is reused; bounded waits.
@@ -970,10 +1020,14 @@ __device__ void tc_packed_warp(const char* pages_bh, int lo_h, int pre, int pre_
   __syncwarp();
   if (flush) {
     // the page image is complete once its four quarters have arrived
+    char* dst = const_cast<char*>(block_addr(pm, tw, flush_blk));
     if (__all_sync(0xffffffffu, mbar_wait(fl_bar, 0u))) {
-      uint4* dst =
-          reinterpret_cast<uint4*>(const_cast<char*>(pages_bh) + (long long)flush_blk * page);
-      for (int i = lane; i < page / 16; i += 32) dst[i] = reinterpret_cast<const uint4*>(image)[i];
+      if (dst) {
+        uint4* d4 = reinterpret_cast<uint4*>(dst);
+        for (int i = lane; i < page / 16; i += 32) d4[i] = reinterpret_cast<const uint4*>(image)[i];
+      } else if (lane == 0) {
+        atomicOr(flag, (unsigned)KVQ_FLAG_BAD_PAGE);
+      }
       const char* pg[1] = {image};
       tc_unit<BK, BV, 1, kWide>(pg, zero, qb, ln, scale_log2, st);
     } else if (lane == 0) {
@@ -1094,7 +1148,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   const int v = blockIdx.x * kWarps + warp;
   pdl_launch_dependents();
   const long long bh = (long long)b * d.hkv + h;
-  const char* pages = static_cast<const char*>(c.pages) + bh * d.max_blocks * d.page_bytes;
+  const PageMap pm = page_map(d, c, b, h);
+  TableWin tw;
+  table_win_init(tw);
   const __half* ring_k = reinterpret_cast<const __half*>(c.k_resid) + bh * d.ring * kHeadDim;
   const __half* ring_v = reinterpret_cast<const __half*>(c.v_resid) + bh * d.ring * kHeadDim;
   const long long head0 = (long long)b * d.hq + (long long)h * gq;
@@ -1132,7 +1188,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     if (v < ph.np) {
       block_range(ph, v, lo_h, hi_h);
       // the newest block may be the one the previous kernel is writing
-      pre = tc_pre_issue<BK, BV>(pages, lo_h, hi_h, ph.nb - 1, ring, full, R, pre_end);
+      pre = tc_pre_issue<BK, BV>(pm, tw, lo_h, hi_h, ph.nb - 1, ring, full, R, pre_end, flag);
       // a decode step that pushes a group out of the window: its owner brings
       // the group's ring rows (old, unchanging) into L2 for the flush
       if (append && lane == 0 && hi_h == ph.nb && ph.nb > 0 &&
@@ -1212,7 +1268,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         lo = hi = 0;
         if (packed) block_range(p, v, lo, hi);
       }
-      tc_packed_warp<BK, BV, kWide>(pages, lo_h, pre, pre_end, lo, hi, ring, full, R,
+      tc_packed_warp<BK, BV, kWide>(pm, tw, lo_h, pre, pre_end, lo, hi, ring, full, R,
                              reinterpret_cast<const char*>(zero), q_s, gq, scale_log2, flag, st,
                              flush_blk, &fl_bar, image);
     }

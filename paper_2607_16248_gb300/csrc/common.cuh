@@ -126,6 +126,45 @@ inline Dims make_dims(const kvq_config& c) {
   return d;
 }
 
+// Pages of one (sequence b, kv-head h).  Contiguous layout: block j at
+// base + j * page_bytes.  Paged layout (kvq.h): block j in page set
+// row[j] of the pool, at base + row[j] * set_bytes with base = pool + h *
+// page_bytes; an entry outside [0, n_pages) maps to no page.
+struct PageMap {
+  char* base;
+  const int32_t* row;  // nullptr: contiguous
+  long long page, set_bytes;
+  int n_pages, max_blocks;
+  __device__ __forceinline__ bool paged() const { return row != nullptr; }
+  // address of block j given its table entry (ignored when contiguous);
+  // nullptr when the entry is outside the pool
+  __device__ __forceinline__ char* at(int j, int entry) const {
+    if (!row) return base + (long long)j * page;
+    return (entry >= 0 && entry < n_pages) ? base + (long long)entry * set_bytes : nullptr;
+  }
+  // address of block j, reading its table entry (single-thread use)
+  __device__ __forceinline__ char* at(int j) const {
+    return at(j, row ? (j < max_blocks ? row[j] : -1) : 0);
+  }
+};
+
+__device__ __forceinline__ PageMap page_map(const Dims& d, const kvq_cache& c, int b, int h) {
+  PageMap m;
+  m.page = d.page_bytes;
+  m.max_blocks = d.max_blocks;
+  m.n_pages = c.n_pages;
+  if (c.block_table) {
+    m.row = c.block_table + (long long)b * d.max_blocks;
+    m.base = static_cast<char*>(c.pages) + (long long)h * d.page_bytes;
+    m.set_bytes = (long long)d.hkv * d.page_bytes;
+  } else {
+    m.row = nullptr;
+    m.base = static_cast<char*>(c.pages) + ((long long)b * d.hkv + h) * d.max_blocks * d.page_bytes;
+    m.set_bytes = 0;
+  }
+  return m;
+}
+
 // Thread-local error message (api.cu).
 void set_error(const char* fmt, ...);
 

@@ -118,8 +118,14 @@ __device__ __forceinline__ void pdl_enter() {
   asm volatile("griddepcontrol.launch_dependents;\ngriddepcontrol.wait;" ::: "memory");
 }
 
-__device__ __forceinline__ char* page_ptr(const Dims& d, void* pages, int b, int h, int j) {
-  return static_cast<char*>(pages) + (((long long)b * d.hkv + h) * d.max_blocks + j) * d.page_bytes;
+// Page of block j of (b, h), or nullptr when a paged cache maps it outside
+// the pool (then KVQ_FLAG_BAD_PAGE is set and the block is not written).
+// Uniform over the CTA.
+__device__ __forceinline__ char* page_ptr(const Dims& d, const kvq_cache& c, int b, int h, int j) {
+  char* p = page_map(d, c, b, h).at(j);
+  if (!p && threadIdx.x == 0)
+    atomicOr(reinterpret_cast<unsigned*>(c.seq_len) + d.batch, (unsigned)KVQ_FLAG_BAD_PAGE);
+  return p;
 }
 
 // Source row (128 fp16) of absolute token p of (b, h): the ring for p < L0,
@@ -180,10 +186,12 @@ __global__ void __launch_bounds__(kPackThreads)
   const int first = max(packed_len(L0, d.residual), ((L0 + kGroup - 1) / kGroup) * kGroup) / kGroup;
   const int j = first + blockIdx.x;
   if (j >= packed_len(L1, d.residual) / kGroup) return;
+  char* page = page_ptr(d, c, b, h, j);
+  if (!page) return;
   const RowSrc src = make_src(d, c, k_new, v_new, n_new, b, bi, h, L0);
   load_tile(tile, src, j);
   __syncthreads();
-  quantize_tile(tile, page_ptr(d, c.pages, b, h, j), d.bits_k, d.bits_v);
+  quantize_tile(tile, page, d.bits_k, d.bits_v);
 }
 
 // Blocks that touch the ring, the ring append, and the length update.
@@ -207,9 +215,11 @@ __global__ void __launch_bounds__(kPackThreads)
   // 1. Groups leaving the window that start below L0 (they read the ring).
   const int j_end = min(Lq1, ((L0 + kGroup - 1) / kGroup) * kGroup) / kGroup;
   for (int j = Lq0 / kGroup; j < j_end; ++j) {
+    char* page = page_ptr(d, c, b, h, j);
+    if (!page) continue;
     load_tile(tile, src, j);
     __syncthreads();
-    quantize_tile(tile, page_ptr(d, c.pages, b, h, j), d.bits_k, d.bits_v);
+    quantize_tile(tile, page, d.bits_k, d.bits_v);
     __syncthreads();
   }
 

@@ -20,11 +20,13 @@ STATUS_NAMES = {0: "KVQ_OK", 1: "KVQ_ERR_ARG", 2: "KVQ_ERR_SHAPE", 3: "KVQ_ERR_U
                 4: "KVQ_ERR_CAPACITY", 5: "KVQ_ERR_ALIGN", 6: "KVQ_ERR_CUDA"}
 FLAG_OVERFLOW = 1
 FLAG_WAIT_TIMEOUT = 2
+FLAG_BAD_PAGE = 4
 
 # Every symbol include/kvq.h declares.
 EXPORTS = (
     "kvq_last_error", "kvq_version", "kvq_validate_config", "kvq_page_bytes",
     "kvq_cache_layout", "kvq_cache_bind", "kvq_cache_reset", "kvq_pack",
+    "kvq_page_pool_bytes", "kvq_paged_cache_layout", "kvq_paged_cache_bind",
     "kvq_attn_workspace_bytes", "kvq_attn_default_splits", "kvq_attn_splits_for_lengths",
     "kvq_workspace_init",
     "kvq_decode_attn", "kvq_decode_attn_f32", "kvq_decode_step", "kvq_decode_step_f32",
@@ -49,7 +51,8 @@ class _Config(ctypes.Structure):
 
 class _Cache(ctypes.Structure):
     _fields_ = [("pages", ctypes.c_void_p), ("k_resid", ctypes.c_void_p),
-                ("v_resid", ctypes.c_void_p), ("seq_len", ctypes.c_void_p)]
+                ("v_resid", ctypes.c_void_p), ("seq_len", ctypes.c_void_p),
+                ("block_table", ctypes.c_void_p), ("n_pages", ctypes.c_int32)]
 
 
 class _DriftParams(ctypes.Structure):
@@ -82,6 +85,10 @@ def lib():
             "kvq_page_bytes": (SZ, [cfg_p]),
             "kvq_cache_layout": (I32, [cfg_p, ctypes.POINTER(SZ), ctypes.POINTER(SZ * 4)]),
             "kvq_cache_bind": (I32, [cfg_p, P, cache_p]),
+            "kvq_page_pool_bytes": (SZ, [cfg_p, I32]),
+            "kvq_paged_cache_layout": (I32, [cfg_p, ctypes.POINTER(SZ),
+                                             ctypes.POINTER(SZ * 4)]),
+            "kvq_paged_cache_bind": (I32, [cfg_p, P, P, I32, P, cache_p]),
             "kvq_cache_reset": (I32, [cfg_p, cache_p, P]),
             "kvq_pack": (I32, [cfg_p, cache_p, P, P, I32, I32, I32, P]),
             "kvq_attn_workspace_bytes": (SZ, [cfg_p, I32]),
@@ -185,19 +192,61 @@ def packed_len(L, residual=128, group=32):
 
 
 class QuantKVCache:
-    """A KbVb cache in one device buffer, bound through kvq_cache_bind."""
+    """A KbVb cache bound through the C ABI.
 
-    def __init__(self, cfg: CacheConfig, device="cuda"):
+    Contiguous (``n_pages=None``): one device buffer from kvq_cache_layout.
+    Paged (``n_pages=N``): the fp16 rings and lengths in one buffer
+    (kvq_paged_cache_layout), a pool of N page sets and a device block table
+    [batch, max_len / 32] of int32 (all -1, i.e. unmapped, at first); the
+    caller maps blocks with ``map_blocks`` before a call writes or reads them.
+    """
+
+    def __init__(self, cfg: CacheConfig, device="cuda", n_pages=None):
         self.cfg = cfg
-        total, self.offsets = cfg.layout()
+        self.n_pages = n_pages
+        c = cfg.c()
+        if n_pages is None:
+            total, self.offsets = cfg.layout()
+        else:
+            tot = ctypes.c_size_t()
+            offs = (ctypes.c_size_t * 4)()
+            _check(lib().kvq_paged_cache_layout(ctypes.byref(c), ctypes.byref(tot),
+                                                ctypes.byref(offs)))
+            total, self.offsets = tot.value, tuple(offs)
         self._raw = torch.empty(total + 256, dtype=torch.uint8, device=device)
         shift = (-self._raw.data_ptr()) % 256
         self.buffer = self._raw[shift:shift + total]
         self._c = _Cache()
-        c = cfg.c()
-        _check(lib().kvq_cache_bind(ctypes.byref(c), ctypes.c_void_p(self.buffer.data_ptr()),
-                                    ctypes.byref(self._c)))
+        if n_pages is None:
+            self.pool = None
+            self.block_table = None
+            _check(lib().kvq_cache_bind(ctypes.byref(c), ctypes.c_void_p(self.buffer.data_ptr()),
+                                        ctypes.byref(self._c)))
+        else:
+            nbytes = lib().kvq_page_pool_bytes(ctypes.byref(c), int(n_pages))
+            if nbytes == 0:
+                raise KvqError(1, last_error())
+            self.pool = torch.zeros(nbytes, dtype=torch.uint8, device=device)
+            self.block_table = torch.full((cfg.batch, cfg.max_blocks), -1, dtype=torch.int32,
+                                          device=device)
+            _check(lib().kvq_paged_cache_bind(
+                ctypes.byref(c), ctypes.c_void_p(self.buffer.data_ptr()),
+                ctypes.c_void_p(self.pool.data_ptr()), int(n_pages),
+                ctypes.c_void_p(self.block_table.data_ptr()), ctypes.byref(self._c)))
         self.reset()
+
+    @property
+    def paged(self):
+        return self.n_pages is not None
+
+    def map_blocks(self, b, blocks, page_sets):
+        """Paged caches: block_table[b, blocks[i]] = page_sets[i] (a copy to
+        the device on the current stream)."""
+        if not self.paged:
+            raise ValueError("map_blocks needs a paged cache")
+        idx = torch.as_tensor(list(blocks), dtype=torch.long)
+        val = torch.as_tensor(list(page_sets), dtype=torch.int32)
+        self.block_table[b, idx.to(self.block_table.device)] = val.to(self.block_table.device)
 
     def reset(self, stream=None):
         c = self.cfg.c()
@@ -205,11 +254,28 @@ class QuantKVCache:
 
     # Views of the raw storage (layout of include/kvq.h).
     def pages(self):
+        """Contiguous caches: the page array [batch, n_kv_heads, max_blocks,
+        page_bytes]."""
         cfg = self.cfg
+        if self.paged:
+            raise ValueError("a paged cache has no page array: use head_pages")
         n = cfg.batch * cfg.n_kv_heads * cfg.max_blocks * cfg.page_bytes
         o = self.offsets[0]
         return self.buffer[o:o + n].view(cfg.batch, cfg.n_kv_heads, cfg.max_blocks,
                                          cfg.page_bytes)
+
+    def pool_sets(self):
+        """Paged caches: the pool as [n_pages, n_kv_heads, page_bytes]."""
+        cfg = self.cfg
+        return self.pool.view(self.n_pages, cfg.n_kv_heads, cfg.page_bytes)
+
+    def head_pages(self, b, h, nb):
+        """Blocks 0 .. nb - 1 of (sequence b, kv-head h) as [nb, page_bytes]
+        (gathered through the block table for a paged cache)."""
+        if not self.paged:
+            return self.pages()[b, h, :nb]
+        sets = self.block_table[b, :nb].long()
+        return self.pool_sets()[sets, h]
 
     def resid(self):
         cfg = self.cfg
@@ -228,6 +294,13 @@ class QuantKVCache:
 
     def flags(self):
         return int(self.seq_region()[self.cfg.batch].item())
+
+
+def blocks_written(L, n_new, residual=128, group=32):
+    """Blocks a call that appends n_new tokens to a sequence of L tokens
+    writes: [packed_len(L) / 32, packed_len(L + n_new) / 32)."""
+    return range(packed_len(L, residual, group) // group,
+                 packed_len(L + n_new, residual, group) // group)
 
 
 def kvq_pack(cache: QuantKVCache, k_new, v_new, batch_begin=0, stream=None):

@@ -59,7 +59,7 @@ def head_arrays(cache, b, h, L):
     Lq = kvq.packed_len(L, cfg.residual)
     nb = Lq // 32
     bk, bv = cfg.bits_k, cfg.bits_v
-    pages = cache.pages()[b, h, :nb].cpu().numpy()
+    pages = cache.head_pages(b, h, nb).cpu().numpy()
 
     def sl(a, c):
         return np.ascontiguousarray(pages[:, a:c])

@@ -68,6 +68,50 @@ def test_layout_sizes(L):
     assert L.kvq_page_bytes(ctypes.byref(c)) == 512 * 5 + 1024
 
 
+def test_paged_layout_and_bind(L):
+    cfg = _cfg(bits_k=1, bits_v=4)
+    c = cfg.c()
+    total, offs = cfg.layout()
+    tot = ctypes.c_size_t()
+    po = (ctypes.c_size_t * 4)()
+    assert L.kvq_paged_cache_layout(ctypes.byref(c), ctypes.byref(tot), ctypes.byref(po)) == 0
+    # the rings and lengths only: the page region of the contiguous layout is gone
+    assert po[0] == 0 and po[1] == 0
+    assert tot.value == total - offs[1]
+    assert L.kvq_page_pool_bytes(ctypes.byref(c), 10) == 10 * 8 * (512 * 5 + 1024)
+    assert L.kvq_page_pool_bytes(ctypes.byref(c), 0) == 0
+    cache = kvq._Cache()
+    base, pool, tbl = ctypes.c_void_p(0x10000), ctypes.c_void_p(0x20000), ctypes.c_void_p(0x30000)
+    assert L.kvq_paged_cache_bind(ctypes.byref(c), base, pool, 10, tbl, ctypes.byref(cache)) == 0
+    assert cache.pages == 0x20000 and cache.block_table == 0x30000 and cache.n_pages == 10
+    assert cache.k_resid == 0x10000 + po[1] and cache.seq_len == 0x10000 + po[3]
+    nul = ctypes.c_void_p(None)
+    assert L.kvq_paged_cache_bind(ctypes.byref(c), base, pool, 10, nul, ctypes.byref(cache)) == 1
+    assert L.kvq_paged_cache_bind(ctypes.byref(c), base, pool, 0, tbl, ctypes.byref(cache)) == 1
+    assert L.kvq_paged_cache_bind(ctypes.byref(c), base, ctypes.c_void_p(0x20008), 10, tbl,
+                                  ctypes.byref(cache)) == 5
+    assert L.kvq_paged_cache_bind(ctypes.byref(c), base, pool, 10, ctypes.c_void_p(0x30002),
+                                  ctypes.byref(cache)) == 5
+    # the contiguous bind clears the paged fields
+    assert L.kvq_cache_bind(ctypes.byref(c), base, ctypes.byref(cache)) == 0
+    assert not cache.block_table and cache.n_pages == 0
+    # a paged cache with n_pages < 1 is rejected before any launch
+    bad = kvq._Cache(pool, base, base, base, tbl, 0)
+    fake = ctypes.c_void_p(0x1000)
+    assert L.kvq_pack(ctypes.byref(c), ctypes.byref(bad), fake, fake, 1, 0, 2, nul) == 1
+
+
+def test_paged_helpers():
+    # 4096 tokens: Lq = 32 * floor(3968 / 32) = 3968, blocks 0 .. 123
+    assert list(kvq.blocks_written(0, 4096)) == list(range(0, 124))
+    assert list(kvq.blocks_written(159, 1)) == [0]      # 160 tokens: the first group leaves
+    assert list(kvq.blocks_written(160, 1)) == []
+    assert list(kvq.blocks_written(190, 1)) == []
+    assert list(kvq.blocks_written(191, 1)) == [1]      # 192 - 128 = 64: the second group
+    assert list(kvq.blocks_written(100, 45)) == []
+    assert list(kvq.blocks_written(100, 92)) == [0, 1]   # 192 tokens: Lq = 64
+
+
 def test_workspace_sizes(L):
     cfg = _cfg()
     c = cfg.c()
