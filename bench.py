@@ -65,6 +65,8 @@ def parse():
     p.add_argument("--layers", type=int, default=0, help="override the layer count")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--splits", type=int, default=0,
+                   help="CTAs per (sequence, kv-head); 0 = kvq_attn_splits_for_lengths")
     p.add_argument("--paged", action="store_true",
                    help="run the caches on the paged layout (block table, shuffled pool)")
     p.add_argument("--cpu-worker", default="", help=argparse.SUPPRESS)
@@ -89,6 +91,8 @@ def workload_spec(args):
         spec["layers"] = args.layers
     if getattr(args, "paged", False):
         spec["paged"] = True
+    if getattr(args, "splits", 0):
+        spec["splits"] = args.splits
     return spec
 
 
@@ -440,7 +444,7 @@ class Step:
         self.k_new = torch.randn(layers, B, hkv, 128, generator=g, device=device).half()
         self.v_new = torch.randn(layers, B, hkv, 128, generator=g, device=device).half()
         self.out = torch.empty(layers, B, hq, 128, dtype=torch.float16, device=device)
-        self.n_splits = kvq.splits_for_lengths(self.cfg, self.lengths0)
+        self.n_splits = spec.get("splits") or kvq.splits_for_lengths(self.cfg, self.lengths0)
         self.ws_attn = kvq.attn_workspace(self.cfg, self.n_splits, device)
         self.dgap = kvq.DGAP(synth.dgap_weights(seed, K=DGAP_K, hidden=DGAP_HIDDEN), K=DGAP_K,
                              tau=DGAP_TAU, device=device)

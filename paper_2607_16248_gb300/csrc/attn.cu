@@ -295,14 +295,19 @@ struct TcState {
 };
 
 // Online softmax over NB 32-token blocks (per block 4 token rows x 2 heads
-// per lane), then the probabilities as fp16 high / low parts moved to the
-// B-operand layout of the value MMAs with movmatrix.
-//   narrow (up to 4 heads): columns 0..3 / 4..7 hold the high / low parts of
-//     heads 0..3 (lanes tig and tig^2 hold the same scores); pt is one
-//     operand whose columns carry both parts;
-//   wide (5..8 heads): column = head; pt holds the high parts, pl the low
-//     parts, each one operand of its own MMA.
-template <int NB, bool kWide>
+// per lane), then the probabilities moved to the B-operand layout of the
+// value MMAs with movmatrix.
+//   exact (kCompact false): p as an fp16 high part and its fp16 residual;
+//     narrow (up to 4 heads): columns 0..3 / 4..7 hold the high / low parts
+//     of heads 0..3 (lanes tig and tig^2 hold the same scores), pt is one
+//     operand whose columns carry both parts; wide (5..8 heads): column =
+//     head, pt holds the high parts, pl the low parts, each one operand of
+//     its own MMA.
+//   compact (1-bit values): the weights are p~ = RN16(p), used alike in the
+//     row sum and in the value MMAs (so they are a consistent softmax of
+//     scores perturbed by at most 2^-11 relative); pt holds p~ (column =
+//     head; narrow: columns 4..7 zero), pl is unused.
+template <int NB, bool kWide, bool kCompact>
 __device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, const Lane& ln,
                                            uint32_t (&pt)[NB][2][2], uint32_t (&pl)[NB][2][2]) {
   float mx[2];
@@ -348,10 +353,16 @@ __device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, c
         const int j = 2 * mt + rh;
         const float p0 = fast_exp2(sc[bi][j][0] - st.m[0]);
         const float p1 = fast_exp2(sc[bi][j][1] - st.m[1]);
-        st.l[0] += p0;
-        st.l[1] += p1;
         const __half2 h = __floats2half2_rn(p0, p1);
         const float2 hf = __half22float2(h);
+        if constexpr (kCompact) {
+          st.l[0] += hf.x;
+          st.l[1] += hf.y;
+          pt[bi][mt][rh] = movmatrix_t(kWide || ln.tig < 2 ? h2u(h) : 0u);
+          continue;
+        }
+        st.l[0] += p0;
+        st.l[1] += p1;
         if constexpr (kWide) {
           pt[bi][mt][rh] = movmatrix_t(h2u(h));
           pl[bi][mt][rh] = movmatrix_t(h2u(__floats2half2_rn(p0 - hf.x, p1 - hf.y)));
@@ -456,8 +467,9 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
         }
   }
 
+  constexpr bool kCompact = BV == 1;
   uint32_t pt[NB][2][2], pl[NB][2][2];
-  tc_softmax<NB, kWide>(sc, st, ln, pt, pl);
+  tc_softmax<NB, kWide, kCompact>(sc, st, ln, pt, pl);
 
   // ---- values: o^T[c][h] ----
   // Value scales and zeros are stored in token pairs (t, t + 4), so the
@@ -471,6 +483,33 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
     const uint4 z8 = *reinterpret_cast<const uint4*>(vzrow + 2 * (kHeadDim + 32 * (gid & 3) + 8 * tig));
     mma16816(st.zv, z8.x, 0u, z8.y, 0u, pt[bi][0][0], pt[bi][0][1]);
     mma16816(st.zv, z8.z, 0u, z8.w, 0u, pt[bi][1][0], pt[bi][1][1]);
+    if constexpr (kCompact) {
+      // 1-bit values: B = RN16(p~ s), one MMA per operand for every head
+      const uint4 vw = *reinterpret_cast<const uint4*>(vc + 16 * lane);
+#pragma unroll
+      for (int g = 0; g < 4; ++g) {
+        const uint4 s8 = *reinterpret_cast<const uint4*>(vmeta + 2 * (32 * g + 8 * tig));
+        const uint32_t mw[4] = {s8.x, s8.y, s8.z, s8.w};
+#pragma unroll
+        for (int ks = 0; ks < 2; ++ks) {
+          uint32_t am0[4], am1[4], bv[2];
+#pragma unroll
+          for (int dl = 0; dl < 2; ++dl) {
+            const int ia = 2 * ks + dl;
+            uint32_t v[4];
+            Codes<1>::rot(comp(vw, g), ia, v);
+            am0[2 * dl] = v[0];
+            am0[2 * dl + 1] = v[1];
+            am1[2 * dl] = v[2];
+            am1[2 * dl + 1] = v[3];
+            bv[dl] = h2u(__hmul2(u2h(pt[bi][ks][dl]), u2h(mw[ia])));
+          }
+          mma16816(st.acc[2 * g], am0[0], am0[1], am0[2], am0[3], bv[0], bv[1]);
+          mma16816(st.acc[2 * g + 1], am1[0], am1[1], am1[2], am1[3], bv[0], bv[1]);
+        }
+      }
+      continue;
+    }
     if constexpr (kWide) {
       mma16816(st.zv, z8.x, 0u, z8.y, 0u, pl[bi][0][0], pl[bi][0][1]);
       mma16816(st.zv, z8.z, 0u, z8.w, 0u, pl[bi][1][0], pl[bi][1][1]);
@@ -664,7 +703,7 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t 
                : "memory");
 }
 
-template <bool kWide>
+template <bool kWide, bool kCompact>
 __device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
                                                 const uint32_t (&qb)[16], const Lane& ln,
                                                 float scale_log2, TcState& st,
@@ -690,10 +729,10 @@ __device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
       for (int hh = 0; hh < 2; ++hh)
         sc[0][2 * mt + rh][hh] = ok ? dk[mt][2 * rh + hh] * scale_log2 : -INFINITY;
     }
-  tc_softmax<1, kWide>(sc, st, ln, pt, pl);
+  tc_softmax<1, kWide, kCompact>(sc, st, ln, pt, pl);
 }
 
-template <bool kWide>
+template <bool kWide, bool kCompact>
 __device__ __forceinline__ void tc_resid_values(const __half* vs_s, const uint32_t (&pt)[1][2][2],
                                                 const uint32_t (&pl)[1][2][2], TcState& st) {
   const int lane = threadIdx.x & 31;
@@ -705,7 +744,8 @@ __device__ __forceinline__ void tc_resid_values(const __half* vs_s, const uint32
       uint32_t a[4];
       ldsm_x4_t(a, vs_s + (16 * ks + 8 * (mi >> 1) + r8) * kResRow + 16 * mtp + 8 * (mi & 1));
       mma16816(st.acc[mtp], a[0], a[1], a[2], a[3], pt[0][ks][0], pt[0][ks][1]);
-      if constexpr (kWide) mma16816(st.acc[mtp], a[0], a[1], a[2], a[3], pl[0][ks][0], pl[0][ks][1]);
+      if constexpr (kWide && !kCompact)
+        mma16816(st.acc[mtp], a[0], a[1], a[2], a[3], pl[0][ks][0], pl[0][ks][1]);
     }
 }
 
@@ -1101,13 +1141,13 @@ __device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half
       if ((threadIdx.x & 31) == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
       return;
     }
-    tc_resid_scores<kWide>(rows, n_tok, qb, ln, scale_log2, st, pt, pl);
+    tc_resid_scores<kWide, BV == 1>(rows, n_tok, qb, ln, scale_log2, st, pt, pl);
     __syncwarp();
     if (!stage_rows_bulk(rows, ring_v, p0, n_tok, d.ring, p_new, v_row, bar, phase++ & 1u)) {
       if ((threadIdx.x & 31) == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
       return;
     }
-    tc_resid_values<kWide>(rows, pt, pl, st);
+    tc_resid_values<kWide, BV == 1>(rows, pt, pl, st);
     __syncwarp();
   }
 }

@@ -8,6 +8,16 @@ import pytest
 import torch
 
 import _util
+
+
+def pair_tol(cfg):
+    """How far the fused step may sit from pack-then-attend on the same
+    split count: fp32 summation order only (1e-5 x rms) for wider value
+    codes; for 1-bit values the fp16 softmax weights are rounded relative to
+    each warp's running maximum, which the flushed block (folded from shared
+    memory at the end of its warp's range) can change, so 2^-12-relative
+    rounding differences of single weights show (3e-4 x rms)."""
+    return 3e-4 if cfg.bits_v == 1 else 1e-5
 from oracle import attention
 from paper_2607_16248_gb300 import kvq, synth
 
@@ -34,7 +44,7 @@ def _steps(cfg, lengths, n_steps, seed, check_oracle_every=0, n_splits=0):
         out_a = kvq.kvq_decode_step(a, kn.cuda(), vn.cuda(), q.cuda(), n_splits=n_splits,
                                     out_dtype=torch.float32)
         kvq.kvq_pack(b_, kn[:, :, None].cuda(), vn[:, :, None].cuda())
-        out_b = kvq.kvq_decode_attn(b_, q.cuda(), out_dtype=torch.float32)
+        out_b = kvq.kvq_decode_attn(b_, q.cuda(), n_splits=n_splits, out_dtype=torch.float32)
         torch.cuda.synchronize()
         oa, ob = out_a.cpu().numpy(), out_b.cpu().numpy()
         for s in range(cfg.batch):
@@ -62,7 +72,7 @@ def test_steps_equal_pack_then_attention(kvq_lib, bk, bv):
     cfg = kvq.CacheConfig(batch=len(lengths), n_q_heads=8, n_kv_heads=2, bits_k=bk, bits_v=bv,
                           max_len=1024)
     pair, oracle = _steps(cfg, lengths, 36, seed=bk * 7 + bv, check_oracle_every=12)
-    assert pair <= 1e-5, pair
+    assert pair <= pair_tol(cfg), pair
     assert oracle <= _util.ATTN_TOL, oracle
 
 
@@ -73,7 +83,7 @@ def test_wide_query_groups(kvq_lib, gq):
     cfg = kvq.CacheConfig(batch=3, n_q_heads=2 * gq, n_kv_heads=2, bits_k=1, bits_v=2,
                           max_len=1024)
     pair, oracle = _steps(cfg, [158, 400, 159], 5, seed=21 + gq, check_oracle_every=5)
-    assert pair <= 1e-5, pair
+    assert pair <= pair_tol(cfg), pair
     assert oracle <= _util.ATTN_TOL, oracle
 
 
@@ -89,7 +99,7 @@ def test_flush_workers_for_window_sizes(kvq_lib, residual, n_splits, bk, bv):
                           max_len=4 * R + 128, residual=R)
     pair, oracle = _steps(cfg, lengths, 34, seed=R + n_splits, check_oracle_every=17,
                           n_splits=n_splits)
-    assert pair <= 1e-5, pair
+    assert pair <= pair_tol(cfg), pair
     assert oracle <= _util.ATTN_TOL, oracle
 
 
