@@ -616,6 +616,7 @@ def run_gpu(args, spec):
     attn_bytes_total = sum(st.bytes_for_step(ph_step0 + i) for i in range(K))
 
     single = single_layer_times(st, device) if rank == 0 else None
+    prefill = prefill_rate(st, device) if rank == 0 else None
 
     value = job_gbs(world, bytes_total, total_ms)
     launches = K * st.launches_per_step()
@@ -659,6 +660,7 @@ def run_gpu(args, spec):
         "attn_us_per_layer": round(attn_ms / attn_launches * 1e3, 3),
         "epilogue_us_per_step": round(epi_ms / K * 1e3, 3),
         "single_layer": single,
+        "prefill": prefill,
         "epilogue_frac_of_step_attn": round(epi_ms / attn_ms, 5),
         "breakdown": "attn_us_per_layer: the step's kvq_decode_step launches (append + "
                      "attention) alone in one graph; epilogue_us_per_step: a graph of 10 x (logits "
@@ -684,6 +686,42 @@ def run_gpu(args, spec):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def prefill_rate(st, device, reps=3):
+    """kvq_pack of one layer's prefill (every sequence, its whole context)
+    into a scratch cache, inputs already on the device: algorithmic bytes
+    (fp16 K/V read, pages and fp16 window rows written) over the device time
+    of the calls, best of `reps`."""
+    import torch
+    from paper_2607_16248_gb300 import kvq, synth
+    s = st.spec
+    hkv, b = s["n_kv_heads"], s["bits"]
+    scratch = kvq.QuantKVCache(st.cfg, device)
+    kv = [synth.kv_heads(777 + i, hkv, L, device=device) for i, L in enumerate(st.lengths0)]
+    byts = 0
+    for L in st.lengths0:
+        Lq = packed_len(L)
+        byts += hkv * (L * 512 + Lq * (16 * (b + b) + 32) + (L - Lq) * 512)
+    best = None
+    for _ in range(reps):
+        scratch.reset()
+        torch.cuda.synchronize()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for i, (k, v) in enumerate(kv):
+            kvq.kvq_pack(scratch, k[None], v[None], batch_begin=i)
+        t1.record()
+        torch.cuda.synchronize()
+        ms = t0.elapsed_time(t1)
+        best = ms if best is None else min(best, ms)
+    del kv, scratch
+    peak, _ = measured_peak_hbm()
+    gbs = byts / (best * 1e-3) / 1e9
+    return {"gbs": round(gbs, 2), "frac": round(gbs / peak, 4), "bytes": byts,
+            "us": round(best * 1e3, 2),
+            "note": "one layer's kvq_pack of every sequence's prefill (fp16 K/V in, pages and "
+                    "window out), inputs resident, best of 3"}
 
 
 def single_layer_times(st, device, reps=50, warm=5):

@@ -891,102 +891,20 @@ __device__ __forceinline__ int tc_pre_issue(const PageMap& pm, TableWin& tw, int
 
 // Decode step with a flush: the 32-token block of positions [p0, p0 + 32),
 // still fp16 in the ring, leaves the window and is quantized exactly as
-// kvq_pack does (same quantizer, same page layout) into a page image in
-// shared memory.  The work comes in four quarters: quarter qi is the key
-// groups of channels 32 qi .. 32 qi + 31 (lane = channel) and value group qi
-// of the 32 tokens (lane = token).  The quarters write disjoint words of the
-// image (1-bit codes: words 4 l + qi, l = 0..31), so different warps can
-// take them.  Rows are read straight from global memory (L2); nothing in
-// this kernel writes them.  Kept out of line: it is rare and its registers
-// would otherwise crowd the streaming loop.
+// kvq_pack does (quantize_quarter, common.cuh) into a page image in shared
+// memory.  The work comes in four quarters (key channels 32 qi .. 32 qi + 31,
+// value group qi), so different warps can take them.  Rows are read straight
+// from global memory (L2); nothing in this kernel writes them.  Kept out of
+// line: it is rare and its registers would otherwise crowd the streaming
+// loop.
 template <int BK, int BV>
 __device__ __noinline__ void flush_quarter(const __half* ring_k, const __half* ring_v, int p0,
                                            int ring, int qi, char* image) {
-  const int lane = threadIdx.x & 31;
-  uint32_t* kcodes = reinterpret_cast<uint32_t*>(image);
-  uint32_t* vcodes = reinterpret_cast<uint32_t*>(image + page_off_vcodes(BK));
-  __half* kmeta = reinterpret_cast<__half*>(image + page_off_kmeta(BK));
-  __half* vmeta = reinterpret_cast<__half*>(image + page_off_vmeta(BK, BV));
   const int s0 = p0 % ring;
-  const int c = kGroup * qi + lane;  // this lane's key channel
-  float xk[kGroup], xv[kGroup];
-#pragma unroll
-  for (int t = 0; t < kGroup; ++t) {
-    const int s = s0 + t < ring ? s0 + t : s0 + t - ring;
-    xk[t] = __half2float(ring_k[(long long)s * kHeadDim + c]);
-  }
-  {
-    const int s = s0 + lane < ring ? s0 + lane : s0 + lane - ring;
-    const uint4* row = reinterpret_cast<const uint4*>(ring_v + (long long)s * kHeadDim + kGroup * qi);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const uint4 u = row[k];
-      const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 f = __half22float2(u2h(wd[e]));
-        xv[8 * k + 2 * e] = f.x;
-        xv[8 * k + 2 * e + 1] = f.y;
-      }
-    }
-  }
-  uint32_t wk[BK], wv[BV];
-  __half sk, zk, sv, zv;
-  quantize_group<BK>(xk, wk, sk, zk);
-  quantize_group<BV>(xv, wv, sv, zv);
-  kmeta[c] = sk;
-  kmeta[kHeadDim + c] = zk;
-  vmeta[vmeta_index(qi, lane)] = sv;
-  vmeta[kHeadDim + vmeta_index(qi, lane)] = zv;
-  // 1-bit codes: lane l = 4 gid + tig assembles word 4 l + qi from ballots
-  // (bit positions of key1_bit / val1_bit)
-  const int gid = lane >> 2, tig = lane & 3;
-  if constexpr (BK == 1) {
-    uint32_t mine[4] = {0u, 0u, 0u, 0u};  // ballots of tokens 4 gid + j over channels
-#pragma unroll
-    for (int t = 0; t < kGroup; ++t) {
-      const uint32_t bt = __ballot_sync(0xffffffffu, (wk[0] >> t) & 1u);
-      if ((t >> 2) == gid) mine[t & 3] = bt;
-    }
-    uint32_t word = 0u;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t m = mine[j] >> (4 * tig);
-#pragma unroll
-      for (int ks1 = 0; ks1 < 2; ++ks1)
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int e = 0; e < 2; ++e)
-            word |= ((m >> (16 * ks1 + 2 * h + e)) & 1u) << ((10 + 16 * e + j - 4 * (2 * ks1 + h)) & 31);
-    }
-    kcodes[4 * lane + qi] = word;
-  } else {
-#pragma unroll
-    for (int j = 0; j < BK; ++j) kcodes[c * BK + j] = wk[j];
-  }
-  if constexpr (BV == 1) {
-    uint32_t mine[4] = {0u, 0u, 0u, 0u};  // ballots of channels 4 gid + j over tokens
-#pragma unroll
-    for (int ci = 0; ci < kGroup; ++ci) {
-      const uint32_t bc = __ballot_sync(0xffffffffu, (wv[0] >> ci) & 1u);
-      if ((ci >> 2) == gid) mine[ci & 3] = bc;
-    }
-    uint32_t word = 0u;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t m = mine[j] >> (8 * tig);
-#pragma unroll
-      for (int e = 0; e < 2; ++e)
-#pragma unroll
-        for (int r = 0; r < 4; ++r)
-          word |= ((m >> (4 * e + r)) & 1u) << ((10 + 16 * e + j - 4 * r) & 31);
-    }
-    vcodes[4 * lane + qi] = word;
-  } else {
-#pragma unroll
-    for (int j = 0; j < BV; ++j) vcodes[(qi * kGroup + lane) * BV + j] = wv[j];
-  }
+  quantize_quarter<BK, BV>(
+      [&](int t) { return ring_k + (long long)(s0 + t < ring ? s0 + t : s0 + t - ring) * kHeadDim; },
+      [&](int t) { return ring_v + (long long)(s0 + t < ring ? s0 + t : s0 + t - ring) * kHeadDim; },
+      qi, image);
 }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {

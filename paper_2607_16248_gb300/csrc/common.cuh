@@ -98,6 +98,99 @@ __device__ __forceinline__ void quantize_group(const float (&x)[kGroup], uint32_
   zero = __float2half_rn(lo);  // lo is an fp16 value: exact
 }
 
+// One quarter qi of a 32-token block, quantized by one warp into a page (or
+// a page image): key groups of channels 32 qi .. 32 qi + 31 (lane = channel)
+// and value group qi of the 32 tokens (lane = token).  row_k(t), row_v(t)
+// give the fp16 rows [128] of token t of the block.  The quarters write
+// disjoint words, scales and zeros (1-bit codes: words 4 l + qi, l = 0..31,
+// assembled from warp ballots in the order key1_bit / val1_bit give), so the
+// four may run in different warps.  Used by kvq_pack and by the decode
+// step's flush, which are therefore bit-identical.
+template <int BK, int BV, typename RowK, typename RowV>
+__device__ __forceinline__ void quantize_quarter(RowK row_k, RowV row_v, int qi, char* image) {
+  const int lane = threadIdx.x & 31;
+  uint32_t* kcodes = reinterpret_cast<uint32_t*>(image);
+  uint32_t* vcodes = reinterpret_cast<uint32_t*>(image + page_off_vcodes(BK));
+  __half* kmeta = reinterpret_cast<__half*>(image + page_off_kmeta(BK));
+  __half* vmeta = reinterpret_cast<__half*>(image + page_off_vmeta(BK, BV));
+  const int c = kGroup * qi + lane;  // this lane's key channel
+  float xk[kGroup], xv[kGroup];
+#pragma unroll
+  for (int t = 0; t < kGroup; ++t) xk[t] = __half2float(row_k(t)[c]);
+  {
+    const uint4* row = reinterpret_cast<const uint4*>(row_v(lane) + kGroup * qi);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint4 u = row[k];
+      const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&wd[e]));
+        xv[8 * k + 2 * e] = f.x;
+        xv[8 * k + 2 * e + 1] = f.y;
+      }
+    }
+  }
+  uint32_t wk[BK], wv[BV];
+  __half sk, zk, sv, zv;
+  quantize_group<BK>(xk, wk, sk, zk);
+  quantize_group<BV>(xv, wv, sv, zv);
+  kmeta[c] = sk;
+  kmeta[kHeadDim + c] = zk;
+  vmeta[vmeta_index(qi, lane)] = sv;
+  vmeta[kHeadDim + vmeta_index(qi, lane)] = zv;
+  // 1-bit codes: lane l = 4 gid + tig assembles word 4 l + qi from ballots
+  // (bit positions of key1_bit / val1_bit)
+  const int gid = lane >> 2, tig = lane & 3;
+  if constexpr (BK == 1) {
+    uint32_t mine[4] = {0u, 0u, 0u, 0u};  // ballots of tokens 4 gid + j over channels
+#pragma unroll
+    for (int t = 0; t < kGroup; ++t) {
+      const uint32_t bt = __ballot_sync(0xffffffffu, (wk[0] >> t) & 1u);
+      if ((t >> 2) == gid) mine[t & 3] = bt;
+    }
+    uint32_t word = 0u;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t m = mine[j] >> (4 * tig);
+#pragma unroll
+      for (int ks1 = 0; ks1 < 2; ++ks1)
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int e = 0; e < 2; ++e)
+            word |= ((m >> (16 * ks1 + 2 * h + e)) & 1u) << ((10 + 16 * e + j - 4 * (2 * ks1 + h)) & 31);
+    }
+    kcodes[4 * lane + qi] = word;
+  } else {
+#pragma unroll
+    for (int j = 0; j < BK; ++j) kcodes[c * BK + j] = wk[j];
+  }
+  if constexpr (BV == 1) {
+    uint32_t mine[4] = {0u, 0u, 0u, 0u};  // ballots of channels 4 gid + j over tokens
+#pragma unroll
+    for (int ci = 0; ci < kGroup; ++ci) {
+      const uint32_t bc = __ballot_sync(0xffffffffu, (wv[0] >> ci) & 1u);
+      if ((ci >> 2) == gid) mine[ci & 3] = bc;
+    }
+    uint32_t word = 0u;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t m = mine[j] >> (8 * tig);
+#pragma unroll
+      for (int e = 0; e < 2; ++e)
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          word |= ((m >> (4 * e + r)) & 1u) << ((10 + 16 * e + j - 4 * r) & 31);
+    }
+    vcodes[4 * lane + qi] = word;
+  } else {
+#pragma unroll
+    for (int j = 0; j < BV; ++j) vcodes[(qi * kGroup + lane) * BV + j] = wv[j];
+  }
+}
+
+
 // Tokens held in quantized blocks when L tokens are cached.
 __host__ __device__ inline int packed_len(int L, int residual) {
   int over = L - residual;

@@ -173,11 +173,17 @@ __device__ __forceinline__ RowSrc make_src(const Dims& d, const kvq_cache& c, co
   return s;
 }
 
-// Blocks made only of new tokens (prefill).  grid (x, hkv, batch_count).
-__global__ void __launch_bounds__(kPackThreads)
+// Blocks made only of new tokens (prefill): one warp per quarter of a block
+// (quantize_quarter: key channels 32 w .. 32 w + 31 and value group w),
+// reading the rows straight from the input, so no staging tile and no
+// shared-memory atomics; many small CTAs keep the loads of many blocks in
+// flight.  grid (blocks, hkv, batch_count) of 128 threads.
+constexpr int kInputThreads = 4 * 32;
+
+template <int BK, int BV>
+__global__ void __launch_bounds__(kInputThreads)
     pack_input_blocks_kernel(Dims d, kvq_cache c, const __half* __restrict__ k_new,
                              const __half* __restrict__ v_new, int n_new, int batch_begin) {
-  __shared__ Tile tile;
   pdl_enter();
   const int bi = blockIdx.z, b = batch_begin + bi, h = blockIdx.y;
   const int L0 = c.seq_len[b];
@@ -188,10 +194,35 @@ __global__ void __launch_bounds__(kPackThreads)
   if (j >= packed_len(L1, d.residual) / kGroup) return;
   char* page = page_ptr(d, c, b, h, j);
   if (!page) return;
-  const RowSrc src = make_src(d, c, k_new, v_new, n_new, b, bi, h, L0);
-  load_tile(tile, src, j);
-  __syncthreads();
-  quantize_tile(tile, page, d.bits_k, d.bits_v);
+  const long long nh = ((long long)bi * d.hkv + h) * n_new;
+  const __half* nk = k_new + (nh + (long long)j * kGroup - L0) * kHeadDim;
+  const __half* nv = v_new + (nh + (long long)j * kGroup - L0) * kHeadDim;
+  quantize_quarter<BK, BV>([&](int t) { return nk + (long long)t * kHeadDim; },
+                           [&](int t) { return nv + (long long)t * kHeadDim; },
+                           threadIdx.x >> 5, page);
+}
+
+template <int BK>
+cudaError_t launch_input_blocks_bv(const Dims& d, cudaLaunchConfig_t& cfg, const kvq_cache& cache,
+                                   const __half* k_new, const __half* v_new, int n_new,
+                                   int batch_begin) {
+  switch (d.bits_v) {
+    case 1: return cudaLaunchKernelEx(&cfg, pack_input_blocks_kernel<BK, 1>, d, cache, k_new, v_new, n_new, batch_begin);
+    case 2: return cudaLaunchKernelEx(&cfg, pack_input_blocks_kernel<BK, 2>, d, cache, k_new, v_new, n_new, batch_begin);
+    case 4: return cudaLaunchKernelEx(&cfg, pack_input_blocks_kernel<BK, 4>, d, cache, k_new, v_new, n_new, batch_begin);
+    default: return cudaLaunchKernelEx(&cfg, pack_input_blocks_kernel<BK, 8>, d, cache, k_new, v_new, n_new, batch_begin);
+  }
+}
+
+cudaError_t launch_input_blocks(const Dims& d, cudaLaunchConfig_t& cfg, const kvq_cache& cache,
+                                const __half* k_new, const __half* v_new, int n_new,
+                                int batch_begin) {
+  switch (d.bits_k) {
+    case 1: return launch_input_blocks_bv<1>(d, cfg, cache, k_new, v_new, n_new, batch_begin);
+    case 2: return launch_input_blocks_bv<2>(d, cfg, cache, k_new, v_new, n_new, batch_begin);
+    case 4: return launch_input_blocks_bv<4>(d, cfg, cache, k_new, v_new, n_new, batch_begin);
+    default: return launch_input_blocks_bv<8>(d, cfg, cache, k_new, v_new, n_new, batch_begin);
+  }
 }
 
 // Blocks that touch the ring, the ring append, and the length update.
@@ -264,9 +295,10 @@ cudaError_t launch_pack(const Dims& d, const kvq_cache& cache, const __half* k_n
   cudaError_t e;
   if (n_new > kGroup) {
     cfg.gridDim = dim3(n_new / kGroup + 1, d.hkv, batch_count);
-    e = cudaLaunchKernelEx(&cfg, pack_input_blocks_kernel, d, cache, k_new, v_new, n_new,
-                           batch_begin);
+    cfg.blockDim = dim3(kInputThreads);
+    e = launch_input_blocks(d, cfg, cache, k_new, v_new, n_new, batch_begin);
     if (e != cudaSuccess) return e;
+    cfg.blockDim = dim3(kPackThreads);
   }
   cfg.gridDim = dim3(d.hkv, batch_count);
   e = cudaLaunchKernelEx(&cfg, pack_append_kernel, d, cache, k_new, v_new, n_new, batch_begin);
