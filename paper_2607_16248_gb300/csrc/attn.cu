@@ -22,6 +22,8 @@
 //           A = codes (M = tokens, K = channels), B = q*s split into an fp16
 //           high part and its exact fp16 residual, so the products are
 //           exact; the zero-point term is one more MMA with A = z, B = q.
+//           1-bit keys with 5..8-head groups instead scale A: A = code * s
+//           (one fp16 multiply per register), B = q, one MMA per tile.
 //   values  o[c][h] += sum_t code[t][c] * (p_h[t] s_t,g) + sum_t p_h[t] z_t,g
 //           A = codes (M = channels, K = tokens), B = p*s with p split into
 //           high / low fp16 parts; P moves from the score (accumulator)
@@ -58,6 +60,7 @@ constexpr int kRingBudget = (kCtasPerSm == 2 ? 96 : 192) * 1024;  // staged page
 constexpr int kHeads = kMaxGq;  // query heads per CTA (the wide layout's head columns)
 constexpr long long kWaitCycles = 4000000000LL;  // bounded mbarrier waits (~2 s)
 constexpr int kZeroBytes = 512;                   // all-zero metadata rows
+constexpr int kOnesWord0 = 64;                    // ... but for fp16 ones at bytes 256..319
 
 struct Ws {
   float* m;       // [B][Hq][S]
@@ -296,7 +299,12 @@ struct TcState {
 
 // Online softmax over NB 32-token blocks (per block 4 token rows x 2 heads
 // per lane), then the probabilities moved to the B-operand layout of the
-// value MMAs with movmatrix.
+// value MMAs with movmatrix.  The scores arrive as t = score - m_eff (log2
+// domain), m_eff being the lane's running maximum (0 before its first
+// block), so the common case (no score above the maximum) costs one exp2 per
+// score and a vote; only when some score exceeds it (or before the first
+// block) is the new maximum found across the warp, the state rescaled and t
+// shifted.
 //   exact (kCompact false): p as an fp16 high part and its fp16 residual;
 //     narrow (up to 4 heads): columns 0..3 / 4..7 hold the high / low parts
 //     of heads 0..3 (lanes tig and tig^2 hold the same scores), pt is one
@@ -307,27 +315,33 @@ struct TcState {
 //     row sum and in the value MMAs (so they are a consistent softmax of
 //     scores perturbed by at most 2^-11 relative); pt holds p~ (column =
 //     head; narrow: columns 4..7 zero), pl is unused.
-template <int NB, bool kWide, bool kCompact>
-__device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, const Lane& ln,
+// kSumL: add the weights to st.l here (window chunks).  Packed blocks leave
+// it: their row sums come out of the value zero-point MMA, whose A row 4 is
+// all ones (see tc_unit).
+template <int NB, bool kWide, bool kCompact, bool kSumL>
+__device__ __forceinline__ void tc_softmax(float (&t)[NB][4][2], TcState& st, const Lane& ln,
                                            uint32_t (&pt)[NB][2][2], uint32_t (&pl)[NB][2][2]) {
-  float mx[2];
+  float tm[2];
 #pragma unroll
   for (int hh = 0; hh < 2; ++hh) {
     float x = -INFINITY;
 #pragma unroll
     for (int bi = 0; bi < NB; ++bi)
-      x = fmaxf(x, fmaxf(fmaxf(sc[bi][0][hh], sc[bi][1][hh]), fmaxf(sc[bi][2][hh], sc[bi][3][hh])));
-    x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 4));
-    x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 8));
-    x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16));
-    mx[hh] = x;
+      x = fmaxf(x, fmaxf(fmaxf(t[bi][0][hh], t[bi][1][hh]), fmaxf(t[bi][2][hh], t[bi][3][hh])));
+    tm[hh] = x;
   }
-  const bool grow = mx[0] > st.m[0] || mx[1] > st.m[1];
-  if (__any_sync(0xffffffffu, grow)) {
-    float corr[2];
+  const bool fresh = st.m[0] == -INFINITY;
+  if (__any_sync(0xffffffffu, tm[0] > 0.0f || tm[1] > 0.0f || fresh)) {
+    float corr[2], delta[2];
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
-      const float mn = fmaxf(st.m[hh], mx[hh]);
+      float x = tm[hh];
+      x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 4));
+      x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 8));
+      x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16));
+      const float me = st.m[hh] == -INFINITY ? 0.0f : st.m[hh];
+      const float mn = fmaxf(st.m[hh], me + x);
+      delta[hh] = mn == -INFINITY ? 0.0f : mn - me;
       corr[hh] = fast_exp2(st.m[hh] - mn);
       st.m[hh] = mn;
       st.l[hh] *= corr[hh];
@@ -343,6 +357,13 @@ __device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, c
     st.zv[1] *= corr[1];
     st.zv[2] *= corr[0];
     st.zv[3] *= corr[1];
+#pragma unroll
+    for (int bi = 0; bi < NB; ++bi)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        t[bi][j][0] -= delta[0];
+        t[bi][j][1] -= delta[1];
+      }
   }
 #pragma unroll
   for (int bi = 0; bi < NB; ++bi)
@@ -351,18 +372,23 @@ __device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, c
 #pragma unroll
       for (int rh = 0; rh < 2; ++rh) {
         const int j = 2 * mt + rh;
-        const float p0 = fast_exp2(sc[bi][j][0] - st.m[0]);
-        const float p1 = fast_exp2(sc[bi][j][1] - st.m[1]);
+        const float p0 = fast_exp2(t[bi][j][0]);
+        const float p1 = fast_exp2(t[bi][j][1]);
         const __half2 h = __floats2half2_rn(p0, p1);
-        const float2 hf = __half22float2(h);
         if constexpr (kCompact) {
-          st.l[0] += hf.x;
-          st.l[1] += hf.y;
+          if constexpr (kSumL) {
+            const float2 hf = __half22float2(h);
+            st.l[0] += hf.x;
+            st.l[1] += hf.y;
+          }
           pt[bi][mt][rh] = movmatrix_t(kWide || ln.tig < 2 ? h2u(h) : 0u);
           continue;
         }
-        st.l[0] += p0;
-        st.l[1] += p1;
+        if constexpr (kSumL) {
+          st.l[0] += p0;
+          st.l[1] += p1;
+        }
+        const float2 hf = __half22float2(h);
         if constexpr (kWide) {
           pt[bi][mt][rh] = movmatrix_t(h2u(h));
           pl[bi][mt][rh] = movmatrix_t(h2u(__floats2half2_rn(p0 - hf.x, p1 - hf.y)));
@@ -373,6 +399,10 @@ __device__ __forceinline__ void tc_softmax(float (&sc)[NB][4][2], TcState& st, c
         }
       }
 }
+
+// Offset subtracted from a lane's scores before its softmax update: its
+// running maximum, or 0 before the first block.
+__device__ __forceinline__ float m_offset(float m) { return m == -INFINITY ? 0.0f : m; }
 
 // NB packed 32-token blocks (pages in shared memory) for one warp: scores of
 // all blocks, one softmax update, then the value MMAs.  Narrow: one MMA per
@@ -397,6 +427,14 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
   // K slots of k-step ks: lane tig's slots (2tig, 2tig+1) and (2tig+8, 2tig+9)
   // hold channels 16ks + 4tig + (0, 1) and (2, 3), so its four channels are
   // contiguous (one 16-byte load of codes and one of scale/zero).
+  // 1-bit codes in the wide layout scale the A operand instead of B: the
+  // code of row j is 0 or 2^e_j (e_j = -14, -13, -11, -7), so A = code * s is
+  // one fp16 multiply per register and exact unless it falls below the
+  // normal range (s < 2^(-14 - e_j), e.g. s < 1 on row 0), where it is
+  // rounded to a subnormal: at most 2^-25 * 2^-e_j <= 2^-11 in key units,
+  // far below the quantization step s / 2.  B = q then needs no high/low
+  // split, which halves the key MMAs (the tensor pipe bounds this layout).
+  constexpr bool kScaledA = BK == 1 && kWide;
   float dk[NB][2][4] = {};
   float dz[4] = {};  // zero-point term: row bi of the MMA = block bi
 #pragma unroll
@@ -424,7 +462,16 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
         a1[2 * half] = v[2];
         a1[2 * half + 1] = v[3];
         const uint32_t s2 = half ? sw.y : sw.x;
-        if constexpr (kWide) {
+        if constexpr (kScaledA) {
+          // 1-bit codes, wide layout: A = code * s (a power of two times the
+          // scale, or 0) and B = q, one MMA per tile
+#pragma unroll
+          for (int i = 0; i < 2; ++i) {
+            a0[2 * half + i] = h2u(__hmul2(u2h(a0[2 * half + i]), u2h(s2)));
+            a1[2 * half + i] = h2u(__hmul2(u2h(a1[2 * half + i]), u2h(s2)));
+          }
+          b[half] = qb[2 * ks + half];
+        } else if constexpr (kWide) {
           // q*s as its fp16 high part and exact residual, two operands
           const __half2 hi = __hmul2(u2h(qb[2 * ks + half]), u2h(s2));
           b[half] = h2u(hi);
@@ -439,7 +486,7 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
       }
       mma16816(dk[bi][0], a0[0], a0[1], a0[2], a0[3], b[0], b[1]);
       mma16816(dk[bi][1], a1[0], a1[1], a1[2], a1[3], b[0], b[1]);
-      if constexpr (kWide) {
+      if constexpr (kWide && !kScaledA) {
         mma16816(dk[bi][0], a0[0], a0[1], a0[2], a0[3], bl[0], bl[1]);
         mma16816(dk[bi][1], a1[0], a1[1], a1[2], a1[3], bl[0], bl[1]);
       }
@@ -447,13 +494,16 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
     const uint2 zw = *reinterpret_cast<const uint2*>(zrow + 2 * (kHeadDim + c));
     mma16816(dz, zw.x, 0u, zw.y, 0u, qb[2 * ks], qb[2 * ks + 1]);
   }
-  // Scores in the log2 domain.  Narrow: lanes tig and tig^2 hold the two
-  // parts; wide: the accumulator holds the whole score.
+  // Scores in the log2 domain, less the running maximum (one fma each: the
+  // zero-point term and the offset are folded into the addend).  Narrow:
+  // lanes tig and tig^2 hold the two parts; wide: the accumulator holds the
+  // whole score.
   float sc[NB][4][2];
+  const float me0 = m_offset(st.m[0]), me1 = m_offset(st.m[1]);
 #pragma unroll
   for (int bi = 0; bi < NB; ++bi) {
-    const float z0 = __shfl_sync(0xffffffffu, dz[0], 4 * bi + tig) * scale_log2;
-    const float z1 = __shfl_sync(0xffffffffu, dz[1], 4 * bi + tig) * scale_log2;
+    const float z0 = fmaf(__shfl_sync(0xffffffffu, dz[0], 4 * bi + tig), scale_log2, -me0);
+    const float z1 = fmaf(__shfl_sync(0xffffffffu, dz[1], 4 * bi + tig), scale_log2, -me1);
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
@@ -469,12 +519,15 @@ __device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char*
 
   constexpr bool kCompact = BV == 1;
   uint32_t pt[NB][2][2], pl[NB][2][2];
-  tc_softmax<NB, kWide, kCompact>(sc, st, ln, pt, pl);
+  tc_softmax<NB, kWide, kCompact, false>(sc, st, ln, pt, pl);
 
   // ---- values: o^T[c][h] ----
   // Value scales and zeros are stored in token pairs (t, t + 4), so the
   // B-operand scale of (k-step ks, dl) is word 2ks + dl of the lane's 8-token
-  // run; zero-point MMA rows 0..3 = groups (lane groups gid >= 4 read zeros).
+  // run; zero-point MMA rows 0..3 = groups, row 4 = ones (the lanes of gid 4
+  // read bytes 256..319 of the zero area), so it accumulates the row sum of
+  // the weights; rows 5..7 read zeros.  (In the key zero-point MMA above the
+  // rows past NB read the same area; their results are never used.)
 #pragma unroll
   for (int bi = 0; bi < NB; ++bi) {
     const char* vc = pg[bi] + page_off_vcodes(BK);
@@ -645,6 +698,11 @@ __device__ __forceinline__ void tc_write_state(const TcState& st, WarpState& ws,
   float zsum[2];
   zsum[0] = kWide ? st.zv[0] : st.zv[0] + __shfl_xor_sync(0xffffffffu, st.zv[0], 2);
   zsum[1] = kWide ? st.zv[1] : st.zv[1] + __shfl_xor_sync(0xffffffffu, st.zv[1], 2);
+  if constexpr (kPacked) {
+    // packed blocks: the row sum is row 4 of the value zero-point MMA
+    l0 += __shfl_sync(0xffffffffu, zsum[0], 16 + tig);
+    l1 += __shfl_sync(0xffffffffu, zsum[1], 16 + tig);
+  }
   if (gid == 0 && (kWide || tig < 2)) {
     ws.m[2 * tig] = st.m[0];
     ws.m[2 * tig + 1] = st.m[1];
@@ -720,6 +778,7 @@ __device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
       mma16816(dk[mt], a[0], a[1], a[2], a[3], qb[2 * ks], qb[2 * ks + 1]);
     }
   float sc[1][4][2];
+  const float me[2] = {m_offset(st.m[0]), m_offset(st.m[1])};
 #pragma unroll
   for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
@@ -727,9 +786,9 @@ __device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
       const bool ok = 16 * mt + ln.gid + 8 * rh < n_tok;
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh)
-        sc[0][2 * mt + rh][hh] = ok ? dk[mt][2 * rh + hh] * scale_log2 : -INFINITY;
+        sc[0][2 * mt + rh][hh] = ok ? fmaf(dk[mt][2 * rh + hh], scale_log2, -me[hh]) : -INFINITY;
     }
-  tc_softmax<1, kWide, kCompact>(sc, st, ln, pt, pl);
+  tc_softmax<1, kWide, kCompact, true>(sc, st, ln, pt, pl);
 }
 
 template <bool kWide, bool kCompact>
@@ -1126,10 +1185,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     const int wbytes = warp_ring_bytes(page);
     char* ring = reinterpret_cast<char*>(smem) + (size_t)warp * wbytes;
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kWarps * wbytes) + warp * R;
-    // 512 zero bytes at the end of shared memory: metadata rows of the
-    // zero-point MMAs that carry no block.
+    // 512 bytes at the end of shared memory: metadata rows of the
+    // zero-point MMAs that carry no block, all zero except bytes 256..319,
+    // which only the value zero-point MMA's row 4 reads: fp16 ones, so that
+    // row sums the softmax weights (the row sum l).
     unsigned* zero = reinterpret_cast<unsigned*>(smem + smem_size - 16 - kZeroBytes);
-    for (int i = threadIdx.x; i < kZeroBytes / 4; i += kThreads) zero[i] = 0u;
+    for (int i = threadIdx.x; i < kZeroBytes / 4; i += kThreads)
+      zero[i] = i >= kOnesWord0 && i < kOnesWord0 + 16 ? 0x3C003C00u : 0u;
     int hint = 0;
     if (lane == 0) {
       for (int i = 0; i < R; ++i) mbar_init(full + i, 1);
