@@ -219,34 +219,31 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache,
                     void* stream);
 
 /*
- * Split-K workspace for kvq_decode_attn / kvq_decode_step: per (sequence,
- * query head, split) partial max, sum and fp32 output row for the n_splits
- * CTAs of one call, plus one ticket per (sequence, kv-head) (the size allows
- * one per query head).  n_splits = 0 means the library's choice.  Returns 0
- * on an invalid config.
+ * Split-K workspace for kvq_decode_attn / kvq_decode_step with the given
+ * n_splits (see kvq_decode_attn: > 0 the split plan, 0 the flat plan): a
+ * partial max, sum and fp32 output row per query head for every CTA of the
+ * launch and two per (sequence, kv-head) pair, one ticket per pair and one
+ * counter.  Returns 0 on an invalid config or n_splits outside [0, 255].
  */
 size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits);
 
 /*
- * The split count kvq_decode_attn uses when passed n_splits = 0: one
- * 512-thread CTA per SM over all (sequence, kv-head) pairs,
- * SMs / (batch * n_kv_heads), between 1 and 255.
+ * The split plan's count for one wave: one 512-thread CTA per SM over all
+ * (sequence, kv-head) pairs, SMs / (batch * n_kv_heads), between 1 and 255
+ * (capped at a quarter of the blocks of max_len).
  */
 int32_t kvq_attn_default_splits(const kvq_config* cfg);
 
 /*
- * A split count for kvq_decode_attn / kvq_decode_step from the sequence
+ * The n_splits to pass kvq_decode_attn / kvq_decode_step for the sequence
  * lengths, which the caller knows on the host (the library keeps them on the
  * device).  lengths: host int32 [batch], each in [0, max_len].
- *   Pairs (sequence, kv-head) filling at most half the SMs: one wave of
- *   kvq_attn_default_splits, unless up to four waves of shorter splits fill
- *   the SMs that one wave leaves idle and are estimated at least 2% faster
- *   (waves x (32-token blocks per split + 46), 46 blocks being a CTA's
- *   measured fixed cost).
- *   More pairs: kvq_attn_default_splits when the longest length is within
- *   15% of the mean, else about four waves of CTAs (a ragged batch is
- *   balanced by the CTA scheduler).
- * Returns 0 on an invalid argument.
+ *   kvq_attn_default_splits (the split plan) when one wave of its CTAs fills
+ *   at least 90% of the GPU, as for batch-1 decoding, where a launch is
+ *   bound by latency and dedicated window warps keep the fp16 chunks off the
+ *   block warps' path; otherwise 0, the flat plan, which streams every pair
+ *   in one wave (no CTA start and merges per wave).
+ * Returns -1 on an invalid argument.
  */
 int32_t kvq_attn_splits_for_lengths(const kvq_config* cfg, const int32_t* lengths);
 
@@ -267,11 +264,17 @@ kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream);
  *   q              device fp16 [batch][n_q_heads][128], 16-byte aligned.
  *   out            device fp16 [batch][n_q_heads][128], 16-byte aligned.
  *   softmax_scale  0 selects 1/sqrt(128).
- *   n_splits       CTAs per (sequence, kv-head) that share its 32-token
- *                  blocks and window chunks; 0 = kvq_attn_default_splits(cfg);
- *                  else 1..255.  With more than one, each CTA writes a partial
- *                  (max, sum, output row) to the workspace and the last to
- *                  finish merges them.
+ *   n_splits       the work plan.  1..255: the split plan, n_splits CTAs per
+ *                  (sequence, kv-head) pair share its 32-token blocks
+ *                  (contiguous ranges, one per warp) and its window chunks
+ *                  (dedicated warps).  0: the flat plan, one CTA per SM; all
+ *                  pairs' blocks and window chunks lie end to end, weighted
+ *                  by their measured cost, and every warp takes an equal
+ *                  contiguous share, crossing pair boundaries as it goes.
+ *                  Either way a pair's CTAs (and a warp that leaves a pair
+ *                  for the next) write partials (max, sum, output row) to the
+ *                  workspace and the last to finish merges them; a pair with
+ *                  a single partial is written directly.
  *   workspace      device, >= kvq_attn_workspace_bytes(cfg, n_splits), zeroed
  *                  once by kvq_workspace_init.
  * A sequence with L = 0 gets a zero output.  Calls that share a workspace

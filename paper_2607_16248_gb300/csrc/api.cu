@@ -145,6 +145,17 @@ static int default_splits(const kvq_config& c) {
   return attn_default_splits(make_dims(c), sm_count());
 }
 
+// n_splits as the launchers take it: > 0 the split plan, 0 -> the flat plan
+// on one CTA per resident slot (a negative count).
+static int resolve_splits(int32_t n_splits) {
+  return n_splits == 0 ? -attn_flat_ctas(sm_count()) : n_splits;
+}
+// Workspace bytes of a resolved n_splits.
+static size_t attn_ws_bytes(const Dims& d, int n_splits) {
+  return n_splits > 0 ? attn_split_workspace_bytes(d, n_splits)
+                      : attn_workspace_bytes(d, -n_splits);
+}
+
 }  // namespace kvq
 
 using namespace kvq;
@@ -272,15 +283,15 @@ kvq_status kvq_pack(const kvq_config* cfg, const kvq_cache* cache, const uint16_
 }
 
 int32_t kvq_attn_splits_for_lengths(const kvq_config* cfg, const int32_t* lengths) {
-  if (check_config(cfg) != KVQ_OK) return 0;
+  if (check_config(cfg) != KVQ_OK) return -1;
   if (!lengths) {
     fail(KVQ_ERR_ARG, "lengths is NULL");
-    return 0;
+    return -1;
   }
   for (int b = 0; b < cfg->batch; ++b)
     if (lengths[b] < 0 || lengths[b] > cfg->max_len) {
       fail(KVQ_ERR_ARG, "lengths[%d] = %d outside [0, max_len]", b, lengths[b]);
-      return 0;
+      return -1;
     }
   return attn_splits_for_lengths(make_dims(*cfg), sm_count(), lengths);
 }
@@ -292,12 +303,11 @@ int32_t kvq_attn_default_splits(const kvq_config* cfg) {
 
 size_t kvq_attn_workspace_bytes(const kvq_config* cfg, int32_t n_splits) {
   if (check_config(cfg) != KVQ_OK) return 0;
-  if (n_splits == 0) n_splits = default_splits(*cfg);
-  if (n_splits < 1 || n_splits > kMaxSplits - 1) {
-    set_error("n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, n_splits);
+  if (n_splits < 0 || n_splits > kMaxSplits - 1) {
+    set_error("n_splits must be in [0, %d] (got %d)", kMaxSplits - 1, n_splits);
     return 0;
   }
-  return attn_workspace_bytes(make_dims(*cfg), n_splits);
+  return attn_ws_bytes(make_dims(*cfg), resolve_splits(n_splits));
 }
 
 kvq_status kvq_workspace_init(void* workspace, size_t ws_bytes, void* stream) {
@@ -324,10 +334,10 @@ static kvq_status check_attn_call(const kvq_config* cfg, const kvq_cache* cache,
   if (!aligned16(q) || !aligned16(out)) return fail(KVQ_ERR_ALIGN, "q / out must be 16-byte aligned");
   if (!(softmax_scale >= 0.0f) || isinf(softmax_scale))
     return fail(KVQ_ERR_ARG, "softmax_scale must be finite and >= 0");
-  if (*n_splits == 0) *n_splits = default_splits(*cfg);
-  if (*n_splits < 1 || *n_splits > kMaxSplits - 1)
-    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, *n_splits);
-  const size_t need = attn_workspace_bytes(make_dims(*cfg), *n_splits);
+  if (*n_splits < 0 || *n_splits > kMaxSplits - 1)
+    return fail(KVQ_ERR_ARG, "n_splits must be in [0, %d] (got %d)", kMaxSplits - 1, *n_splits);
+  *n_splits = resolve_splits(*n_splits);
+  const size_t need = attn_ws_bytes(make_dims(*cfg), *n_splits);
   if (!workspace) return fail(KVQ_ERR_ARG, "workspace is NULL");
   if (!aligned16(workspace)) return fail(KVQ_ERR_ALIGN, "workspace must be 16-byte aligned");
   if (ws_bytes < need)
@@ -345,12 +355,17 @@ static kvq_status decode_attn(const kvq_config* cfg, const kvq_cache* cache, con
                                  ws_bytes, &sl2);
   if (s != KVQ_OK) return s;
   Dims d = make_dims(*cfg);
-  trace("kvq_decode_attn%s batch %d heads %d/%d bits K%dV%d grid (%d, %d, %d) x 512, %d splits",
-        out_f16 ? "" : "_f32", d.batch, d.hq, d.hkv, d.bits_k, d.bits_v, n_splits, d.hkv,
-        d.batch, n_splits);
-  return cuda_status(launch_decode_attn(d, *cache, reinterpret_cast<const __half*>(q), out,
-                                        out_f16, sl2, n_splits, workspace,
-                                        static_cast<cudaStream_t>(stream)),
+  trace("kvq_decode_attn%s batch %d heads %d/%d bits K%dV%d grid (%d) x 512, %s %d",
+        out_f16 ? "" : "_f32", d.batch, d.hq, d.hkv, d.bits_k, d.bits_v,
+        n_splits > 0 ? n_splits * d.batch * d.hkv : -n_splits,
+        n_splits > 0 ? "splits" : "flat plan, CTAs", n_splits > 0 ? n_splits : -n_splits);
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const __half* qh = reinterpret_cast<const __half*>(q);
+  return cuda_status(n_splits > 0
+                         ? launch_decode_attn_split(d, *cache, qh, out, out_f16, sl2, n_splits,
+                                                    workspace, st)
+                         : launch_decode_attn(d, *cache, qh, out, out_f16, sl2, -n_splits,
+                                              workspace, st),
                      "kvq_decode_attn launch");
 }
 
@@ -366,13 +381,19 @@ static kvq_status decode_step(const kvq_config* cfg, const kvq_cache* cache,
                                  ws_bytes, &sl2);
   if (s != KVQ_OK) return s;
   Dims d = make_dims(*cfg);
-  trace("kvq_decode_step%s batch %d heads %d/%d bits K%dV%d grid (%d, %d, %d) x 512, %d splits",
-        out_f16 ? "" : "_f32", d.batch, d.hq, d.hkv, d.bits_k, d.bits_v, n_splits, d.hkv,
-        d.batch, n_splits);
-  return cuda_status(launch_decode_step(d, *cache, reinterpret_cast<const __half*>(k_new),
-                                        reinterpret_cast<const __half*>(v_new),
-                                        reinterpret_cast<const __half*>(q), out, out_f16, sl2,
-                                        n_splits, workspace, static_cast<cudaStream_t>(stream)),
+  trace("kvq_decode_step%s batch %d heads %d/%d bits K%dV%d grid (%d) x 512, %s %d",
+        out_f16 ? "" : "_f32", d.batch, d.hq, d.hkv, d.bits_k, d.bits_v,
+        n_splits > 0 ? n_splits * d.batch * d.hkv : -n_splits,
+        n_splits > 0 ? "splits" : "flat plan, CTAs", n_splits > 0 ? n_splits : -n_splits);
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const __half* kh = reinterpret_cast<const __half*>(k_new);
+  const __half* vh = reinterpret_cast<const __half*>(v_new);
+  const __half* qh = reinterpret_cast<const __half*>(q);
+  return cuda_status(n_splits > 0
+                         ? launch_decode_step_split(d, *cache, kh, vh, qh, out, out_f16, sl2,
+                                                    n_splits, workspace, st)
+                         : launch_decode_step(d, *cache, kh, vh, qh, out, out_f16, sl2,
+                                              -n_splits, workspace, st),
                      "kvq_decode_step launch");
 }
 
@@ -418,11 +439,11 @@ kvq_status kvq_decode_attn_noalloc(const kvq_config* cfg, const kvq_cache* cache
   if (!aligned16(q) || !aligned16(out)) return fail(KVQ_ERR_ALIGN, "q / out must be 16-byte aligned");
   if (!(softmax_scale >= 0.0f) || isinf(softmax_scale))
     return fail(KVQ_ERR_ARG, "softmax_scale must be finite and >= 0");
-  if (n_splits == 0) n_splits = default_splits(*cfg);
-  if (n_splits < 1 || n_splits > kMaxSplits - 1)
-    return fail(KVQ_ERR_ARG, "n_splits must be in [1, %d] (got %d)", kMaxSplits - 1, n_splits);
+  if (n_splits < 0 || n_splits > kMaxSplits - 1)
+    return fail(KVQ_ERR_ARG, "n_splits must be in [0, %d] (got %d)", kMaxSplits - 1, n_splits);
+  n_splits = resolve_splits(n_splits);
   Dims d = make_dims(*cfg);
-  const size_t need = attn_workspace_bytes(d, n_splits);
+  const size_t need = attn_ws_bytes(d, n_splits);
   if (need > attn_static_scratch_bytes())
     return fail(KVQ_ERR_CAPACITY,
                 "this config needs %zu bytes of scratch but the built-in array holds %zu; "

@@ -50,31 +50,30 @@
 namespace kvq {
 namespace {
 
-#ifndef KVQ_ATTN_WARPS
-#define KVQ_ATTN_WARPS 16
-#endif
-constexpr int kWarps = KVQ_ATTN_WARPS;            // warps per CTA
-constexpr int kThreads = 32 * kWarps;
-constexpr int kCtasPerSm = kWarps <= 8 ? 2 : 1;   // resident CTAs per SM
-constexpr int kRingBudget = (kCtasPerSm == 2 ? 96 : 192) * 1024;  // staged page bytes per CTA
-constexpr int kHeads = kMaxGq;  // query heads per CTA (the wide layout's head columns)
-constexpr long long kWaitCycles = 4000000000LL;  // bounded mbarrier waits (~2 s)
-constexpr int kZeroBytes = 512;                   // all-zero metadata rows
-constexpr int kOnesWord0 = 64;                    // ... but for fp16 ones at bytes 256..319
+#include "attn_core.cuh"
 
+constexpr int kFinCap = 2 * kWarps + 2;           // final merges one CTA can owe (<= kWarps + 1)
+constexpr int kLenCap = 1024;                     // sequence lengths a CTA keeps in shared memory
+
+// Split partials: slots [0, ctas + P) for the CTA partials, then one warp
+// partial per pair (P = batch * n_kv_heads pairs); tickets: one per pair,
+// then the decode step's count of finished CTAs.
 struct Ws {
-  float* m;       // [B][Hq][S]
-  float* l;       // [B][Hq][S]
-  float* o;       // [B][Hq][S][128]
-  unsigned* tk;   // [B][Hkv] (sized [B][Hq])
+  float* m;       // [slots][gq] row maxima (log2 domain)
+  float* l;       // [slots][gq] row sums
+  float* o;       // [slots][gq][128] unnormalised rows
+  unsigned* tk;   // [P + 1]
 };
 
 __host__ __device__ inline size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
-__host__ __device__ inline Ws carve(void* base, int batch, int hq, int hkv, int S) {
+__host__ __device__ inline size_t ws_slots(int batch, int hkv, int ctas) {
+  return (size_t)ctas + 2 * (size_t)batch * hkv;
+}
+__host__ __device__ inline Ws carve(void* base, int batch, int hq, int hkv, int ctas) {
   Ws w;
   char* p = static_cast<char*>(base);
-  const size_t nml = (size_t)batch * hq * S;
+  const size_t nml = ws_slots(batch, hkv, ctas) * (size_t)(hq / hkv);
   w.m = reinterpret_cast<float*>(p);
   p += align256(nml * 4);
   w.l = reinterpret_cast<float*>(p);
@@ -85,931 +84,304 @@ __host__ __device__ inline Ws carve(void* base, int batch, int hq, int hkv, int 
   return w;
 }
 
-// A warp's final state (row maximum, row sum, unnormalised output row per
-// query head of the kv-head), written at the start of the warp's own
-// ring as soon as it is done.
-struct WarpState {
-  float m[kHeads];
-  float l[kHeads];
-  float o[kHeads][kHeadDim];
-};
 // Small shared arrays of the merges (static shared memory).
 struct MergeSmall {
   float ww[kWarps][kHeads];             // warp merge weights 2^(m_w - M)
-  float cta_m[kHeads];
-  int last;
+  float gm[kWarps][kHeads];             // a group's maximum M
+};
+// The CTA's merge groups: warps [w0, w1) end in the same pair; cnt = the
+// pair's partials in all.
+struct MergeGroups {
+  int w0[kWarps], w1[kWarps], cnt[kWarps];
+  int n;
 };
 
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
+// ---------------------------------------------------------------------------
+// The flat work plan.  Pair p = b * Hkv + h (sequence b, kv-head h) is a list
+// of items: its packed 32-token blocks (cost 1 each), then the 32-token
+// chunks of its fp16 window (cost cw each); the first item costs sc more (a
+// warp that starts a pair waits once for its first pages).  All pairs' items
+// lie end to end in cost units, cut into n_v equal contiguous unit ranges,
+// one per virtual warp; an item belongs to the virtual warp whose range holds
+// its first unit.  The virtual warps are cut into n_cta contiguous groups of
+// at most kWarps, one per CTA.  So every warp streams one contiguous run of
+// blocks, possibly across pair boundaries, and all warps carry the same
+// cost: the launch is one wave of CTAs with no per-pair split count.
+// n_v <= units / (cw + sc) keeps every range long enough to hold the first
+// unit of an item, so no virtual warp is empty.
+//
+// Partials.  A warp keeps one softmax state per pair it touches.  The state
+// of its last pair goes to its CTA, which merges the warps that end in the
+// same pair into one CTA partial (slot cta + p, unique: CTA ranges and pair
+// ranges are both ordered).  A state of a pair the warp leaves for the next
+// one is a warp partial (slot n_slots_cta + p; at most one per pair: only the
+// owner of the pair's last item can continue past it).  Each partial bumps
+// the pair's ticket; the one that completes it merges the pair's partials
+// (pair_partials gives their number).  A pair with one partial in all is
+// written out directly.
+// ---------------------------------------------------------------------------
+
+// Cost weights: a window chunk costs cw units, the first item of a pair sc
+// more (measured: a chunk takes ~4 blocks' time, a pair start ~1).  A launch
+// with too little work for every warp to hold an item under those weights
+// takes lighter ones (FlatGrid::cw, sc), down to one unit per item.
+struct Costs {
+  int cw, sc;
+};
+
+struct PairShape {
+  int Lq, nb, nr;  // packed tokens, packed blocks, window chunks
+};
+__host__ __device__ inline PairShape pair_shape(int L, int residual) {
+  PairShape s;
+  s.Lq = packed_len(L, residual);
+  s.nb = s.Lq / kGroup;
+  s.nr = (L - s.Lq + kGroup - 1) / kGroup;
+  return s;
 }
-__device__ __forceinline__ float warp_sum(float v) {
+__host__ __device__ inline int pair_cost(const PairShape& s, Costs k) {
+  return s.nb + s.nr > 0 ? k.sc + s.nb + k.cw * s.nr : 0;
+}
+// First unit (pair-local) of item i.
+__host__ __device__ inline int item_unit(int i, int nb, Costs k) {
+  return i == 0 ? 0 : k.sc + (i < nb ? i : nb + k.cw * (i - nb));
+}
+// Number of items of a pair whose first unit (pair-local) is below x.
+__host__ __device__ inline int items_below(long long x, int nb, int nr, Costs k) {
+  if (x <= 0 || nb + nr == 0) return 0;
+  int c = 1;
+  if (nb > 1) c += (int)min((long long)(nb - 1), max(0LL, x - k.sc - 1));
+  const int lo_w = nb == 0 ? 1 : 0;
+  if (nr > lo_w) {
+    const long long t = x - k.sc - nb;
+    const int sh = k.cw == 4 ? 2 : k.cw == 2 ? 1 : 0;  // cw is 1, 2 or 4
+    const long long n = t <= 0 ? 0 : (t + k.cw - 1) >> sh;
+    c += (int)max(0LL, min(n, (long long)nr) - lo_w);
+  }
+  return c;
+}
+
+// Work totals of a launch: packed blocks, window chunks, non-empty pairs.
+struct WorkSums {
+  long long nb, nr, np;
+};
+
+// floor(x / d) from r = floor((2^64 - 1) / d): the high half of x * r is at
+// most two below the quotient (r >= 2^64 / d - 1, x < 2^64), so two checks
+// make it exact.  Integer division on the GPU is a long software sequence;
+// the plan divides by the same N and n_v many times.
+__host__ __device__ inline unsigned long long rcp64(unsigned long long d) {
+  return d ? ~0ULL / d : 0ULL;
+}
+__host__ __device__ inline long long div_rcp(unsigned long long x, unsigned long long d,
+                                             unsigned long long r) {
+#ifdef __CUDA_ARCH__
+  unsigned long long q = __umul64hi(x, r);
+#else
+  unsigned long long q = (unsigned long long)(((unsigned __int128)x * r) >> 64);
+#endif
+  if ((q + 1) * d <= x) ++q;
+  if ((q + 1) * d <= x) ++q;
+  return (long long)q;
+}
+
+struct FlatGrid {
+  long long N;               // cost units of all pairs
+  int n_v;                   // virtual warps (0 when N == 0)
+  int n_cta;                 // CTAs that carry work, <= gridDim.x
+  Costs k;                   // cost weights
+  unsigned long long rN, rV; // reciprocals of N and n_v (div_rcp)
+};
+__host__ __device__ inline FlatGrid flat_grid(const WorkSums& w, int ctas) {
+  FlatGrid g;
+  const long long cap = (long long)kWarps * ctas;
+  // the heaviest weights under which every one of the cap warps can still
+  // hold an item start (each range >= the largest item cost)
+  const Costs pick[3] = {{4, 1}, {2, 1}, {1, 0}};
+  int i = 0;
+  for (; i < 2; ++i) {
+    const long long N = w.nb + pick[i].cw * w.nr + pick[i].sc * w.np;
+    if (N / (pick[i].cw + pick[i].sc) >= cap) break;
+  }
+  g.k = pick[i];
+  g.N = w.nb + g.k.cw * w.nr + g.k.sc * w.np;
+  const long long nv = g.N / (g.k.cw + g.k.sc);
+  g.n_v = g.N == 0 ? 0 : (int)(nv < 1 ? 1 : (nv < cap ? nv : cap));
+  g.n_cta = g.n_v < ctas ? g.n_v : ctas;
+  g.rN = rcp64((unsigned long long)g.N);
+  g.rV = rcp64((unsigned long long)g.n_v);
+  return g;
+}
+__host__ __device__ inline int unit_owner(long long u, const FlatGrid& g) {
+  return (int)div_rcp((unsigned long long)(u + 1) * g.n_v - 1, g.N, g.rN);
+}
+__host__ __device__ inline long long v_first_unit(int v, const FlatGrid& g) {
+  return div_rcp((unsigned long long)g.N * v, g.n_v, g.rV);
+}
+// (n_v < 2^12 and n_cta < 2^8: 32-bit arithmetic)
+__host__ __device__ inline int cta_of(int v, const FlatGrid& g) {
+  return (int)(((unsigned)(v + 1) * (unsigned)g.n_cta - 1u) / (unsigned)g.n_v);
+}
+__host__ __device__ inline int cta_first_v(int c, const FlatGrid& g) {
+  return (int)((unsigned)g.n_v * (unsigned)c / (unsigned)g.n_cta);
+}
+// Partials of a non-empty pair (first unit U, cost C): the CTA partials of
+// CTAs [c_a, c_a + n_cta) and, if `cont`, one warp partial.
+__host__ __device__ inline int pair_partials(long long U, int C, int nb, int nr,
+                                             const FlatGrid& g, int& c_a, int& n_cta,
+                                             bool& cont) {
+  const int wf = unit_owner(U, g);
+  const int wl = unit_owner(U + item_unit(nb + nr - 1, nb, g.k), g);
+  cont = U + C < g.N && unit_owner(U + C, g) == wl;
+  const int hv = wl - (cont ? 1 : 0);
+  c_a = cta_of(wf, g);
+  n_cta = hv >= wf ? cta_of(hv, g) - c_a + 1 : 0;
+  return n_cta + (cont ? 1 : 0);
+}
+
+// Length a kernel attends: the decode step counts its own token.
+__device__ __forceinline__ int attended_len(int L0, const Dims& d, bool append) {
+  return append && L0 < d.max_len ? L0 + 1 : L0;
+}
+__device__ __forceinline__ long long warp_sum_ll(long long v) {
 #pragma unroll
   for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
-
-// ---------------------------------------------------------------------------
-// PTX helpers: mbarrier, bulk async copy, mma.sync, movmatrix
-// ---------------------------------------------------------------------------
-
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
-               "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n"
-      " mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}"
-      : "=r"(ok)
-      : "r"(smem_addr(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Wait for the phase with the given parity to complete; false after ~2 s.
-__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, long long limit) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity))
-    if (clock64() - t0 > limit) return false;
-  return true;
-}
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  return mbar_wait_for(bar, parity, kWaitCycles);
-}
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_addr(dst)),
-      "l"(src), "r"(bytes), "r"(smem_addr(bar))
-      : "memory");
-}
-__device__ __forceinline__ void fence_mbar_init() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-// Programmatic dependent launch: let the next kernel in the stream start
-// launching, and wait until the previous one has completed and its writes
-// are visible.  Both are no-ops when the kernel was launched without the
-// programmatic-serialization attribute.
-__device__ __forceinline__ void pdl_launch_dependents() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ int read_len(const int* p) {
-  return *reinterpret_cast<const volatile int*>(p);
-}
-
-__device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
-                                         uint32_t a3, uint32_t b0, uint32_t b1) {
-  asm(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ uint32_t movmatrix_t(uint32_t a) {
-  uint32_t d;
-  asm("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
-  return d;
-}
-
-// 2^x with the SFU (x <= 0 here; -inf gives +0).
-__device__ __forceinline__ float fast_exp2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-__device__ __forceinline__ uint32_t h2u(__half2 h) { return *reinterpret_cast<uint32_t*>(&h); }
-__device__ __forceinline__ __half2 u2h(uint32_t u) { return *reinterpret_cast<__half2*>(&u); }
-__device__ __forceinline__ uint32_t hsub1024(uint32_t x) {
-  return h2u(__hsub2(u2h(x), u2h(0x64006400u)));
-}
-
-// ---------------------------------------------------------------------------
-// Tensor-core path for packed blocks (query groups of up to 4 heads).
-// Lane = 4 * gid + tig (mma fragment coordinates).
-// ---------------------------------------------------------------------------
-
-// Codes of four rows j = 0..3 of a lane (tokens 4*gid + j for keys, channels
-// 4*gid + j of a 32-channel group for values) from two packed words a, b (two
-// channels for keys, two tokens for values): v[j] = (f_j code_a, f_j code_b)
-// as fp16, exact.  inv(j) = 1 / f_j.
-template <int B>
-struct Codes;
-
-// 1-bit codes are stored in fragment order (key1_bit / val1_bit): the word
-// w of a lane rotated left by 4 r holds, at bit 10 + 16 e + j, the code of
-// row j and half e of one fragment register, so each register is one AND
-// (an fp16 with a single exponent bit set: 2^-14, 2^-13, 2^-11, 2^-7).
-template <>
-struct Codes<1> {
-  __device__ static constexpr float inv(int j) {
-    return j == 0 ? 16384.0f : j == 1 ? 8192.0f : j == 2 ? 2048.0f : 128.0f;
-  }
-  __device__ static int word(int gid) { return 0; }
-  __device__ static void rot(uint32_t w, int r, uint32_t (&v)[4]) {
-    // r = 1, 2 only read bits that a plain shift keeps; r = 3 wraps around.
-    const uint32_t y = r == 0 ? w : r == 1 ? w << 4 : r == 2 ? w << 8 : __funnelshift_l(w, w, 12);
-    v[0] = y & 0x04000400u;
-    v[1] = y & 0x08000800u;
-    v[2] = y & 0x10001000u;
-    v[3] = y & 0x20002000u;
-  }
-};
-
-__device__ __forceinline__ uint32_t comp(const uint4& u, int i) {
-  return i == 0 ? u.x : i == 1 ? u.y : i == 2 ? u.z : u.w;
-}
-template <>
-struct Codes<2> {
-  __device__ static constexpr float inv(int j) {
-    return j == 0 ? 1.0f : j == 1 ? 0.25f : j == 2 ? 0.0625f : 0.015625f;
-  }
-  __device__ static int word(int gid) { return gid >> 2; }
-  __device__ static void get(uint32_t a, uint32_t b, uint32_t sel, uint32_t (&v)[4]) {
-    const uint32_t x = __byte_perm(a, b, sel);  // the lane's byte -> bits 0..7 of each half
-#pragma unroll
-    for (int j = 0; j < 4; ++j) v[j] = hsub1024((x & (0x00030003u << (2 * j))) | 0x64006400u);
-  }
-};
-template <>
-struct Codes<4> {
-  __device__ static constexpr float inv(int j) { return (j & 1) ? 0.0625f : 1.0f; }
-  __device__ static int word(int gid) { return gid >> 1; }
-  __device__ static void get(uint32_t a, uint32_t b, uint32_t sel, uint32_t (&v)[4]) {
-    const uint32_t x = __byte_perm(a, b, sel);  // the lane's 16 bits -> each half
-    const uint32_t y = x >> 8;
-    v[0] = hsub1024((x & 0x000F000Fu) | 0x64006400u);
-    v[1] = hsub1024((x & 0x00F000F0u) | 0x64006400u);
-    v[2] = hsub1024((y & 0x000F000Fu) | 0x64006400u);
-    v[3] = hsub1024((y & 0x00F000F0u) | 0x64006400u);
-  }
-};
-template <>
-struct Codes<8> {
-  __device__ static constexpr float inv(int) { return 1.0f; }
-  __device__ static int word(int gid) { return gid; }
-  __device__ static void get(uint32_t a, uint32_t b, uint32_t, uint32_t (&v)[4]) {
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t x = __byte_perm(a, b, j | (j << 4) | ((4 + j) << 8) | ((4 + j) << 12));
-      v[j] = hsub1024((x & 0x00FF00FFu) | 0x64006400u);
-    }
-  }
-};
-
-template <int B>
-__device__ __forceinline__ uint32_t code_selector(int gid) {
-  int k;
-  if (B == 1) k = gid >> 1;
-  else if (B == 2) k = gid & 3;
-  else if (B == 4) {
-    const int kk = gid & 1;
-    return (2 * kk) | ((2 * kk + 1) << 4) | ((4 + 2 * kk) << 8) | ((5 + 2 * kk) << 12);
-  } else k = 0;
-  return k | (k << 4) | ((4 + k) << 8) | ((4 + k) << 12);
-}
-
-struct Lane {
-  int gid, tig;
-  uint32_t sel_k, sel_v;   // byte-permute selectors for key / value words
-  int wk, wv;               // word of a group that holds the lane's 4 codes
-  uint32_t neg_lo;          // fp16x2 -1 for lanes holding B columns 4..7, else 0
-  float p_lo;               // 1 for lanes holding score columns 4..7
-};
-
-struct TcState {
-  float acc[8][4];  // o^T[channel][head, part] per value m-tile
-  float zv[4];      // sum_t p z per (group, head, part)
-  float m[2], l[2]; // heads 2*(tig&1) + {0, 1}
-};
-
-// Online softmax over NB 32-token blocks (per block 4 token rows x 2 heads
-// per lane), then the probabilities moved to the B-operand layout of the
-// value MMAs with movmatrix.  The scores arrive as t = score - m_eff (log2
-// domain), m_eff being the lane's running maximum (0 before its first
-// block), so the common case (no score above the maximum) costs one exp2 per
-// score and a vote; only when some score exceeds it (or before the first
-// block) is the new maximum found across the warp, the state rescaled and t
-// shifted.
-//   exact (kCompact false): p as an fp16 high part and its fp16 residual;
-//     narrow (up to 4 heads): columns 0..3 / 4..7 hold the high / low parts
-//     of heads 0..3 (lanes tig and tig^2 hold the same scores), pt is one
-//     operand whose columns carry both parts; wide (5..8 heads): column =
-//     head, pt holds the high parts, pl the low parts, each one operand of
-//     its own MMA.
-//   compact (1-bit values): the weights are p~ = RN16(p), used alike in the
-//     row sum and in the value MMAs (so they are a consistent softmax of
-//     scores perturbed by at most 2^-11 relative); pt holds p~ (column =
-//     head; narrow: columns 4..7 zero), pl is unused.
-// kSumL: add the weights to st.l here (window chunks).  Packed blocks leave
-// it: their row sums come out of the value zero-point MMA, whose A row 4 is
-// all ones (see tc_unit).
-template <int NB, bool kWide, bool kCompact, bool kSumL>
-__device__ __forceinline__ void tc_softmax(float (&t)[NB][4][2], TcState& st, const Lane& ln,
-                                           uint32_t (&pt)[NB][2][2], uint32_t (&pl)[NB][2][2]) {
-  float tm[2];
-#pragma unroll
-  for (int hh = 0; hh < 2; ++hh) {
-    float x = -INFINITY;
-#pragma unroll
-    for (int bi = 0; bi < NB; ++bi)
-      x = fmaxf(x, fmaxf(fmaxf(t[bi][0][hh], t[bi][1][hh]), fmaxf(t[bi][2][hh], t[bi][3][hh])));
-    tm[hh] = x;
-  }
-  const bool fresh = st.m[0] == -INFINITY;
-  if (__any_sync(0xffffffffu, tm[0] > 0.0f || tm[1] > 0.0f || fresh)) {
-    float corr[2], delta[2];
-#pragma unroll
-    for (int hh = 0; hh < 2; ++hh) {
-      float x = tm[hh];
-      x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 4));
-      x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 8));
-      x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16));
-      const float me = st.m[hh] == -INFINITY ? 0.0f : st.m[hh];
-      const float mn = fmaxf(st.m[hh], me + x);
-      delta[hh] = mn == -INFINITY ? 0.0f : mn - me;
-      corr[hh] = fast_exp2(st.m[hh] - mn);
-      st.m[hh] = mn;
-      st.l[hh] *= corr[hh];
-    }
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      st.acc[i][0] *= corr[0];
-      st.acc[i][1] *= corr[1];
-      st.acc[i][2] *= corr[0];
-      st.acc[i][3] *= corr[1];
-    }
-    st.zv[0] *= corr[0];
-    st.zv[1] *= corr[1];
-    st.zv[2] *= corr[0];
-    st.zv[3] *= corr[1];
-#pragma unroll
-    for (int bi = 0; bi < NB; ++bi)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        t[bi][j][0] -= delta[0];
-        t[bi][j][1] -= delta[1];
-      }
-  }
-#pragma unroll
-  for (int bi = 0; bi < NB; ++bi)
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int rh = 0; rh < 2; ++rh) {
-        const int j = 2 * mt + rh;
-        const float p0 = fast_exp2(t[bi][j][0]);
-        const float p1 = fast_exp2(t[bi][j][1]);
-        const __half2 h = __floats2half2_rn(p0, p1);
-        if constexpr (kCompact) {
-          if constexpr (kSumL) {
-            const float2 hf = __half22float2(h);
-            st.l[0] += hf.x;
-            st.l[1] += hf.y;
-          }
-          pt[bi][mt][rh] = movmatrix_t(kWide || ln.tig < 2 ? h2u(h) : 0u);
-          continue;
-        }
-        if constexpr (kSumL) {
-          st.l[0] += p0;
-          st.l[1] += p1;
-        }
-        const float2 hf = __half22float2(h);
-        if constexpr (kWide) {
-          pt[bi][mt][rh] = movmatrix_t(h2u(h));
-          pl[bi][mt][rh] = movmatrix_t(h2u(__floats2half2_rn(p0 - hf.x, p1 - hf.y)));
-        } else {
-          const __half2 r =
-              __floats2half2_rn(fmaf(-ln.p_lo, hf.x, p0), fmaf(-ln.p_lo, hf.y, p1));
-          pt[bi][mt][rh] = movmatrix_t(h2u(r));
-        }
-      }
-}
-
-// Offset subtracted from a lane's scores before its softmax update: its
-// running maximum, or 0 before the first block.
-__device__ __forceinline__ float m_offset(float m) { return m == -INFINITY ? 0.0f : m; }
-
-// NB packed 32-token blocks (pages in shared memory) for one warp: scores of
-// all blocks, one softmax update, then the value MMAs.  Narrow: one MMA per
-// operand pair, B columns = (head, part); wide: B column = head, and the
-// high and low parts of B are two MMAs into the same accumulator.
-template <int BK, int BV, int NB, bool kWide>
-__device__ __forceinline__ void tc_unit(const char* const (&pg)[NB], const char* zero,
-                                        const uint32_t (&qb)[16], const Lane& ln,
-                                        float scale_log2, TcState& st) {
-  const int gid = ln.gid, tig = ln.tig, lane = 4 * gid + tig;
-  // Zero-point MMA rows: row bi (lane group gid = bi) reads block bi's key
-  // metadata, the other rows the all-zero area (same 512-byte extent).
-  const char* zrow = gid == 0 ? pg[0] + page_off_kmeta(BK)
-                     : (NB == 2 && gid == 1) ? pg[NB - 1] + page_off_kmeta(BK) : zero;
-  uint4 kw1[NB];
-  if constexpr (BK == 1) {
-#pragma unroll
-    for (int bi = 0; bi < NB; ++bi) kw1[bi] = *reinterpret_cast<const uint4*>(pg[bi] + 16 * lane);
-  }
-
-  // ---- keys: S[t][h] ----
-  // K slots of k-step ks: lane tig's slots (2tig, 2tig+1) and (2tig+8, 2tig+9)
-  // hold channels 16ks + 4tig + (0, 1) and (2, 3), so its four channels are
-  // contiguous (one 16-byte load of codes and one of scale/zero).
-  // 1-bit codes in the wide layout scale the A operand instead of B: the
-  // code of row j is 0 or 2^e_j (e_j = -14, -13, -11, -7), so A = code * s is
-  // one fp16 multiply per register and exact unless it falls below the
-  // normal range (s < 2^(-14 - e_j), e.g. s < 1 on row 0), where it is
-  // rounded to a subnormal: at most 2^-25 * 2^-e_j <= 2^-11 in key units,
-  // far below the quantization step s / 2.  B = q then needs no high/low
-  // split, which halves the key MMAs (the tensor pipe bounds this layout).
-  constexpr bool kScaledA = BK == 1 && kWide;
-  float dk[NB][2][4] = {};
-  float dz[4] = {};  // zero-point term: row bi of the MMA = block bi
-#pragma unroll
-  for (int ks = 0; ks < 8; ++ks) {
-    const int c = 16 * ks + 4 * tig;
-#pragma unroll
-    for (int bi = 0; bi < NB; ++bi) {
-      const char* kc = pg[bi];
-      const char* kmeta = pg[bi] + page_off_kmeta(BK);
-      // scales of channels c..c+3 (two fp16 per word)
-      const uint2 sw = *reinterpret_cast<const uint2*>(kmeta + 2 * c);
-      uint32_t a0[4], a1[4], b[2], bl[2];
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        uint32_t v[4];
-        if constexpr (BK == 1) {
-          Codes<1>::rot(comp(kw1[bi], ks >> 1), 2 * (ks & 1) + half, v);
-        } else {
-          const uint32_t wa = *reinterpret_cast<const uint32_t*>(kc + 4 * ((c + 2 * half) * BK + ln.wk));
-          const uint32_t wb = *reinterpret_cast<const uint32_t*>(kc + 4 * ((c + 2 * half + 1) * BK + ln.wk));
-          Codes<BK>::get(wa, wb, ln.sel_k, v);
-        }
-        a0[2 * half] = v[0];
-        a0[2 * half + 1] = v[1];
-        a1[2 * half] = v[2];
-        a1[2 * half + 1] = v[3];
-        const uint32_t s2 = half ? sw.y : sw.x;
-        if constexpr (kScaledA) {
-          // 1-bit codes, wide layout: A = code * s (a power of two times the
-          // scale, or 0) and B = q, one MMA per tile
-#pragma unroll
-          for (int i = 0; i < 2; ++i) {
-            a0[2 * half + i] = h2u(__hmul2(u2h(a0[2 * half + i]), u2h(s2)));
-            a1[2 * half + i] = h2u(__hmul2(u2h(a1[2 * half + i]), u2h(s2)));
-          }
-          b[half] = qb[2 * ks + half];
-        } else if constexpr (kWide) {
-          // q*s as its fp16 high part and exact residual, two operands
-          const __half2 hi = __hmul2(u2h(qb[2 * ks + half]), u2h(s2));
-          b[half] = h2u(hi);
-          bl[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hneg2(hi)));
-        } else {
-          // q*s as fp16 high part (columns 0..3) or its exact residual (4..7):
-          // qn = -q on the lanes of columns 4..7 and 0 elsewhere (the same
-          // for every block), RN16(qn s) = -RN16(q s) there
-          const __half2 qn = __hmul2(u2h(qb[2 * ks + half]), u2h(ln.neg_lo));
-          b[half] = h2u(__hfma2(u2h(qb[2 * ks + half]), u2h(s2), __hmul2(qn, u2h(s2))));
-        }
-      }
-      mma16816(dk[bi][0], a0[0], a0[1], a0[2], a0[3], b[0], b[1]);
-      mma16816(dk[bi][1], a1[0], a1[1], a1[2], a1[3], b[0], b[1]);
-      if constexpr (kWide && !kScaledA) {
-        mma16816(dk[bi][0], a0[0], a0[1], a0[2], a0[3], bl[0], bl[1]);
-        mma16816(dk[bi][1], a1[0], a1[1], a1[2], a1[3], bl[0], bl[1]);
-      }
-    }
-    const uint2 zw = *reinterpret_cast<const uint2*>(zrow + 2 * (kHeadDim + c));
-    mma16816(dz, zw.x, 0u, zw.y, 0u, qb[2 * ks], qb[2 * ks + 1]);
-  }
-  // Scores in the log2 domain, less the running maximum (one fma each: the
-  // zero-point term and the offset are folded into the addend).  Narrow:
-  // lanes tig and tig^2 hold the two parts; wide: the accumulator holds the
-  // whole score.
-  float sc[NB][4][2];
-  const float me0 = m_offset(st.m[0]), me1 = m_offset(st.m[1]);
-#pragma unroll
-  for (int bi = 0; bi < NB; ++bi) {
-    const float z0 = fmaf(__shfl_sync(0xffffffffu, dz[0], 4 * bi + tig), scale_log2, -me0);
-    const float z1 = fmaf(__shfl_sync(0xffffffffu, dz[1], 4 * bi + tig), scale_log2, -me1);
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-      for (int rh = 0; rh < 2; ++rh)
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const int j = 2 * mt + rh;
-          const float d = dk[bi][mt][2 * rh + hh];
-          const float full = kWide ? d : d + __shfl_xor_sync(0xffffffffu, d, 2);
-          sc[bi][j][hh] = fmaf(full, Codes<BK>::inv(j) * scale_log2, hh ? z1 : z0);
-        }
-  }
-
-  constexpr bool kCompact = BV == 1;
-  uint32_t pt[NB][2][2], pl[NB][2][2];
-  tc_softmax<NB, kWide, kCompact, false>(sc, st, ln, pt, pl);
-
-  // ---- values: o^T[c][h] ----
-  // Value scales and zeros are stored in token pairs (t, t + 4), so the
-  // B-operand scale of (k-step ks, dl) is word 2ks + dl of the lane's 8-token
-  // run; zero-point MMA rows 0..3 = groups, row 4 = ones (the lanes of gid 4
-  // read bytes 256..319 of the zero area), so it accumulates the row sum of
-  // the weights; rows 5..7 read zeros.  (In the key zero-point MMA above the
-  // rows past NB read the same area; their results are never used.)
-#pragma unroll
-  for (int bi = 0; bi < NB; ++bi) {
-    const char* vc = pg[bi] + page_off_vcodes(BK);
-    const char* vmeta = pg[bi] + page_off_vmeta(BK, BV);
-    const char* vzrow = gid < 4 ? vmeta : zero;
-    const uint4 z8 = *reinterpret_cast<const uint4*>(vzrow + 2 * (kHeadDim + 32 * (gid & 3) + 8 * tig));
-    mma16816(st.zv, z8.x, 0u, z8.y, 0u, pt[bi][0][0], pt[bi][0][1]);
-    mma16816(st.zv, z8.z, 0u, z8.w, 0u, pt[bi][1][0], pt[bi][1][1]);
-    if constexpr (kCompact) {
-      // 1-bit values: B = RN16(p~ s), one MMA per operand for every head
-      const uint4 vw = *reinterpret_cast<const uint4*>(vc + 16 * lane);
-#pragma unroll
-      for (int g = 0; g < 4; ++g) {
-        const uint4 s8 = *reinterpret_cast<const uint4*>(vmeta + 2 * (32 * g + 8 * tig));
-        const uint32_t mw[4] = {s8.x, s8.y, s8.z, s8.w};
-#pragma unroll
-        for (int ks = 0; ks < 2; ++ks) {
-          uint32_t am0[4], am1[4], bv[2];
-#pragma unroll
-          for (int dl = 0; dl < 2; ++dl) {
-            const int ia = 2 * ks + dl;
-            uint32_t v[4];
-            Codes<1>::rot(comp(vw, g), ia, v);
-            am0[2 * dl] = v[0];
-            am0[2 * dl + 1] = v[1];
-            am1[2 * dl] = v[2];
-            am1[2 * dl + 1] = v[3];
-            bv[dl] = h2u(__hmul2(u2h(pt[bi][ks][dl]), u2h(mw[ia])));
-          }
-          mma16816(st.acc[2 * g], am0[0], am0[1], am0[2], am0[3], bv[0], bv[1]);
-          mma16816(st.acc[2 * g + 1], am1[0], am1[1], am1[2], am1[3], bv[0], bv[1]);
-        }
-      }
-      continue;
-    }
-    if constexpr (kWide) {
-      mma16816(st.zv, z8.x, 0u, z8.y, 0u, pl[bi][0][0], pl[bi][0][1]);
-      mma16816(st.zv, z8.z, 0u, z8.w, 0u, pl[bi][1][0], pl[bi][1][1]);
-    }
-    // B = p * s in two fp16 parts: the high part is RN16(p_hi s); the low
-    // part RN16(p_lo s + (p_hi s - RN16(p_hi s))), so rounding the product
-    // costs no accuracy.  Narrow: columns 0..3 / 4..7, lanes of columns 4..7
-    // hold p_lo after movmatrix and fetch p_hi from lane - 16; wide: every
-    // lane has both parts of its head.
-    // Narrow: pn = -p_hi on lanes of columns 4..7 and 0 elsewhere, so
-    // RN16(pn s) is -RN16(p_hi s) there (rounding is symmetric) and the
-    // residual fma needs no separate product.
-    uint32_t pa[2][2], pb[2][2], pn[2][2];
-#pragma unroll
-    for (int ks = 0; ks < 2; ++ks)
-#pragma unroll
-      for (int dl = 0; dl < 2; ++dl) {
-        if constexpr (kWide) {
-          pa[ks][dl] = pt[bi][ks][dl];
-          pb[ks][dl] = pl[bi][ks][dl];
-        } else {
-          const uint32_t other = __shfl_xor_sync(0xffffffffu, pt[bi][ks][dl], 16);
-          pa[ks][dl] = lane < 16 ? pt[bi][ks][dl] : other;
-          pb[ks][dl] = lane < 16 ? 0u : pt[bi][ks][dl];
-          pn[ks][dl] = h2u(__hmul2(u2h(pa[ks][dl]), u2h(ln.neg_lo)));
-        }
-      }
-    uint4 vw1;
-    if constexpr (BV == 1) vw1 = *reinterpret_cast<const uint4*>(vc + 16 * lane);
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-      const uint4 s8 = *reinterpret_cast<const uint4*>(vmeta + 2 * (32 * g + 8 * tig));
-      const uint32_t mw[4] = {s8.x, s8.y, s8.z, s8.w};  // scale pairs of tokens (8tig + i, + 4)
-      uint32_t cw[8];
-      if constexpr (BV != 1) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          cw[i] = *reinterpret_cast<const uint32_t*>(vc + 4 * ((32 * g + 8 * tig + i) * BV + ln.wv));
-      }
-#pragma unroll
-      for (int ks = 0; ks < 2; ++ks) {
-        uint32_t am0[4], am1[4], bv[2], bw[2];
-#pragma unroll
-        for (int dl = 0; dl < 2; ++dl) {
-          const int ia = 2 * ks + dl, ib = ia + 4;  // tokens 8tig + ia, 8tig + ib
-          uint32_t v[4];
-          if constexpr (BV == 1) Codes<1>::rot(comp(vw1, g), ia, v);
-          else Codes<BV>::get(cw[ia], cw[ib], ln.sel_v, v);
-          am0[2 * dl] = v[0];
-          am0[2 * dl + 1] = v[1];
-          am1[2 * dl] = v[2];
-          am1[2 * dl + 1] = v[3];
-          const __half2 sc = u2h(mw[ia]);
-          if constexpr (kWide) {
-            const __half2 t = __hmul2(u2h(pa[ks][dl]), sc);
-            const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hneg2(t));
-            bv[dl] = h2u(t);
-            bw[dl] = h2u(__hfma2(u2h(pb[ks][dl]), sc, err));
-          } else {
-            // columns 0..3: RN16(p_hi s); 4..7: RN16(p_lo s + exact residual)
-            const __half2 err = __hfma2(u2h(pa[ks][dl]), sc, __hmul2(u2h(pn[ks][dl]), sc));
-            bv[dl] = h2u(__hfma2(u2h(pb[ks][dl]), sc, err));
-          }
-        }
-        mma16816(st.acc[2 * g], am0[0], am0[1], am0[2], am0[3], bv[0], bv[1]);
-        mma16816(st.acc[2 * g + 1], am1[0], am1[1], am1[2], am1[3], bv[0], bv[1]);
-        if constexpr (kWide) {
-          mma16816(st.acc[2 * g], am0[0], am0[1], am0[2], am0[3], bw[0], bw[1]);
-          mma16816(st.acc[2 * g + 1], am1[0], am1[1], am1[2], am1[3], bw[0], bw[1]);
-        }
-      }
-    }
-  }
-}
-
-template <int BK, int BV>
-__device__ __forceinline__ Lane make_lane(int lane) {
-  Lane ln;
-  ln.gid = lane >> 2;
-  ln.tig = lane & 3;
-  ln.sel_k = code_selector<BK>(ln.gid);
-  ln.sel_v = code_selector<BV>(ln.gid);
-  ln.wk = Codes<BK>::word(ln.gid);
-  ln.wv = Codes<BV>::word(ln.gid);
-  ln.neg_lo = ln.gid >= 4 ? 0xBC00BC00u : 0u;
-  ln.p_lo = ln.tig >= 2 ? 1.0f : 0.0f;
-  return ln;
-}
-
-// q of head gid & 3 (narrow) or gid (wide) in the B layout (exact fp16),
-// zero beyond the group.  kPermuted: the packed path's K-slot order (four
-// contiguous channels per lane); otherwise slot k of a k-step is channel
-// 16 ks + k.
-template <bool kPermuted, bool kWide>
-__device__ __forceinline__ void load_qb(uint32_t (&qb)[16], const __half* qh, int gq,
-                                        const Lane& ln) {
-  const int head = kWide ? ln.gid : ln.gid & 3;
-#pragma unroll
-  for (int ks = 0; ks < 8; ++ks)
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int c = kPermuted ? 16 * ks + 4 * ln.tig + 2 * half : 16 * ks + 2 * ln.tig + 8 * half;
-      qb[2 * ks + half] =
-          head < gq ? *reinterpret_cast<const uint32_t*>(qh + head * kHeadDim + c) : 0u;
-    }
-}
-
-__device__ __forceinline__ void init_state(TcState& st) {
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int r = 0; r < 4; ++r) st.acc[i][r] = 0.0f;
-#pragma unroll
-  for (int r = 0; r < 4; ++r) st.zv[r] = 0.0f;
-  st.m[0] = st.m[1] = -INFINITY;
-  st.l[0] = st.l[1] = 0.0f;
-}
-
-// A warp's running state to the merge area: row maximum, row sum and the
-// unnormalised output row of heads 0..3 (narrow: the two parts in columns
-// tig and tig^2 are added) or 0..7 (wide).  kPacked: channel rows follow the
-// packed layout (nibble of a group, power-of-two factors, zero-point term);
-// otherwise channel = 16 * m-tile + row.
-template <bool kPacked, int BV, bool kWide>
-__device__ __forceinline__ void tc_write_state(const TcState& st, WarpState& ws, int lane) {
-  const int gid = lane >> 2, tig = lane & 3;
-  float l0 = st.l[0], l1 = st.l[1];
-#pragma unroll
-  for (int o = 4; o < 32; o <<= 1) {
-    l0 += __shfl_xor_sync(0xffffffffu, l0, o);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, o);
-  }
-  float zsum[2];
-  zsum[0] = kWide ? st.zv[0] : st.zv[0] + __shfl_xor_sync(0xffffffffu, st.zv[0], 2);
-  zsum[1] = kWide ? st.zv[1] : st.zv[1] + __shfl_xor_sync(0xffffffffu, st.zv[1], 2);
-  if constexpr (kPacked) {
-    // packed blocks: the row sum is row 4 of the value zero-point MMA
-    l0 += __shfl_sync(0xffffffffu, zsum[0], 16 + tig);
-    l1 += __shfl_sync(0xffffffffu, zsum[1], 16 + tig);
-  }
-  if (gid == 0 && (kWide || tig < 2)) {
-    ws.m[2 * tig] = st.m[0];
-    ws.m[2 * tig + 1] = st.m[1];
-    ws.l[2 * tig] = l0;
-    ws.l[2 * tig + 1] = l1;
-  }
-#pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    const float zg0 = kPacked ? __shfl_sync(0xffffffffu, zsum[0], 4 * g + tig) : 0.0f;
-    const float zg1 = kPacked ? __shfl_sync(0xffffffffu, zsum[1], 4 * g + tig) : 0.0f;
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int mtp = 2 * g + half;
-#pragma unroll
-      for (int rh = 0; rh < 2; ++rh) {
-        const int jp = 2 * half + rh;
-        const int cch = kPacked ? 32 * g + 4 * gid + jp : 16 * mtp + gid + 8 * rh;
-        const float inv = kPacked ? Codes<BV>::inv(jp) : 1.0f;
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const float a = st.acc[mtp][2 * rh + hh];
-          const float full_v = kWide ? a : a + __shfl_xor_sync(0xffffffffu, a, 2);
-          if (kWide || tig < 2) ws.o[2 * tig + hh][cch] = fmaf(full_v, inv, hh ? zg1 : zg0);
-        }
-      }
-    }
-  }
-}
-
-// ---------------------------------------------------------------------------
-// Tensor-core path for the fp16 residual window: a warp stages the K rows of
-// a 32-token chunk in shared memory, scores them with ldmatrix-fed MMAs
-// (keys as A with tokens as rows), then stages the V rows in the same place
-// (values transposed, channels as rows).  Rows past the window are zero and
-// their scores -inf.
-// ---------------------------------------------------------------------------
-
-constexpr int kResRow = kHeadDim + 8;                    // halves per staged row (16-byte pad)
-constexpr int kResRowsBytes = kGroup * kResRow * 2;      // one 32-row K or V chunk
-
-__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_addr(p))
-               : "memory");
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_addr(p))
-               : "memory");
-}
-__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(dst)), "l"(src),
-               "r"(src_bytes)
-               : "memory");
-}
-
-template <bool kWide, bool kCompact>
-__device__ __forceinline__ void tc_resid_scores(const __half* ks_s, int n_tok,
-                                                const uint32_t (&qb)[16], const Lane& ln,
-                                                float scale_log2, TcState& st,
-                                                uint32_t (&pt)[1][2][2], uint32_t (&pl)[1][2][2]) {
+// Work totals of all pairs (lengths as the kernel attends them).
+__device__ WorkSums plan_sums(const int* seq_len, const Dims& d, bool append) {
   const int lane = threadIdx.x & 31;
-  const int mi = lane >> 3, r8 = lane & 7;
-  float dk[2][4] = {};
-#pragma unroll
-  for (int ks = 0; ks < 8; ++ks)
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt) {
-      uint32_t a[4];
-      ldsm_x4(a, ks_s + (16 * mt + 8 * (mi & 1) + r8) * kResRow + 16 * ks + 8 * (mi >> 1));
-      mma16816(dk[mt], a[0], a[1], a[2], a[3], qb[2 * ks], qb[2 * ks + 1]);
-    }
-  float sc[1][4][2];
-  const float me[2] = {m_offset(st.m[0]), m_offset(st.m[1])};
-#pragma unroll
-  for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-    for (int rh = 0; rh < 2; ++rh) {
-      const bool ok = 16 * mt + ln.gid + 8 * rh < n_tok;
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh)
-        sc[0][2 * mt + rh][hh] = ok ? fmaf(dk[mt][2 * rh + hh], scale_log2, -me[hh]) : -INFINITY;
-    }
-  tc_softmax<1, kWide, kCompact, true>(sc, st, ln, pt, pl);
+  long long nb = 0, nr = 0, np = 0;
+  for (int b0 = 0; b0 < d.batch; b0 += 32) {
+    const int b = b0 + lane;
+    const PairShape s = pair_shape(b < d.batch ? attended_len(read_len(seq_len + b), d, append) : 0, d.residual);
+    nb += warp_sum_ll((long long)d.hkv * s.nb);
+    nr += warp_sum_ll((long long)d.hkv * s.nr);
+    np += warp_sum_ll(s.nb + s.nr > 0 ? d.hkv : 0);
+  }
+  WorkSums w;
+  w.nb = nb;
+  w.nr = nr;
+  w.np = np;
+  return w;
 }
 
-template <bool kWide, bool kCompact>
-__device__ __forceinline__ void tc_resid_values(const __half* vs_s, const uint32_t (&pt)[1][2][2],
-                                                const uint32_t (&pl)[1][2][2], TcState& st) {
+// A warp's walk over the pairs its unit range [a, e) meets, in order.
+struct Walk {
+  int b, h;        // current sequence and kv-head
+  long long Ub;    // first unit of sequence b
+  int L0, L, pc;   // stored and attended length of b, cost of one of its pairs
+};
+__device__ __forceinline__ void walk_load(Walk& w, const int* seq_len, const Dims& d,
+                                          bool append, Costs k) {
+  if (w.b < d.batch) {
+    w.L0 = read_len(seq_len + w.b);
+    w.L = attended_len(w.L0, d, append);
+    w.pc = pair_cost(pair_shape(w.L, d.residual), k);
+  }
+}
+// Position at the first pair whose units reach past a (an empty pair at or
+// after a included): a scan of the sequences' costs, 32 at a time.
+__device__ Walk walk_start(long long a, const int* seq_len, const Dims& d, bool append, Costs k) {
   const int lane = threadIdx.x & 31;
-  const int mi = lane >> 3, r8 = lane & 7;
+  Walk w;
+  long long base = 0;
+  for (int b0 = 0; b0 < d.batch; b0 += 32) {
+    const int b = b0 + lane;
+    const int L0 = b < d.batch ? read_len(seq_len + b) : 0;
+    const int L = attended_len(L0, d, append);
+    const int pc = b < d.batch ? pair_cost(pair_shape(L, d.residual), k) : 0;
+    const long long cst = (long long)d.hkv * pc;
+    long long incl = cst;
 #pragma unroll
-  for (int ks = 0; ks < 2; ++ks)
-#pragma unroll
-    for (int mtp = 0; mtp < 8; ++mtp) {
-      uint32_t a[4];
-      ldsm_x4_t(a, vs_s + (16 * ks + 8 * (mi >> 1) + r8) * kResRow + 16 * mtp + 8 * (mi & 1));
-      mma16816(st.acc[mtp], a[0], a[1], a[2], a[3], pt[0][ks][0], pt[0][ks][1]);
-      if constexpr (kWide && !kCompact)
-        mma16816(st.acc[mtp], a[0], a[1], a[2], a[3], pl[0][ks][0], pl[0][ks][1]);
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
     }
-}
-
-// ---------------------------------------------------------------------------
-// Work of one (sequence, kv-head): nb packed blocks and n_res window chunks
-// over NV warps.  The last n_resw warps take the window chunks (strided), the
-// other np warps contiguous block ranges whose sizes differ by at most one.
-// ---------------------------------------------------------------------------
-
-struct Plan {
-  int Lq, nb, n_res, n_resw, np;
-};
-
-__host__ __device__ inline Plan make_plan(int L, int residual, int NV) {
-  Plan p;
-  p.Lq = packed_len(L, residual);
-  p.nb = p.Lq / kGroup;
-  p.n_res = (L - p.Lq + kGroup - 1) / kGroup;
-  const int cap = p.nb == 0 ? NV : (NV / 4 > 1 ? NV / 4 : 1);
-  p.n_resw = p.n_res < cap ? p.n_res : cap;
-  p.np = NV - p.n_resw;
-  return p;
-}
-
-// Blocks [lo, hi) of packed warp v (v < np), in 32-bit arithmetic while
-// (v + 1) * nb fits (v < 4096 warps).
-__host__ __device__ inline void block_range(const Plan& p, int v, int& lo, int& hi) {
-  if (p.nb < (1 << 20)) {
-    lo = (int)((unsigned)v * (unsigned)p.nb / (unsigned)p.np);
-    hi = (int)((unsigned)(v + 1) * (unsigned)p.nb / (unsigned)p.np);
-  } else {
-    lo = (int)((long long)v * p.nb / p.np);
-    hi = (int)((long long)(v + 1) * p.nb / p.np);
-  }
-}
-
-// Blocks per ring slot and slots per warp for a page size.
-__host__ __device__ constexpr int ring_blocks(int page) { return page <= 3072 ? 2 : 1; }
-__host__ __device__ constexpr int ring_slots(int page) {
-  return kRingBudget / (kWarps * ring_blocks(page) * page) < 1   ? 1
-         : kRingBudget / (kWarps * ring_blocks(page) * page) > 4 ? 4
-                                                                 : kRingBudget / (kWarps * ring_blocks(page) * page);
-}
-// A warp's ring: its slots, and at least one 32-row K (or V) chunk of the
-// window, which a window warp stages there.
-__host__ __device__ constexpr int warp_ring_bytes(int page) {
-  return ((ring_slots(page) * ring_blocks(page) * page > kResRowsBytes
-               ? ring_slots(page) * ring_blocks(page) * page
-               : kResRowsBytes) +
-          127) / 128 * 128;
-}
-static_assert(kWarps * warp_ring_bytes(page_bytes_c(4, 8)) <= kRingBudget + 8 * 1024, "rings fit");
-// Shared-memory page image of a block that leaves the window (decode step).
-__host__ __device__ constexpr int image_bytes(int page) { return (page + 127) / 128 * 128; }
-
-// Packed warps stream their blocks through a private ring of slots.  A page
-// is written once, when its group leaves the window, and never changes
-// afterwards, so before waiting for the previous kernel (programmatic
-// dependent launch) lane 0 already streams the first slots of the range that
-// a length read before the wait gives (tc_pre_issue), up to the block before
-// the newest.  If the range after the wait does not begin with exactly those
-// slots they are consumed without use.
-// A warp's window of 32 consecutive block-table entries (paged caches): lane
-// i holds the entry of block wb + i, refreshed (one coalesced load) when a
-// lookup leaves it.  Lookups are warp-uniform and made by all lanes.
-struct TableWin {
-  int wb, v;
-};
-__device__ __forceinline__ void table_win_init(TableWin& w) {
-  w.wb = -(1 << 30);
-  w.v = -1;
-}
-__device__ __forceinline__ const char* block_addr(const PageMap& pm, TableWin& w, int j) {
-  if (!pm.paged()) return pm.base + (long long)j * pm.page;
-  if (j < w.wb || j >= w.wb + 32) {
-    w.wb = j;
-    const int k = j + (int)(threadIdx.x & 31);
-    w.v = k < pm.max_blocks ? __ldg(pm.row + k) : -1;
-  }
-  return pm.at(j, __shfl_sync(0xffffffffu, w.v, j - w.wb));
-}
-
-// Slot s of the ring: blocks [first, first + nblk) (nblk <= blocks per
-// slot).  Called by all lanes; lane 0 issues.  Contiguous pages come in one
-// bulk copy, paged ones in one copy per page; a block mapped outside the
-// pool is not copied (KVQ_FLAG_BAD_PAGE; its slot bytes are stale and the
-// call's output is flagged invalid) and the barrier expects only the bytes
-// copied.  `fence`: the warp's reads of the slot precede the copies that
-// overwrite it.
-template <int BK, int BV>
-__device__ __forceinline__ void issue_slot(const PageMap& pm, TableWin& tw, char* ring,
-                                           uint64_t* full, int R, int s, int first, int nblk,
-                                           unsigned* flag, bool fence) {
-  constexpr int page = page_bytes_c(BK, BV);
-  constexpr int NB = ring_blocks(page);
-  const bool lead = (threadIdx.x & 31) == 0;
-  uint64_t* bar = full + s % R;
-  char* dst = ring + (size_t)(s % R) * NB * page;
-  if (!pm.paged()) {
-    if (lead) {
-      if (fence) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      const uint32_t bytes = (uint32_t)(nblk * page);
-      mbar_expect_tx(bar, bytes);
-      bulk_g2s(dst, pm.base + (long long)first * page, bytes, bar);
+    incl += base;
+    const long long excl = incl - cst;
+    const unsigned hit = __ballot_sync(0xffffffffu, b < d.batch && (incl > a || (cst == 0 && excl >= a)));
+    if (hit) {
+      const int l = __ffs(hit) - 1;
+      w.b = b0 + l;
+      w.Ub = __shfl_sync(0xffffffffu, excl, l);
+      w.L0 = __shfl_sync(0xffffffffu, L0, l);
+      w.L = __shfl_sync(0xffffffffu, L, l);
+      w.pc = __shfl_sync(0xffffffffu, pc, l);
+      w.h = w.pc > 0 && a > w.Ub ? (int)((a - w.Ub) / w.pc) : 0;
+      return w;
     }
-    return;
+    base = __shfl_sync(0xffffffffu, incl, 31);
   }
-  const char* src[NB];
-  uint32_t bytes = 0;
-#pragma unroll
-  for (int i = 0; i < NB; ++i) {
-    src[i] = i < nblk ? block_addr(pm, tw, first + i) : nullptr;
-    if (src[i]) bytes += page;
-  }
-  if (lead) {
-    if (fence) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    if (bytes < (uint32_t)(nblk * page)) atomicOr(flag, (unsigned)KVQ_FLAG_BAD_PAGE);
-    mbar_expect_tx(bar, bytes);
-#pragma unroll
-    for (int i = 0; i < NB; ++i)
-      if (src[i]) bulk_g2s(dst + i * page, src[i], page, bar);
-  }
+  w.b = d.batch;
+  w.h = 0;
+  w.Ub = base;
+  w.L0 = w.L = w.pc = 0;
+  return w;
+}
+__device__ __forceinline__ void walk_next(Walk& w, const int* seq_len, const Dims& d, bool append,
+                                          Costs k) {
+  if (++w.h < d.hkv) return;
+  w.h = 0;
+  w.Ub += (long long)d.hkv * w.pc;
+  ++w.b;
+  walk_load(w, seq_len, d, append, k);
 }
 
-// Units (slots) of the range [lo_h, hi_h) that end at or before hi_safe:
-// streams them, returns their count and in `end` the block after them.
-template <int BK, int BV>
-__device__ __forceinline__ int tc_pre_issue(const PageMap& pm, TableWin& tw, int lo_h, int hi_h,
-                                            int hi_safe, char* ring, uint64_t* full, int R,
-                                            int& end, unsigned* flag) {
-  constexpr int NB = ring_blocks(page_bytes_c(BK, BV));
-  int n = 0;
-  end = lo_h;
-  for (; n < R; ++n) {
-    const int b0 = lo_h + n * NB;
-    const int nblk = min(NB, hi_h - b0);
-    if (nblk <= 0 || b0 + nblk > hi_safe) break;
-    issue_slot<BK, BV>(pm, tw, ring, full, R, n, b0, nblk, flag, false);
-    end = b0 + nblk;
-  }
-  return n;
-}
 
-// Decode step with a flush: the 32-token block of positions [p0, p0 + 32),
-// still fp16 in the ring, leaves the window and is quantized exactly as
-// kvq_pack does (quantize_quarter, common.cuh) into a page image in shared
-// memory.  The work comes in four quarters (key channels 32 qi .. 32 qi + 31,
-// value group qi), so different warps can take them.  Rows are read straight
-// from global memory (L2); nothing in this kernel writes them.  Kept out of
-// line: it is rare and its registers would otherwise crowd the streaming
-// loop.
-template <int BK, int BV>
-__device__ __noinline__ void flush_quarter(const __half* ring_k, const __half* ring_v, int p0,
-                                           int ring, int qi, char* image) {
-  const int s0 = p0 % ring;
-  quantize_quarter<BK, BV>(
-      [&](int t) { return ring_k + (long long)(s0 + t < ring ? s0 + t : s0 + t - ring) * kHeadDim; },
-      [&](int t) { return ring_v + (long long)(s0 + t < ring ? s0 + t : s0 + t - ring) * kHeadDim; },
-      qi, image);
-}
 
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
-}
 
-// Fold blocks [lo, hi) into st; `pre` slots holding blocks [lo_h, pre_end)
-// were streamed early.
-// Fold blocks [lo, hi) into st; `pre` slots holding blocks [lo_h, pre_end)
-// were streamed early.
+// Fold packed blocks [lo, hi) of one pair into st, streaming their pages
+// through the warp's ring.  *pos_io counts the ring slots the warp has used
+// in this kernel (slot pos % R, phase parity (pos / R) & 1) and moves past
+// this call's slots; `pre` slots holding blocks [lo_h, pre_end) were
+// streamed early from position 0 and are consumed without use unless this
+// range begins with them.  keep_tail: the block after hi leaves the window
+// in this kernel and folds after this call (tc_fold_flush); blocks fold in
+// units of NB from lo, as kvq_decode_attn folds lo .. hi after kvq_pack, so
+// if the range ends in a unit of one, that unit is not folded here and its
+// page stays in the ring (*tail_out; otherwise nullptr) to fold with the
+// flushed block: both paths then take the same softmax updates (1-bit values
+// round their fp16 weights against the running maximum).
 template <int BK, int BV, bool kWide>
-__device__ void tc_packed_warp(const PageMap& pm, TableWin& tw, int lo_h, int pre, int pre_end,
-                               int lo, int hi_all, char* ring, uint64_t* full, int R,
-                               const char* zero, const __half* qh, int gq, float scale_log2,
-                               unsigned* flag, TcState& st, int flush_blk, uint64_t* fl_bar,
-                               char* image) {
+__device__ __forceinline__ TcState tc_packed_warp(TcState st, const PageMap pm, int lo_h, int pre,
+                                                  int pre_end, int lo, int hi, char* ring,
+                                                  uint64_t* full, int* pos_io, const char* zero,
+                                                  const __half* qh, int gq, float scale_log2,
+                                                  unsigned* flag, bool keep_tail,
+                                                  const char** tail_out) {
+  TableWin tw;
+  table_win_init(tw);
   constexpr int page = page_bytes_c(BK, BV);
   constexpr int NB = ring_blocks(page);
+  constexpr int R = ring_slots(page);
   const int lane = threadIdx.x & 31;
-  // a block that leaves the window in this kernel has no page yet: it is
-  // quantized from the ring after the streamed ones
-  const bool flush = flush_blk >= lo && flush_blk == hi_all - 1;
-  const int hi = flush ? hi_all - 1 : hi_all;
-  // the early slots are this range's first units if they start at lo and
-  // cover what its first `pre` units cover
   const bool reuse = pre > 0 && lo == lo_h && min(lo + pre * NB, hi) == pre_end;
   const int skip = reuse ? 0 : pre;
-  const int n_units = (hi - lo + NB - 1) / NB;
+  const int n_units = hi > lo ? (hi - lo + NB - 1) / NB : 0;
   const int total = skip + n_units;
+  const int p0 = *pos_io;
+  const bool hold = keep_tail && NB == 2 && n_units > 0 && ((hi - lo) & 1);
+  const char* tail = nullptr;
   int issued = pre;  // slots issued so far
-  auto real_issue = [&](int s, bool fence) {
+  auto real_issue = [&](int s) {
     const int u = s - skip;
-    issue_slot<BK, BV>(pm, tw, ring, full, R, s, lo + u * NB, min(NB, hi - lo - u * NB), flag,
-                       fence);
+    // the slot may have been read (or written by generic stores: window rows,
+    // a flushed page) before: order that before the copy that overwrites it
+    issue_slot<BK, BV>(pm, tw, ring, full, R, p0 + s, lo + u * NB, min(NB, hi - lo - u * NB), flag,
+                       true);
     issued = s + 1;
   };
-  for (int s = pre; s < min(total, R); ++s) real_issue(s, false);
+  for (int s = pre; s < min(total, R); ++s) real_issue(s);
 
   const Lane ln = make_lane<BK, BV>(lane);
   uint32_t qb[16];
   load_qb<true, kWide>(qb, qh, gq, ln);
   int consumed = 0;
   for (int s = 0; s < total; ++s) {
-    const int slot = s % R;
+    const int slot = (p0 + s) % R;
     // every lane waits; the warp leaves together if any lane gave up
-    if (!__all_sync(0xffffffffu, mbar_wait(full + slot, (s / R) & 1))) {
+    if (!__all_sync(0xffffffffu, mbar_wait(full + slot, ((p0 + s) / R) & 1))) {
       if (lane == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
       break;
     }
@@ -1017,7 +389,9 @@ __device__ void tc_packed_warp(const PageMap& pm, TableWin& tw, int lo_h, int pr
     if (s >= skip) {
       const int u = s - skip;
       const char* base = ring + (size_t)slot * NB * page;
-      if (lo + u * NB + NB <= hi) {
+      if (hold && s == total - 1) {
+        tail = base;
+      } else if (lo + u * NB + NB <= hi) {
         const char* pg[NB];
 #pragma unroll
         for (int i = 0; i < NB; ++i) pg[i] = base + i * page;
@@ -1028,61 +402,58 @@ __device__ void tc_packed_warp(const PageMap& pm, TableWin& tw, int lo_h, int pr
       }
     }
     __syncwarp();
-    if (s + R < total) real_issue(s + R, true);
+    if (s + R < total) real_issue(s + R);
   }
   // Copies issued but not consumed (a wait gave up, or the range shrank) land
   // before the ring is reused; bounded waits.
   if (lane == 0)
-    for (int s = max(consumed, issued - R); s < issued; ++s) mbar_wait(full + s % R, (s / R) & 1);
+    for (int s = max(consumed, issued - R); s < issued; ++s)
+      mbar_wait(full + (p0 + s) % R, ((p0 + s) / R) & 1);
   __syncwarp();
-  if (flush) {
-    // the page image is complete once its four quarters have arrived
-    char* dst = const_cast<char*>(block_addr(pm, tw, flush_blk));
-    if (__all_sync(0xffffffffu, mbar_wait(fl_bar, 0u))) {
-      if (dst) {
-        uint4* d4 = reinterpret_cast<uint4*>(dst);
-        for (int i = lane; i < page / 16; i += 32) d4[i] = reinterpret_cast<const uint4*>(image)[i];
-      } else if (lane == 0) {
-        atomicOr(flag, (unsigned)KVQ_FLAG_BAD_PAGE);
-      }
-      const char* pg[1] = {image};
-      tc_unit<BK, BV, 1, kWide>(pg, zero, qb, ln, scale_log2, st);
-    } else if (lane == 0) {
-      atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
-    }
-  }
+  *pos_io = p0 + issued;
+  *tail_out = tail;
+  return st;
 }
 
-// Copy rows p0 .. p0 + 31 into padded `rows` with one bulk copy per row
-// (issued by the row's lane, completing on `bar`); rows at or past n_tok are
-// zeroed.  The row of position p_new comes from new_row.  Returns false if
-// the bounded wait gave up.
-__device__ __forceinline__ bool stage_rows_bulk(__half* rows, const __half* ring_base, int p0,
-                                                int n_tok, int ring, int p_new,
-                                                const __half* new_row, uint64_t* bar,
-                                                uint32_t parity) {
+// The block `blk` of a pair leaves the window in this kernel (decode step)
+// and has no page yet: the warp quantizes it from the fp16 ring rows exactly
+// as kvq_pack does (quantize_quarter, common.cuh) into its idle ring (or the
+// second page of the held tail unit), writes the page and folds it, with the
+// tail unit if there is one.  Rare (one block in 32 steps), so out of line.
+template <int BK, int BV, bool kWide>
+__device__ __noinline__ TcState tc_fold_flush(TcState st, const PageMap pm, int blk,
+                                              const char* tail, char* ring, const char* zero,
+                                              const __half* qh, int gq, float scale_log2,
+                                              unsigned* flag, const __half* ring_k,
+                                              const __half* ring_v, int ring_len) {
+  constexpr int page = page_bytes_c(BK, BV);
   const int lane = threadIdx.x & 31;
+  TableWin tw;
+  table_win_init(tw);
+  char* img = tail ? const_cast<char*>(tail) + page : ring;
+  for (int qi = 0; qi < 4; ++qi) flush_quarter<BK, BV>(ring_k, ring_v, blk * kGroup, ring_len, qi, img);
   __syncwarp();
-  if (lane >= n_tok) {
-    uint4* r = reinterpret_cast<uint4*>(rows + lane * kResRow);
-#pragma unroll
-    for (int i = 0; i < 16; ++i) r[i] = make_uint4(0u, 0u, 0u, 0u);
+  char* dst = const_cast<char*>(block_addr(pm, tw, blk));
+  if (dst) {
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+    for (int i = lane; i < page / 16; i += 32) d4[i] = reinterpret_cast<const uint4*>(img)[i];
+  } else if (lane == 0) {
+    atomicOr(flag, (unsigned)KVQ_FLAG_BAD_PAGE);
   }
-  if (lane == 0) {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    mbar_expect_tx(bar, (uint32_t)(n_tok * kHeadDim * 2));
+  const Lane ln = make_lane<BK, BV>(lane);
+  uint32_t qb[16];
+  load_qb<true, kWide>(qb, qh, gq, ln);
+  if (ring_blocks(page) == 2 && tail) {
+    const char* pg[2] = {tail, img};
+    tc_unit<BK, BV, 2, kWide>(pg, zero, qb, ln, scale_log2, st);
+  } else {
+    const char* pg[1] = {img};
+    tc_unit<BK, BV, 1, kWide>(pg, zero, qb, ln, scale_log2, st);
   }
   __syncwarp();
-  if (lane < n_tok) {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    const __half* src = p0 + lane == p_new ? new_row
-                                           : ring_base + (long long)((p0 + lane) % ring) * kHeadDim;
-    bulk_g2s(rows + lane * kResRow, src, kHeadDim * 2, bar);
-  }
-  const bool ok = __all_sync(0xffffffffu, mbar_wait(bar, parity));
-  __syncwarp();
-  return ok;
+  return st;
 }
+
 
 // Bring ring rows [p0, p0 + n) (one or two contiguous runs) into L2.
 __device__ __forceinline__ void prefetch_rows_l2(const __half* ring_base, int p0, int n, int ring) {
@@ -1097,50 +468,178 @@ __device__ __forceinline__ void prefetch_rows_l2(const __half* ring_base, int p0
                  : "memory");
 }
 
-// Window warp: chunks c0, c0 + stride, ... of the fp16 window.
+// Window chunks [i0, i1) of one pair (chunk u = tokens Lq + 32 u ...), staged
+// in the warp's (idle) ring; *phase_io is the parity count of the warp's
+// staging barrier, kept across calls.  A bounded wait that gives up sets
+// KVQ_FLAG_WAIT_TIMEOUT and ends the chunks.
+// Out of line, like tc_packed_warp.
 template <int BK, int BV, bool kWide>
-__device__ void tc_window_warp(const Dims& d, const __half* ring_k, const __half* ring_v,
-                               const Plan& p, int L, int c0, int stride, char* area,
-                               const __half* qh, int gq, float scale_log2, TcState& st,
-                               int p_new, const __half* k_row, const __half* v_row,
-                               uint64_t* bar, unsigned* flag) {
+__device__ __noinline__ TcState tc_window_chunks(TcState st, const Dims d, const __half* ring_k,
+                                                 const __half* ring_v, int Lq, int L, int i0,
+                                                 int i1, char* area, const __half* qh, int gq,
+                                                 float scale_log2, int p_new,
+                                                 const __half* k_row, const __half* v_row,
+                                                 uint64_t* bar, uint32_t* phase_io,
+                                                 unsigned* flag) {
+  uint32_t phase = *phase_io;
   const int lane = threadIdx.x & 31;
   const Lane ln = make_lane<BK, BV>(lane);
   uint32_t qb[16];
   load_qb<false, kWide>(qb, qh, gq, ln);
   __half* rows = reinterpret_cast<__half*>(area);
-  uint32_t phase = 0u;
-  for (int u = c0; u < p.n_res; u += stride) {
-    const int p0 = p.Lq + u * kGroup;
+  for (int u = i0; u < i1; ++u) {
+    const int p0 = Lq + u * kGroup;
     const int n_tok = min(kGroup, L - p0);
     uint32_t pt[1][2][2], pl[1][2][2];
     if (!stage_rows_bulk(rows, ring_k, p0, n_tok, d.ring, p_new, k_row, bar, phase++ & 1u)) {
-      if ((threadIdx.x & 31) == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
-      return;
+      if (lane == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
+      break;
     }
     tc_resid_scores<kWide, BV == 1>(rows, n_tok, qb, ln, scale_log2, st, pt, pl);
     __syncwarp();
     if (!stage_rows_bulk(rows, ring_v, p0, n_tok, d.ring, p_new, v_row, bar, phase++ & 1u)) {
-      if ((threadIdx.x & 31) == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
-      return;
+      if (lane == 0) atomicOr(flag, KVQ_FLAG_WAIT_TIMEOUT);
+      break;
     }
     tc_resid_values<kWide, BV == 1>(rows, pt, pl, st);
     __syncwarp();
   }
+  *phase_io = phase;
+  return st;
 }
 
-// One element of the attention output: the fp32 result, or its fp16
-// rounding to nearest even.
-__device__ __forceinline__ void store_out(void* out, int out_f16, long long i, float v) {
-  if (out_f16) static_cast<__half*>(out)[i] = __float2half_rn(v);
-  else static_cast<float*>(out)[i] = v;
+
+// Inverse of tc_write_state<false>: a WarpState (natural channel order) back
+// into registers in the window layout (channel = 16 m-tile + row, no
+// zero-point term), so the window chunks of a pair continue the state its
+// packed blocks began.  Row sums go to the lanes of gid 0.
+template <bool kWide>
+__device__ __forceinline__ void tc_read_state(TcState& st, const WarpState& ws, int lane) {
+  const int gid = lane >> 2, tig = lane & 3;
+  const bool keep = kWide || tig < 2;  // narrow: lanes tig and tig^2 share heads
+#pragma unroll
+  for (int hh = 0; hh < 2; ++hh) {
+    const int head = 2 * (kWide ? tig : (tig & 1)) + hh;
+    st.m[hh] = ws.m[head];
+    st.l[hh] = gid == 0 ? ws.l[head] : 0.0f;
+  }
+#pragma unroll
+  for (int mtp = 0; mtp < 8; ++mtp)
+#pragma unroll
+    for (int rh = 0; rh < 2; ++rh)
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const int head = 2 * (kWide ? tig : (tig & 1)) + hh;
+        st.acc[mtp][2 * rh + hh] = keep ? ws.o[head][16 * mtp + gid + 8 * rh] : 0.0f;
+      }
+#pragma unroll
+  for (int r = 0; r < 4; ++r) st.zv[r] = 0.0f;
 }
 
-__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
-  unsigned old;
-  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
-  return old;
+// Global partial slots: CTA partials [0, n_cta_slots + P), then one warp
+// partial per pair.  Each holds m[gq], l[gq], o[gq][128] (Ws arrays).
+__device__ __forceinline__ long long warp_slot(int ctas, int P, int p) {
+  return (long long)ctas + P + p;
 }
+
+// A pair whose partials this CTA completed (final merge at the end), or a
+// warp's final state.
+struct SegRec {
+  long long U;      // first cost unit of the pair
+  int p, pc, nb, nr;
+};
+
+// Row o / l of every head of a WarpState into out (a pair's only partial).
+__device__ __forceinline__ void warp_state_out(const WarpState& s, void* out, int out_f16,
+                                               long long head0, int gq, int lane) {
+  for (int i = lane; i < gq * kHeadDim; i += 32) {
+    const int g = i / kHeadDim, ch = i % kHeadDim;
+    const float l = s.l[g];
+    store_out(out, out_f16, (head0 + g) * kHeadDim + ch, l > 0.0f ? s.o[g][ch] / l : 0.0f);
+  }
+}
+
+// The final merge of pair p: its partials are the CTA slots [c_a + p,
+// c_a + p + n_cta) and, if cont, its warp slot.  All threads of the CTA; the
+// partials are copied into shared memory (`scratch`, the idle rings, of
+// scratch_bytes) with one round of independent loads when they fit.
+__device__ void final_merge(const SegRec& r, const FlatGrid& g, const Dims& d, const Ws& ws,
+                            void* out, int out_f16, float* scratch, size_t scratch_bytes) {
+  const int P = d.batch * d.hkv, gq = d.gq;
+  int c_a, n_cta;
+  bool cont;
+  const int cnt = pair_partials(r.U, r.pc, r.nb, r.nr, g, c_a, n_cta, cont);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rows = gq * kHeadDim;                  // floats of one partial's rows
+  float* wv = scratch;                             // [gq][cnt] maxima, then weights
+  float* lv = wv + gq * cnt;                       // [gq][cnt] sums
+  float* lsum = lv + gq * cnt;                     // [gq]
+  float* osm = scratch + ((2 * gq * cnt + gq + 3) / 4) * 4;  // [cnt][gq][128], 16-byte aligned
+  const bool staged = ((size_t)(osm - scratch) + (size_t)cnt * rows) * 4 <= scratch_bytes;
+  const long long s0 = (long long)c_a + r.p;       // first CTA slot
+  const long long sw = warp_slot(gridDim.x, P, r.p);
+  auto slot = [&](int k) -> long long { return k < n_cta ? s0 + k : sw; };
+  for (int i = threadIdx.x; i < gq * cnt; i += kThreads) {
+    const int gg = i / cnt, k = i % cnt;
+    wv[i] = __ldcg(ws.m + slot(k) * gq + gg);
+    lv[i] = __ldcg(ws.l + slot(k) * gq + gg);
+  }
+  if (staged) {
+    const float4* src = reinterpret_cast<const float4*>(ws.o + s0 * rows);
+    float4* dst = reinterpret_cast<float4*>(osm);
+    const int n4 = n_cta * rows / 4;
+    for (int i = threadIdx.x; i < n4; i += kThreads) dst[i] = __ldcg(src + i);
+    if (cont) {
+      const float4* sw4 = reinterpret_cast<const float4*>(ws.o + sw * rows);
+      for (int i = threadIdx.x; i < rows / 4; i += kThreads) dst[n4 + i] = __ldcg(sw4 + i);
+    }
+  }
+  __syncthreads();
+  for (int gg = warp; gg < gq; gg += kWarps) {
+    float M = -INFINITY;
+    for (int k = lane; k < cnt; k += 32) M = fmaxf(M, wv[gg * cnt + k]);
+    M = warp_max(M);
+    float Ls = 0.0f;
+    for (int k = lane; k < cnt; k += 32) {
+      const float m = wv[gg * cnt + k];
+      const float w = (m == -INFINITY) ? 0.0f : exp2f(m - M);
+      Ls += w * lv[gg * cnt + k];
+      wv[gg * cnt + k] = w;
+    }
+    Ls = warp_sum(Ls);
+    if (lane == 0) lsum[gg] = Ls;
+  }
+  __syncthreads();
+  const long long head0 = (long long)(r.p / d.hkv) * d.hq + (long long)(r.p % d.hkv) * gq;
+  for (int it = threadIdx.x; it < rows; it += kThreads) {
+    const int gg = it / kHeadDim;
+    float o = 0.0f;
+    if (staged) {
+      for (int k = 0; k < cnt; ++k) o = fmaf(wv[gg * cnt + k], osm[k * rows + it], o);
+    } else {
+      for (int k = 0; k < cnt; ++k) o = fmaf(wv[gg * cnt + k], __ldcg(ws.o + slot(k) * rows + it), o);
+    }
+    const float Ls = lsum[gg];
+    store_out(out, out_f16, head0 * kHeadDim + it, Ls > 0.0f ? o / Ls : 0.0f);
+  }
+  if (threadIdx.x == 0) ws.tk[r.p] = 0u;
+  __syncthreads();
+}
+
+
+// A warp's walk over its pairs and the segment it is folding, in shared
+// memory.
+struct WarpCtx {
+  Walk w;                        // the pair the walk is at
+  SegRec seg;                    // the segment being folded
+  long long a, e;                // the warp's unit range
+  int i0, i1;                    // the segment's window chunks
+  int last, last_v;              // the segment ends the range; last virtual warp
+  int pre, pre_end, lo_h, p_h;   // early copies: count, end block, first block, pair
+  int pos;                       // ring slots used
+  uint32_t wphase;               // window staging barrier parity count
+  int j1;                        // the segment's end block
+};
 
 // ---------------------------------------------------------------------------
 // The kernel
@@ -1149,275 +648,384 @@ __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
 template <int BK, int BV, bool kWide>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     decode_attn_kernel(Dims d, kvq_cache c, const __half* __restrict__ q, void* __restrict__ out,
-                       int out_f16, float scale_log2, int S, unsigned smem_size, Ws ws,
+                       int out_f16, float scale_log2, unsigned smem_size, Ws ws,
                        const __half* __restrict__ k_new, const __half* __restrict__ v_new) {
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ MergeSmall ms;
-  __shared__ int len_s[2];  // length attended, length before the append
-  __shared__ __align__(16) __half q_s[kHeads * kHeadDim];  // the CTA's query heads
-  __shared__ __align__(8) uint64_t wbar[kWarps];      // a window warp's staging barrier
-  __shared__ __align__(8) uint64_t fl_bar;            // page image of a flush complete
+  __shared__ __align__(8) uint64_t wbar[kWarps];  // a warp's window-row staging barrier
+  __shared__ SegRec rec[kWarps];                  // each warp's final state (p < 0: none)
+  __shared__ SegRec fin[kFinCap];                 // pairs whose partials this CTA completed
+  __shared__ int fin_n;
+  __shared__ int pub_last;
+  __shared__ WarpCtx wctx[kWarps];                // each warp's walk and segment
+  __shared__ FlatGrid grid_s;                     // the plan's grid
+  __shared__ int len_s[kLenCap];                  // the lengths the plan reads (batch <= kLenCap)
+  __shared__ MergeGroups mg;
 
-  const int h = blockIdx.y, b = blockIdx.z;
-  const int gq = d.gq;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int NV = gridDim.x * kWarps;     // warps per (sequence, kv-head)
-  const int v = blockIdx.x * kWarps + warp;
   pdl_launch_dependents();
-  const long long bh = (long long)b * d.hkv + h;
-  const PageMap pm = page_map(d, c, b, h);
-  TableWin tw;
-  table_win_init(tw);
-  const __half* ring_k = reinterpret_cast<const __half*>(c.k_resid) + bh * d.ring * kHeadDim;
-  const __half* ring_v = reinterpret_cast<const __half*>(c.v_resid) + bh * d.ring * kHeadDim;
-  const long long head0 = (long long)b * d.hq + (long long)h * gq;
-  const __half* qh = q + head0 * kHeadDim;
-  unsigned* flag = reinterpret_cast<unsigned*>(c.seq_len) + d.batch;
-  // Decode step (k_new given): this kernel appends one token per sequence
-  // before attending.  seq_len[b] is read once per CTA; the last CTA of the
-  // sequence to have read it (ticket) publishes L0 + 1.
   const bool append = k_new != nullptr;
-  unsigned seq_ticket = 0u;
+  const int P = d.batch * d.hkv, gq = d.gq;
+  constexpr int page = page_bytes_c(BK, BV);
+  constexpr int R = ring_slots(page);
+  const int wbytes = warp_ring_bytes(page);
+  char* ring = reinterpret_cast<char*>(smem) + (size_t)warp * wbytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kWarps * wbytes) + warp * R;
+  // 512 bytes at the end of shared memory: metadata rows of the zero-point
+  // MMAs that carry no block, all zero except bytes 256..319, which only the
+  // value zero-point MMA's row 4 reads: fp16 ones, so that row sums the
+  // softmax weights (the row sum l).
+  unsigned* zero = reinterpret_cast<unsigned*>(smem + smem_size - 16 - kZeroBytes);
+  for (int i = threadIdx.x; i < kZeroBytes / 4; i += kThreads)
+    zero[i] = i >= kOnesWord0 && i < kOnesWord0 + 16 ? 0x3C003C00u : 0u;
+  unsigned* flag = reinterpret_cast<unsigned*>(c.seq_len) + d.batch;
+  if (threadIdx.x == 0) fin_n = 0;
+  if (lane == 0) {
+    for (int i = 0; i < R; ++i) mbar_init(full + i, 1);
+    mbar_init(&wbar[warp], 1);
+    fence_mbar_init();
+    rec[warp].p = -1;
+  }
+  __syncwarp();
 
+  WarpCtx& X = wctx[warp];
+  if (lane == 0) {
+    X.pre = 0;
+    X.pre_end = 0;
+    X.lo_h = -1;
+    X.p_h = -1;
+    X.pos = 0;
+    X.wphase = 0u;
+    X.last = 0;
+  }
+  __syncwarp();
+  // The plan reads the lengths many times: one coalesced read into shared
+  // memory after the dependency wait instead of global round trips.  (No
+  // copies are started before the wait: the next CTA of an SM starts only
+  // when the previous kernel's CTA there has left, so little would overlap,
+  // and the reads after the wait would queue behind them.)
+  const int* lens = d.batch <= kLenCap ? len_s : c.seq_len;
+  __syncthreads();  // zero rows written
+  pdl_wait();
+
+  // ---- the plan from the lengths after the wait ----
+  // (kept in shared memory: it is needed again only after the streaming)
+  if (d.batch <= kLenCap)
+    for (int b = threadIdx.x; b < d.batch; b += kThreads) len_s[b] = read_len(c.seq_len + b);
+  __syncthreads();
   {
-    constexpr int page = page_bytes_c(BK, BV);
-    const int R = ring_slots(page);
-    const int wbytes = warp_ring_bytes(page);
-    char* ring = reinterpret_cast<char*>(smem) + (size_t)warp * wbytes;
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kWarps * wbytes) + warp * R;
-    // 512 bytes at the end of shared memory: metadata rows of the
-    // zero-point MMAs that carry no block, all zero except bytes 256..319,
-    // which only the value zero-point MMA's row 4 reads: fp16 ones, so that
-    // row sums the softmax weights (the row sum l).
-    unsigned* zero = reinterpret_cast<unsigned*>(smem + smem_size - 16 - kZeroBytes);
-    for (int i = threadIdx.x; i < kZeroBytes / 4; i += kThreads)
-      zero[i] = i >= kOnesWord0 && i < kOnesWord0 + 16 ? 0x3C003C00u : 0u;
-    int hint = 0;
-    if (lane == 0) {
-      for (int i = 0; i < R; ++i) mbar_init(full + i, 1);
-      mbar_init(&wbar[warp], 1);
-      if (warp == 0) mbar_init(&fl_bar, 4 * 32);
-      fence_mbar_init();
-      hint = read_len(c.seq_len + b);
-    }
-    hint = __shfl_sync(0xffffffffu, hint, 0);
-    if (append && hint < d.max_len) ++hint;  // the length this kernel will attend
-    __syncwarp();
-    const Plan ph = make_plan(hint, d.residual, NV);
-    int lo_h = 0, hi_h = 0, pre = 0, pre_end = 0;
-    if (v < ph.np) {
-      block_range(ph, v, lo_h, hi_h);
-      // the newest block may be the one the previous kernel is writing
-      pre = tc_pre_issue<BK, BV>(pm, tw, lo_h, hi_h, ph.nb - 1, ring, full, R, pre_end, flag);
-      // a decode step that pushes a group out of the window: its owner brings
-      // the group's ring rows (old, unchanging) into L2 for the flush
-      if (append && lane == 0 && hi_h == ph.nb && ph.nb > 0 &&
-          ph.Lq > packed_len(hint - 1, d.residual)) {
-        prefetch_rows_l2(ring_k, ph.Lq - kGroup, kGroup, d.ring);
-        prefetch_rows_l2(ring_v, ph.Lq - kGroup, kGroup, d.ring);
-      }
-    } else if (lane == 0) {
-      // window rows of the length read before the wait into L2 (rows below
-      // the newest token do not change; this is a hint, nothing waits on it)
-      const int last = hint - (append ? 1 : 0) - 1;  // newest row not yet written
-      for (int u = v - ph.np; u < ph.n_res; u += ph.n_resw) {
-        const int p0 = ph.Lq + u * kGroup;
-        const int n = min(kGroup, last - p0);
-        if (n > 0) {
-          prefetch_rows_l2(ring_k, p0, n, d.ring);
-          prefetch_rows_l2(ring_v, p0, n, d.ring);
-        }
-      }
-    }
-    __syncthreads();  // zero rows written
-    pdl_wait();
-    // q (written by the previous kernel) into shared memory while the length
-    // is read: one round trip for both
-    if (threadIdx.x < gq * kHeadDim / 8)
-      cp_async16(q_s + threadIdx.x * 8, qh + threadIdx.x * 8, 16u);
-    asm volatile("cp.async.commit_group;" ::: "memory");
-    if (threadIdx.x == 0) {
-      const int L0 = read_len(c.seq_len + b);
-      int L = L0;
-      if (append) {
-        if (L0 < d.max_len) L = L0 + 1;
-        else atomicOr(flag, (unsigned)KVQ_FLAG_OVERFLOW);
-      }
-      len_s[0] = L;
-      len_s[1] = L0;
-    }
-    asm volatile("cp.async.wait_group 0;" ::: "memory");
-    __syncthreads();
-    const int L = len_s[0], L0 = len_s[1];
-    const bool grew = L > L0;  // this kernel appends the token at position L0
-    if (append && threadIdx.x == 0)
-      seq_ticket = atomicAdd(reinterpret_cast<unsigned*>(c.seq_len) + d.batch + 2 + b, 1u);
-    const __half* k_row = grew ? k_new + bh * kHeadDim : nullptr;
-    const __half* v_row = grew ? v_new + bh * kHeadDim : nullptr;
-    if (grew && blockIdx.x == 0 && warp == 0) {  // the new token into its ring slot
-      const long long slot = (long long)(L0 % d.ring) * kHeadDim;
-      __half* rk = const_cast<__half*>(ring_k) + slot;
-      __half* rv = const_cast<__half*>(ring_v) + slot;
-      if (lane < 16) reinterpret_cast<uint4*>(rk)[lane] = reinterpret_cast<const uint4*>(k_row)[lane];
-      else reinterpret_cast<uint4*>(rv)[lane - 16] = reinterpret_cast<const uint4*>(v_row)[lane - 16];
-    }
-    const bool same = L == hint;  // the plan made before the wait holds
-    const Plan p = same ? ph : make_plan(L, d.residual, NV);
-    const int flush_blk = grew && p.Lq > packed_len(L0, d.residual) ? p.nb - 1 : -1;
-    const bool packed = v < p.np;
-    // A flush is folded in by the packed warp np - 1 (it owns the last
-    // block).  The window warps of its CTA quantize the block's four quarters
-    // into the image while it streams; with no window warp in that CTA it
-    // does them itself, before streaming.
-    char* image = reinterpret_cast<char*>(smem + smem_size - 16 - kZeroBytes - image_bytes(page));
-    const int cta_f = (p.np - 1) / kWarps;
-    const int n_help = (cta_f + 1) * kWarps - p.np;  // window warps in CTA cta_f
-    if (flush_blk >= 0 && (int)blockIdx.x == cta_f && (n_help > 0 ? !packed : v == p.np - 1)) {
-      const int nw = n_help > 0 ? n_help : 1;
-      for (int qi = n_help > 0 ? v - p.np : 0; qi < 4; qi += nw) {
-        flush_quarter<BK, BV>(ring_k, ring_v, flush_blk * kGroup, d.ring, qi, image);
-        mbar_arrive(&fl_bar);
-      }
-    }
-    TcState st;
-    init_state(st);
-    if (packed || pre > 0) {
-      // a warp that streamed early retires its slots even if it now has no blocks
-      int lo = lo_h, hi = hi_h;
-      if (!same) {
-        lo = hi = 0;
-        if (packed) block_range(p, v, lo, hi);
-      }
-      tc_packed_warp<BK, BV, kWide>(pm, tw, lo_h, pre, pre_end, lo, hi, ring, full, R,
-                             reinterpret_cast<const char*>(zero), q_s, gq, scale_log2, flag, st,
-                             flush_blk, &fl_bar, image);
-    }
-    if (!packed)
-      tc_window_warp<BK, BV, kWide>(d, ring_k, ring_v, p, L, v - p.np, p.n_resw, ring, q_s, gq,
-                             scale_log2, st, grew ? L0 : -1, k_row, v_row, &wbar[warp], flag);
-    // the warp's ring is idle now: its state goes to the start of it
-    WarpState& mine = *reinterpret_cast<WarpState*>(ring);
-    if (packed) tc_write_state<true, BV, kWide>(st, mine, lane);
-    else tc_write_state<false, BV, kWide>(st, mine, lane);
+    const FlatGrid g0 = flat_grid(plan_sums(lens, d, append), gridDim.x);
+    if (threadIdx.x == 0) grid_s = g0;
   }
   __syncthreads();
+  const FlatGrid& g = grid_s;
+  if (g.N == 0 && blockIdx.x == 0 && warp == 0)
+    for (int i = lane; i < P * gq * kHeadDim; i += 32) store_out(out, out_f16, i, 0.0f);
+  // Early copies still in flight that no packed range consumed land before
+  // the ring is used otherwise (bounded waits).
+  auto drain_pre = [&]() {
+    const int pre = X.pre;
+    if (pre > 0) {
+      if (lane == 0) {
+        for (int s = 0; s < pre; ++s) mbar_wait(full + s % R, (s / R) & 1);
+        X.pos = pre;
+        X.pre = 0;
+      }
+      __syncwarp();
+    }
+  };
+  // A state the warp leaves for the next pair: its pair's only partial goes
+  // out directly, any other to the warp slot and the pair's ticket.
+  auto emit_warp_partial = [&](const TcState& st, bool packed_kind, const SegRec& r,
+                               long long head0) {
+    int c_a, n_cta;
+    bool cont;
+    const int cnt = pair_partials(r.U, r.pc, r.nb, r.nr, g, c_a, n_cta, cont);
+    WarpState& s = *reinterpret_cast<WarpState*>(ring);
+    if (packed_kind) tc_write_state<true, BV, kWide>(st, s, lane);
+    else tc_write_state<false, BV, kWide>(st, s, lane);
+    __syncwarp();
+    if (cnt == 1) {
+      warp_state_out(s, out, out_f16, head0, gq, lane);
+    } else {
+      const long long sl = warp_slot(gridDim.x, P, r.p);
+      for (int i = lane; i < gq * kHeadDim; i += 32)
+        ws.o[sl * gq * kHeadDim + i] = s.o[i / kHeadDim][i % kHeadDim];
+      if (lane < gq) {
+        ws.m[sl * gq + lane] = s.m[lane];
+        ws.l[sl * gq + lane] = s.l[lane];
+      }
+      __threadfence();
+      __syncwarp();
+      if (lane == 0 && atom_add_acq_rel(&ws.tk[r.p], 1u) == (unsigned)cnt - 1u) {
+        const int i = atomicAdd(&fin_n, 1);
+        if (i < kFinCap) fin[i] = r;
+      }
+    }
+    __syncwarp();
+  };
 
-  // ---- merge the warps of this CTA: one partial per query head ----
-  const size_t wstride = (size_t)warp_ring_bytes(page_bytes_c(BK, BV));
+  // The walk and the current segment live in shared memory (X): nothing of
+  // them holds registers across the streaming loop, which gets them all.
+  const int v = (int)blockIdx.x < g.n_cta ? cta_first_v(blockIdx.x, g) + warp : -1;
+  if (v >= 0 && v < cta_first_v(blockIdx.x + 1, g)) {
+    {
+      const long long a = v_first_unit(v, g);
+      const Walk w0 = walk_start(a, lens, d, append, g.k);
+      if (lane == 0) {
+        X.w = w0;
+        X.a = a;
+        X.e = v_first_unit(v + 1, g);
+        X.last_v = v == g.n_v - 1;
+      }
+      __syncwarp();
+    }
+    for (;;) {
+      Walk w = X.w;
+      if (w.b >= d.batch) break;
+      const long long a = X.a, e = X.e;
+      const bool last_v = X.last_v;
+      const long long U = w.Ub + (long long)w.h * w.pc;
+      const int p = w.b * d.hkv + w.h;
+      const long long head0 = (long long)w.b * d.hq + (long long)w.h * gq;
+      // empty pairs: zero output from the warp whose range holds their unit
+      // (the last warp takes those at the very end)
+      if (U >= e && !(last_v && U >= g.N)) break;
+      if (w.pc == 0) {
+        if (U >= a)
+          for (int i = lane; i < gq * kHeadDim; i += 32) store_out(out, out_f16, head0 * kHeadDim + i, 0.0f);
+        walk_next(w, lens, d, append, g.k);
+        __syncwarp();
+        if (lane == 0) X.w = w;
+        __syncwarp();
+        continue;
+      }
+      const PairShape s = pair_shape(w.L, d.residual);
+      const int k0 = items_below(a - U, s.nb, s.nr, g.k), k1 = items_below(e - U, s.nb, s.nr, g.k);
+      if (lane == 0) X.last = U + w.pc >= e;
+      __syncwarp();
+      if (k1 > k0) {
+        const int j0 = min(k0, s.nb), j1 = min(k1, s.nb);
+        const int i0 = max(k0 - s.nb, 0), i1 = max(k1 - s.nb, 0);
+        const long long bh = (long long)w.b * d.hkv + w.h;
+        const __half* ring_k = reinterpret_cast<const __half*>(c.k_resid) + bh * d.ring * kHeadDim;
+        const __half* ring_v = reinterpret_cast<const __half*>(c.v_resid) + bh * d.ring * kHeadDim;
+        const bool grew = w.L > w.L0;  // this kernel appends the token at position L0
+        if (grew && k0 == 0) {  // the new token into its ring slot
+          const long long sl = (long long)(w.L0 % d.ring) * kHeadDim;
+          __half* rk = const_cast<__half*>(ring_k) + sl;
+          __half* rv = const_cast<__half*>(ring_v) + sl;
+          if (lane < 16) reinterpret_cast<uint4*>(rk)[lane] = reinterpret_cast<const uint4*>(k_new + bh * kHeadDim)[lane];
+          else reinterpret_cast<uint4*>(rv)[lane - 16] = reinterpret_cast<const uint4*>(v_new + bh * kHeadDim)[lane - 16];
+        }
+        if (i1 > i0 && lane == 0) {
+          // window rows into L2 while the packed blocks stream (a hint; the
+          // newest row is not written yet)
+          const int p0 = s.Lq + i0 * kGroup;
+          const int n = min(w.L, s.Lq + i1 * kGroup) - (grew ? 1 : 0) - p0;
+          if (n > 0) {
+            prefetch_rows_l2(ring_k, p0, n, d.ring);
+            prefetch_rows_l2(ring_v, p0, n, d.ring);
+          }
+        }
+        if (lane == 0) {
+          X.seg.U = U;
+          X.seg.p = p;
+          X.seg.pc = w.pc;
+          X.seg.nb = s.nb;
+          X.seg.nr = s.nr;
+          X.i0 = i0;
+          X.i1 = i1;
+          X.j1 = j1;
+        }
+        __syncwarp();
+        TcState st;
+        init_state(st);
+        if (j1 > j0) {
+          // the early slots (ring positions 0 .. pre - 1) are this range's
+          // first ones if it begins where the early plan's did; a block that
+          // leaves the window in this kernel folds after the streamed ones
+          const bool flush = grew && s.Lq > packed_len(w.L0, d.residual) && j1 == s.nb;
+          const char* tail = nullptr;
+          st = tc_packed_warp<BK, BV, kWide>(st, page_map(d, c, w.b, w.h), p == X.p_h ? X.lo_h : -1,
+                                             X.pre, X.pre_end, j0, flush ? j1 - 1 : j1, ring, full,
+                                             &X.pos, reinterpret_cast<const char*>(zero),
+                                             q + head0 * kHeadDim, gq, scale_log2, flag, flush,
+                                             &tail);
+          __syncwarp();
+          if (lane == 0) X.pre = 0;
+          __syncwarp();
+          {
+            // the flush (segment read back from X)
+            const Walk wf = X.w;
+            const PairShape sf = pair_shape(wf.L, d.residual);
+            if (wf.L > wf.L0 && sf.Lq > packed_len(wf.L0, d.residual) && X.j1 == sf.nb) {
+              const long long bhf = (long long)wf.b * d.hkv + wf.h;
+              st = tc_fold_flush<BK, BV, kWide>(
+                  st, page_map(d, c, wf.b, wf.h), sf.nb - 1, tail, ring,
+                  reinterpret_cast<const char*>(zero),
+                  q + ((long long)wf.b * d.hq + (long long)wf.h * gq) * kHeadDim, gq, scale_log2,
+                  flag, reinterpret_cast<const __half*>(c.k_resid) + bhf * d.ring * kHeadDim,
+                  reinterpret_cast<const __half*>(c.v_resid) + bhf * d.ring * kHeadDim, d.ring);
+            }
+          }
+          if (X.i1 > X.i0) {
+            // the window chunks continue this state in their own layout
+            WarpState& t = *reinterpret_cast<WarpState*>(ring);
+            tc_write_state<true, BV, kWide>(st, t, lane);
+            __syncwarp();
+            tc_read_state<kWide>(st, t, lane);
+            __syncwarp();
+          }
+        }
+        // everything below reads the segment back from X
+        const SegRec r = X.seg;
+        const Walk wr = X.w;
+        const bool has_w = X.i1 > X.i0;
+        if (has_w) {
+          drain_pre();
+          const long long bh2 = (long long)wr.b * d.hkv + wr.h;
+          const PairShape s2 = pair_shape(wr.L, d.residual);
+          const bool grew2 = wr.L > wr.L0;
+          st = tc_window_chunks<BK, BV, kWide>(
+              st, d, reinterpret_cast<const __half*>(c.k_resid) + bh2 * d.ring * kHeadDim,
+              reinterpret_cast<const __half*>(c.v_resid) + bh2 * d.ring * kHeadDim, s2.Lq, wr.L,
+              X.i0, X.i1, ring, q + ((long long)wr.b * d.hq + (long long)wr.h * gq) * kHeadDim, gq,
+              scale_log2, grew2 ? wr.L0 : -1, grew2 ? k_new + bh2 * kHeadDim : nullptr,
+              grew2 ? v_new + bh2 * kHeadDim : nullptr, &wbar[warp], &X.wphase, flag);
+        }
+        drain_pre();
+        if (X.last) {
+          WarpState& t = *reinterpret_cast<WarpState*>(ring);
+          if (!has_w) tc_write_state<true, BV, kWide>(st, t, lane);
+          else tc_write_state<false, BV, kWide>(st, t, lane);
+          if (lane == 0) rec[warp] = r;
+        } else {
+          emit_warp_partial(st, !has_w, r,
+                            (long long)(r.p / d.hkv) * d.hq + (long long)(r.p % d.hkv) * gq);
+        }
+      }
+      {
+        Walk wn = X.w;
+        const bool stop = X.last && !X.last_v;
+        walk_next(wn, lens, d, append, g.k);
+        __syncwarp();
+        if (lane == 0) X.w = wn;
+        __syncwarp();
+        if (stop) break;
+      }
+    }
+  }
+  drain_pre();
+  __syncthreads();
+
+  // ---- merge the warps of this CTA that end in the same pair ----
+  // Groups are runs of warps with the same final pair (warp order is unit
+  // order).  All groups merge at once, then their tickets go out together.
+  const size_t wstride = (size_t)wbytes;
   auto wstate = [&](int w) -> const WarpState& {
     return *reinterpret_cast<const WarpState*>(smem + (size_t)w * wstride);
   };
-  if (threadIdx.x < kWarps * gq) {
-    const int w = threadIdx.x / gq, g = threadIdx.x % gq;
-    float M = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < kWarps; ++i) M = fmaxf(M, wstate(i).m[g]);
-    const float m = wstate(w).m[g];
-    ms.ww[w][g] = (m == -INFINITY) ? 0.0f : exp2f(m - M);
-    if (w == 0) ms.cta_m[g] = M;
+  if (warp == 0) {  // groups from two ballots over the warps' final pairs
+    const int p = lane < kWarps ? rec[lane].p : -1;
+    const int prev = lane > 0 && lane < kWarps ? rec[lane - 1].p : -2;
+    const int next = lane + 1 < kWarps ? rec[lane + 1].p : -2;
+    const unsigned starts = __ballot_sync(0xffffffffu, p >= 0 && prev != p);
+    const unsigned ends = __ballot_sync(0xffffffffu, p >= 0 && next != p);
+    const unsigned below = (1u << lane) - 1u;
+    if (starts & (1u << lane)) mg.w0[__popc(starts & below)] = lane;
+    if (ends & (1u << lane)) mg.w1[__popc(ends & below)] = lane + 1;
+    if (lane == 0) mg.n = __popc(starts);
   }
   __syncthreads();
-  const int n_items = gq * kHeadDim;
-  for (int it = threadIdx.x; it < n_items; it += kThreads) {
-    const int g = it / kHeadDim, ch = it % kHeadDim;
-    float o = 0.0f, l = 0.0f;
+  const int ng = mg.n;
+  if (threadIdx.x < ng) {  // a group's partial count, once (64-bit divisions)
+    const SegRec r = rec[mg.w0[threadIdx.x]];
+    int c_a, n_cta;
+    bool cont;
+    mg.cnt[threadIdx.x] = pair_partials(r.U, r.pc, r.nb, r.nr, g, c_a, n_cta, cont);
+  }
+  if (threadIdx.x < ng * gq) {  // (group, head): maximum and warp weights
+    const int k = threadIdx.x / gq, gg = threadIdx.x - k * gq;
+    const int w0 = mg.w0[k], w1 = mg.w1[k];
+    float mw[kWarps];
+    float M = -INFINITY;
 #pragma unroll
-    for (int i = 0; i < kWarps; ++i) {
-      const float w = ms.ww[i][g];
-      o = fmaf(w, wstate(i).o[g][ch], o);
-      l = fmaf(w, wstate(i).l[g], l);
+    for (int w = 0; w < kWarps; ++w) {  // independent loads, then the maximum
+      mw[w] = w >= w0 && w < w1 ? wstate(w).m[gg] : -INFINITY;
+      M = fmaxf(M, mw[w]);
     }
-    if (S == 1) {
-      store_out(out, out_f16, (head0 + g) * kHeadDim + ch, l > 0.0f ? o / l : 0.0f);
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w)
+      if (w >= w0 && w < w1) ms.ww[w][gg] = mw[w] == -INFINITY ? 0.0f : fast_exp2(mw[w] - M);
+    ms.gm[k][gg] = M;
+  }
+  __syncthreads();
+  for (int it = threadIdx.x; it < ng * gq * kHeadDim; it += kThreads) {
+    const int ch = it & (kHeadDim - 1), kg = it >> 7;  // kHeadDim == 128
+    const int k = kg / gq, gg = kg - k * gq;
+    const int w0 = mg.w0[k], w1 = mg.w1[k];
+    float o = 0.0f, l = 0.0f;
+    for (int w = w0; w < w1; ++w) {
+      const float wt = ms.ww[w][gg];
+      o = fmaf(wt, wstate(w).o[gg][ch], o);
+      l = fmaf(wt, wstate(w).l[gg], l);
+    }
+    const int pp = rec[w0].p;
+    if (mg.cnt[k] == 1) {
+      const long long head0 = (long long)(pp / d.hkv) * d.hq + (long long)(pp % d.hkv) * gq;
+      store_out(out, out_f16, (head0 + gg) * kHeadDim + ch, l > 0.0f ? o / l : 0.0f);
     } else {
-      const long long row = (head0 + g) * S + blockIdx.x;
-      ws.o[row * kHeadDim + ch] = o;
+      const long long sl = (long long)blockIdx.x + pp;
+      ws.o[(sl * gq + gg) * kHeadDim + ch] = o;
       if (ch == 0) {
-        ws.m[row] = ms.cta_m[g];
-        ws.l[row] = l;
+        ws.m[sl * gq + gg] = ms.gm[k][gg];
+        ws.l[sl * gq + gg] = l;
       }
     }
   }
-  if (append && threadIdx.x == 0 &&
-      seq_ticket == gridDim.y * gridDim.x - 1u) {  // every CTA of b has read L0
-    const int L1 = len_s[0];
-    __threadfence();
-    c.seq_len[b] = L1;
-    reinterpret_cast<unsigned*>(c.seq_len)[d.batch + 2 + b] = 0u;
+  __syncthreads();
+  if (threadIdx.x < ng && mg.cnt[threadIdx.x] > 1) {
+    const SegRec r = rec[mg.w0[threadIdx.x]];
+    __threadfence();  // cumulativity: the CTA's partial rows before the ticket
+    if (atom_add_acq_rel(&ws.tk[r.p], 1u) == (unsigned)mg.cnt[threadIdx.x] - 1u) {
+      const int i = atomicAdd(&fin_n, 1);
+      if (i < kFinCap) fin[i] = r;
+    }
   }
-  if (S == 1) return;
+  __syncthreads();
 
-  // ---- the last CTA of this (sequence, kv-head) merges the S partials ----
-  __syncthreads();
-  if (threadIdx.x == 0) ms.last = atom_add_acq_rel(&ws.tk[bh], 1u) == (unsigned)S - 1;
-  __syncthreads();
-  if (!ms.last) return;
-  // The partial rows of this (sequence, kv-head) are one contiguous range: a
-  // bulk copy brings them into shared memory (when they fit) while the maxima
-  // and sums are loaded and turned into weights.
-  const size_t o_bytes = (size_t)gq * S * kHeadDim * sizeof(float);
-  float* wv = reinterpret_cast<float*>(smem);           // [gq][S] maxima, then weights
-  float* lv = wv + gq * S;                               // [gq][S] sums
-  float* lsum = lv + gq * S;                             // [gq]
-  // the bulk copy's destination starts on a 128-byte boundary
-  const size_t head_bytes = ((size_t)(2 * gq * S + 16) * sizeof(float) + 127) / 128 * 128;
-  float* osm = reinterpret_cast<float*>(smem + head_bytes);  // [gq][S][128]
-  const bool staged = head_bytes + o_bytes + 16 <= smem_size;
-  uint64_t* mbar = reinterpret_cast<uint64_t*>(smem + smem_size - 16);
-  if (staged && threadIdx.x == 0) {
-    mbar_init(mbar, 1);
-    fence_mbar_init();
-    asm volatile("fence.proxy.async.global;" ::: "memory");
-    mbar_expect_tx(mbar, (uint32_t)o_bytes);
-    bulk_g2s(osm, ws.o + head0 * S * kHeadDim, (uint32_t)o_bytes, mbar);
-  }
-  for (int i = threadIdx.x; i < gq * S; i += kThreads) {
-    wv[i] = __ldcg(ws.m + head0 * S + i);
-    lv[i] = __ldcg(ws.l + head0 * S + i);
-  }
-  __syncthreads();
-  for (int g = warp; g < gq; g += kWarps) {
-    float M = -INFINITY;
-    for (int k = lane; k < S; k += 32) M = fmaxf(M, wv[g * S + k]);
-    M = warp_max(M);
-    float Ls = 0.0f;
-    for (int k = lane; k < S; k += 32) {
-      const float m = wv[g * S + k];
-      const float w = (m == -INFINITY) ? 0.0f : exp2f(m - M);
-      Ls += w * lv[g * S + k];
-      wv[g * S + k] = w;
+  // ---- final merges of the pairs whose last partial came from this CTA ----
+  const int nf = min(fin_n, kFinCap);
+  for (int i = 0; i < nf; ++i)
+    final_merge(fin[i], g, d, ws, out, out_f16, reinterpret_cast<float*>(smem),
+                (size_t)kWarps * wbytes);
+
+  // ---- the decode step publishes the new lengths once every CTA is done ----
+  if (append) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      pub_last = atom_add_acq_rel(&ws.tk[P], 1u) == gridDim.x - 1u;
     }
-    Ls = warp_sum(Ls);
-    if (lane == 0) lsum[g] = Ls;
-  }
-  bool ok = true;
-  if (staged) ok = mbar_wait(mbar, 0);
-  __syncthreads();
-  for (int it = threadIdx.x; it < n_items; it += kThreads) {
-    const int g = it / kHeadDim, ch = it % kHeadDim;
-    float o = 0.0f;
-    if (staged && ok) {
-      const float* src = osm + (size_t)g * S * kHeadDim + ch;
-#pragma unroll 8
-      for (int k = 0; k < S; ++k) o = fmaf(wv[g * S + k], src[(size_t)k * kHeadDim], o);
-    } else {
-      const float* src = ws.o + (head0 + g) * S * kHeadDim + ch;
-#pragma unroll 8
-      for (int k = 0; k < S; ++k) o = fmaf(wv[g * S + k], __ldcg(src + (size_t)k * kHeadDim), o);
+    __syncthreads();
+    if (pub_last) {
+      for (int b = threadIdx.x; b < d.batch; b += kThreads) {
+        const int L0 = read_len(c.seq_len + b);
+        if (L0 < d.max_len) c.seq_len[b] = L0 + 1;
+        else atomicOr(flag, (unsigned)KVQ_FLAG_OVERFLOW);
+      }
+      if (threadIdx.x == 0) ws.tk[P] = 0u;
     }
-    const float Ls = lsum[g];
-    store_out(out, out_f16, (head0 + g) * kHeadDim + ch, Ls > 0.0f ? o / Ls : 0.0f);
   }
-  if (threadIdx.x == 0) ws.tk[bh] = 0u;
 }
 
 size_t smem_bytes(const Dims& d) {
   const int page = (int)d.page_bytes;
   const size_t rings = (size_t)kWarps * warp_ring_bytes(page) +
                        (size_t)kWarps * ring_slots(page) * sizeof(uint64_t);
-  // + a flushed block's page image, the zero rows of the packed warps and
-  // the final merge's mbarrier
-  return (rings + image_bytes(page) + kZeroBytes + 16 + 127) / 128 * 128;
+  // + the zero rows of the zero-point MMAs
+  return (rings + kZeroBytes + 16 + 127) / 128 * 128;
 }
 
 template <int BK, int BV, bool kWide>
@@ -1468,7 +1076,7 @@ struct LaunchOp {
     cudaError_t e = prepare<BK, BV, kWide>(d);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(S, d.hkv, d.batch);
+    cfg.gridDim = dim3(S);  // the flat plan's CTAs
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem_bytes(d);
     cfg.stream = st;
@@ -1477,7 +1085,7 @@ struct LaunchOp {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV, kWide>, d, c, q, out, out_f16, sl2, S,
+    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<BK, BV, kWide>, d, c, q, out, out_f16, sl2,
                            (unsigned)smem_bytes(d), ws, k_new, v_new);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
@@ -1507,35 +1115,40 @@ cudaError_t launch_wait_selftest(unsigned* flag, long long limit_cycles, cudaStr
   return cudaGetLastError();
 }
 
-// n_splits = CTAs per (sequence, kv-head); partial rows for exactly the
-// n_splits CTAs of the launch (the same carve the kernel uses).  Tickets: one
-// per (sequence, kv-head), sized one per query head.
-size_t attn_workspace_bytes(const Dims& d, int n_splits) {
-  const int S = n_splits;
-  const size_t nml = (size_t)d.batch * d.hq * S;
+// The flat plan on `ctas` CTAs: partial slots for the launch's CTAs and the
+// pairs (the same carve the kernel uses), one ticket per pair and the decode
+// step's count of finished CTAs.
+size_t attn_workspace_bytes(const Dims& d, int ctas) {
+  const size_t nml = ws_slots(d.batch, d.hkv, ctas) * (size_t)d.gq;
   return align256(nml * 4) * 2 + align256(nml * kHeadDim * 4) +
-         align256((size_t)d.batch * d.hq * 4);
+         align256(((size_t)d.batch * d.hkv + 1) * 4);
 }
 
 cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& c, const __half* q, void* out,
-                               int out_f16, float scale_log2, int n_splits, void* workspace,
+                               int out_f16, float scale_log2, int ctas, void* workspace,
                                cudaStream_t st) {
-  const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, n_splits);
-  return dispatch(d, LaunchOp{d, c, q, out, out_f16, scale_log2, n_splits, ws, st});
+  const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, ctas);
+  return dispatch(d, LaunchOp{d, c, q, out, out_f16, scale_log2, ctas, ws, st});
 }
 
 cudaError_t launch_decode_step(const Dims& d, const kvq_cache& c, const __half* k_new,
                                const __half* v_new, const __half* q, void* out, int out_f16,
-                               float scale_log2, int n_splits, void* workspace, cudaStream_t st) {
-  const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, n_splits);
-  LaunchOp op{d, c, q, out, out_f16, scale_log2, n_splits, ws, st};
+                               float scale_log2, int ctas, void* workspace, cudaStream_t st) {
+  const Ws ws = carve(workspace, d.batch, d.hq, d.hkv, ctas);
+  LaunchOp op{d, c, q, out, out_f16, scale_log2, ctas, ws, st};
   op.k_new = k_new;
   op.v_new = v_new;
   return dispatch(d, op);
 }
 
-// CTAs per (sequence, kv-head): enough for every resident CTA
-// slot of the GPU to hold one, with at least a few blocks per CTA.
+// CTAs of a flat-plan launch: one per resident CTA slot of the GPU.
+int attn_flat_ctas(int sm_count) {
+  const int n = kCtasPerSm * sm_count;
+  return n > kMaxSplits - 1 ? kMaxSplits - 1 : (n < 1 ? 1 : n);
+}
+
+// Split plan: CTAs per (sequence, kv-head) so that every resident CTA slot
+// of the GPU holds one, with at least a few blocks per CTA.
 int attn_default_splits(const Dims& d, int sm_count) {
   const int bh = d.batch * d.hkv;
   int n = kCtasPerSm * sm_count / bh;
@@ -1545,54 +1158,18 @@ int attn_default_splits(const Dims& d, int sm_count) {
   return n < 1 ? 1 : n;
 }
 
-// Split count from the sequence lengths, known to the caller on the host.
-// Up to half the SMs' worth of (sequence, kv-head) pairs: one wave, as
-// attn_default_splits, unless a few waves of shorter splits fill the SMs
-// that one wave leaves idle (the pair count does not divide the SM count).
-// The estimate of a count n, in units of one packed block's compute, is
-// waves(n) x (blocks per split + kCtaFixedBlocks): measured on GB300, a
-// CTA's fixed cost (start, warp and split merges) is ~6.4 us, ~46 blocks
-// (64 pairs of 64k-token K1V1 sequences: 7 splits in 2.95 waves take 140.6
-// us per layer against 156.7 for 2 splits in one wave).  A count is taken
-// only if it is estimated 2% faster, and at most four waves.  More pairs:
-// one split each for lengths within 15% of their mean; for a ragged batch
-// about four waves of CTAs, so the scheduler's dynamic fill evens out the
-// long and short sequences.
-constexpr int kCtaFixedBlocks = 46;
+// The plan for host-known lengths: the split plan (its count) when one wave
+// of its CTAs fills the GPU, as for batch-1 decoding, where a launch is bound
+// by latency;
+// otherwise 0, the flat plan, which streams every warp's share in one wave
+// instead of paying a CTA's start and merges once per wave (Qwen2.5-14B
+// shape, batch 8 x 64k, K1V1: 98.7 against 104.2 us per layer with 7 splits
+// in 2.95 waves).
 int attn_splits_for_lengths(const Dims& d, int sm_count, const int32_t* lengths) {
-  const int bh = d.batch * d.hkv;
-  long long sum = 0;
-  int mx = 0;
-  for (int b = 0; b < d.batch; ++b) {
-    sum += lengths[b];
-    mx = lengths[b] > mx ? lengths[b] : mx;
-  }
-  if (2 * bh <= sm_count) {
-    const int n1 = attn_default_splits(d, sm_count);
-    const double nb = (double)(packed_len(mx, d.residual) / kGroup);
-    const int slots = kCtasPerSm * sm_count;
-    const int cap = min((d.max_blocks + 3) / 4, kMaxSplits - 1);
-    auto estimate = [&](int n) {
-      const long long waves = ((long long)bh * n + slots - 1) / slots;
-      return (double)waves * (nb / n + kCtaFixedBlocks);
-    };
-    int best = n1;
-    double best_t = estimate(n1);
-    for (int n = n1 + 1; n <= cap && (long long)bh * n <= 4LL * slots; ++n) {
-      const double t = estimate(n);
-      if (t < 0.98 * best_t) {
-        best = n;
-        best_t = t;
-      }
-    }
-    return best;
-  }
-  if ((double)mx <= 1.15 * (double)sum / d.batch) return attn_default_splits(d, sm_count);
-  int n = (4 * sm_count + bh / 2) / bh;
-  const int cap = (d.max_blocks + 3) / 4;
-  if (n > cap) n = cap;
-  if (n > kMaxSplits - 1) n = kMaxSplits - 1;
-  return n < 1 ? 1 : n;
+  (void)lengths;
+  const long long bh = (long long)d.batch * d.hkv;
+  const int S = attn_default_splits(d, sm_count);
+  return (long long)S * bh * 10 >= 9LL * kCtasPerSm * sm_count ? S : 0;  // one wave, >= 90% full
 }
 
 // ---------------------------------------------------------------------------
@@ -1643,11 +1220,19 @@ cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& c, const _
   cudaError_t e = static_scratch(&ws);
   if (e != cudaSuccess) return e;
   // The array keeps the previous call's contents: the tickets must start at
-  // zero, the partials are always written before they are read.
-  const Ws w = carve(ws, d.batch, d.hq, d.hkv, n_splits);
-  e = cudaMemsetAsync(w.tk, 0, (size_t)d.batch * d.hq * sizeof(unsigned), st);
+  // zero, the partials are always written before they are read.  n_splits >
+  // 0: the split plan (attn_split.cu); < 0: the flat plan on -n_splits CTAs.
+  if (n_splits > 0) {
+    size_t tk_bytes = 0;
+    unsigned* tk = attn_split_tickets(d, n_splits, ws, &tk_bytes);
+    e = cudaMemsetAsync(tk, 0, tk_bytes, st);
+    if (e != cudaSuccess) return e;
+    return launch_decode_attn_split(d, c, q, out, 0, scale_log2, n_splits, ws, st);
+  }
+  const Ws w = carve(ws, d.batch, d.hq, d.hkv, -n_splits);
+  e = cudaMemsetAsync(w.tk, 0, ((size_t)d.batch * d.hkv + 1) * sizeof(unsigned), st);
   if (e != cudaSuccess) return e;
-  return launch_decode_attn(d, c, q, out, 0, scale_log2, n_splits, ws, st);
+  return launch_decode_attn(d, c, q, out, 0, scale_log2, -n_splits, ws, st);
 }
 
 }  // namespace kvq

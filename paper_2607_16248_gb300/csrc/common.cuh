@@ -12,7 +12,7 @@ namespace kvq {
 constexpr int kHeadDim = 128;
 constexpr int kGroup = 32;
 constexpr int kMaxGq = 8;        // largest n_q_heads / n_kv_heads supported
-constexpr int kMaxSplits = 256;    // splits per (sequence, kv-head), window split included
+constexpr int kMaxSplits = 256;    // bound on n_splits (split plan) and on a flat launch's CTAs
 constexpr int kMaxK = 64;        // largest DGAP recovery window
 constexpr int kMaxHidden = 1024; // largest DGAP hidden width
 
@@ -265,21 +265,35 @@ void set_error(const char* fmt, ...);
 cudaError_t launch_pack(const Dims& d, const kvq_cache& cache, const __half* k_new,
                         const __half* v_new, int n_new, int batch_begin,
                         int batch_count, cudaStream_t stream);
-// out is fp16 [batch][n_q_heads][128] when out_f16, else fp32.
+// Decode attention, the flat plan on `ctas` CTAs (attn.cu).  out is fp16
+// [batch][n_q_heads][128] when out_f16, else fp32.
 cudaError_t launch_decode_attn(const Dims& d, const kvq_cache& cache, const __half* q,
-                               void* out, int out_f16, float scale_log2, int n_splits,
+                               void* out, int out_f16, float scale_log2, int ctas,
                                void* workspace, cudaStream_t stream);
 // Append one token per sequence (k_new / v_new [batch][n_kv_heads][128]) and
-// attend in the same kernel.
+// attend in the same kernel, the flat plan.
 cudaError_t launch_decode_step(const Dims& d, const kvq_cache& cache, const __half* k_new,
                                const __half* v_new, const __half* q, void* out, int out_f16,
-                               float scale_log2, int n_splits, void* workspace,
+                               float scale_log2, int ctas, void* workspace,
                                cudaStream_t stream);
-size_t attn_workspace_bytes(const Dims& d, int n_splits);
+size_t attn_workspace_bytes(const Dims& d, int ctas);
+// The split plan, n_splits CTAs per (sequence, kv-head) (attn_split.cu).
+cudaError_t launch_decode_attn_split(const Dims& d, const kvq_cache& cache, const __half* q,
+                                     void* out, int out_f16, float scale_log2, int n_splits,
+                                     void* workspace, cudaStream_t stream);
+cudaError_t launch_decode_step_split(const Dims& d, const kvq_cache& cache,
+                                     const __half* k_new, const __half* v_new,
+                                     const __half* q, void* out, int out_f16,
+                                     float scale_log2, int n_splits, void* workspace,
+                                     cudaStream_t stream);
+size_t attn_split_workspace_bytes(const Dims& d, int n_splits);
+unsigned* attn_split_tickets(const Dims& d, int n_splits, void* workspace, size_t* bytes);
 int attn_default_splits(const Dims& d, int sm_count);
+int attn_flat_ctas(int sm_count);
 cudaError_t launch_wait_selftest(unsigned* flag, long long limit_cycles, cudaStream_t st);
 int attn_splits_for_lengths(const Dims& d, int sm_count, const int32_t* lengths);
 size_t attn_static_scratch_bytes();
+// n_splits > 0: the split plan; < 0: the flat plan on -n_splits CTAs.
 cudaError_t launch_decode_attn_static(const Dims& d, const kvq_cache& cache, const __half* q,
                                       float* out, float scale_log2, int n_splits,
                                       cudaStream_t stream);

@@ -330,11 +330,12 @@ def default_splits(cfg: CacheConfig):
 
 
 def splits_for_lengths(cfg: CacheConfig, lengths):
-    """kvq_attn_splits_for_lengths: a split count from host-known lengths."""
+    """kvq_attn_splits_for_lengths: the plan for host-known lengths, a split
+    count (> 0, the split plan) or 0 (the flat plan)."""
     c = cfg.c()
     arr = (ctypes.c_int32 * cfg.batch)(*[int(x) for x in lengths])
     n = lib().kvq_attn_splits_for_lengths(ctypes.byref(c), arr)
-    if n == 0:
+    if n < 0:
         raise KvqError(1, last_error())
     return n
 

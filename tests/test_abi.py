@@ -118,7 +118,14 @@ def test_workspace_sizes(L):
     s = L.kvq_attn_default_splits(ctypes.byref(c))
     assert 1 <= s <= 1024
     n = L.kvq_attn_workspace_bytes(ctypes.byref(c), 7)
+    # split plan, 7 CTAs per (sequence, kv-head): a partial (m, l and a
+    # 128-channel row) per (sequence, query head, CTA) and a ticket per pair
     assert n >= 2 * 32 * 7 * (128 + 2) * 4 + 2 * 8 * 4
+    # flat plan (0): a partial per CTA and two per pair, gq heads each, a
+    # ticket per pair and one counter
+    pairs, gq = 2 * 8, 32 // 8
+    flat = L.kvq_attn_workspace_bytes(ctypes.byref(c), 0)
+    assert flat >= (1 + 2 * pairs) * gq * (128 + 2) * 4 + (pairs + 1) * 4
     assert L.kvq_attn_workspace_bytes(ctypes.byref(c), 5000) == 0
     p = kvq._DgapParams(32, 64, 0.6, *([None] * 8))
     assert L.dgap_workspace_bytes(4, 128256, ctypes.byref(p)) > 4 * 32 * 33 * 8
@@ -135,23 +142,21 @@ def test_splits_for_lengths(L):
         c = cfg.c()
         return L.kvq_attn_splits_for_lengths(ctypes.byref(c), (ctypes.c_int32 * cfg.batch)(*lengths))
 
-    big = kvq.CacheConfig(batch=16, n_q_heads=32, n_kv_heads=8, bits_k=2, bits_v=2, max_len=32800)
-    d = L.kvq_attn_default_splits(ctypes.byref(big.c()))
-    assert n(big, [20000] * 16) == d  # uniform lengths: the default
-    assert n(big, [20000] * 15 + [22000]) == d  # within 15% of the mean
-    ragged = [8192 + 1500 * i for i in range(16)]
-    assert 3 <= n(big, ragged) <= 8 and n(big, ragged) > d  # about four waves
+    def default(cfg):
+        return L.kvq_attn_default_splits(ctypes.byref(cfg.c()))
+
+    # batch 1 (8 pairs): the split plan, one wave of 19 CTAs per pair
     one = kvq.CacheConfig(batch=1, n_q_heads=32, n_kv_heads=8, bits_k=1, bits_v=1, max_len=32800)
-    assert n(one, [32768]) == L.kvq_attn_default_splits(ctypes.byref(one.c()))
-    # 64 pairs (Qwen-14B shape, batch 8): one wave of 2 splits leaves 24 of
-    # 152 SMs idle; at 64k tokens 7 splits in 2.95 waves are faster, at 4k
-    # the fixed cost of each wave outweighs the fill
+    assert default(one) * 8 >= 0.9 * 152 and n(one, [32768]) == default(one)
+    # 64 pairs (Qwen-14B shape, batch 8): one wave of 2 splits leaves SMs idle,
+    # so the flat plan (0)
     qwen = kvq.CacheConfig(batch=8, n_q_heads=40, n_kv_heads=8, bits_k=1, bits_v=1, max_len=65664)
-    assert L.kvq_attn_default_splits(ctypes.byref(qwen.c())) == 2
-    assert n(qwen, [65536] * 8) == 7
-    assert n(qwen, [4096] * 8) == 2
-    assert n(big, [20000] * 15 + [40000]) == 0  # beyond max_len
-    assert n(big, [-1] + [20000] * 15) == 0
+    assert default(qwen) == 2 and n(qwen, [65536] * 8) == 0
+    big = kvq.CacheConfig(batch=16, n_q_heads=32, n_kv_heads=8, bits_k=2, bits_v=2, max_len=32800)
+    assert n(big, [20000] * 16) == 0
+    assert n(big, [8192 + 1500 * i for i in range(16)]) == 0
+    assert n(big, [20000] * 15 + [40000]) == -1  # beyond max_len
+    assert n(big, [-1] + [20000] * 15) == -1
 
 
 def test_compute_entry_points_reject_bad_arguments(L):

@@ -35,6 +35,6 @@ def test_trace_lines(kvq_lib, value, expect):
     if expect:
         assert any(l.startswith("kvq: kvq_pack ") for l in lines), r.stderr
         step = [l for l in lines if l.startswith("kvq: kvq_decode_step ")]
-        assert step and "grid (3, 2, 1) x 512, 3 splits" in step[0], lines
+        assert step and "grid (6) x 512, splits 3" in step[0], lines
     else:
         assert not lines
