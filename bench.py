@@ -66,7 +66,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--splits", type=int, default=0,
-                   help="CTAs per (sequence, kv-head); 0 = kvq_attn_splits_for_lengths")
+                   help="CTAs per (sequence, kv-head) (the split plan); default: "
+                        "kvq_attn_splits_for_lengths (0 = the flat plan)")
     p.add_argument("--paged", action="store_true",
                    help="run the caches on the paged layout (block table, shuffled pool)")
     p.add_argument("--cpu-worker", default="", help=argparse.SUPPRESS)
@@ -121,7 +122,10 @@ def attn_profile(workload):
     return PROFILES / f"attn_{workload.replace('-', '_')}.md"
 
 
-def profiled_traffic(path, sources=("attn.cu", "common.cuh"), sha_key="attn_source_sha"):
+ATTN_SOURCES = ("attn.cu", "attn_split.cu", "attn_core.cuh", "common.cuh")
+
+
+def profiled_traffic(path, sources=ATTN_SOURCES, sha_key="attn_source_sha"):
     """DRAM bytes per launch of the profiled kernel from its committed ncu
     summary, if it was taken on the current source."""
     if not path.exists():
@@ -640,6 +644,9 @@ def run_gpu(args, spec):
            "layers": s["layers"], "vocab": s["vocab"], "residual": 128, "group": 32,
            "dgap_K": DGAP_K, "dgap_hidden": DGAP_HIDDEN, "tau": round(st.dgap.tau, 6),
            "n_splits": st.n_splits,
+           "plan": ("flat: every pair's blocks and window chunks cut into equal per-warp "
+                    "ranges over one CTA per SM" if st.n_splits == 0 else
+                    f"split: {st.n_splits} CTAs per (sequence, kv-head)"),
            "kv_layout": (f"paged: block table over a shuffled pool of {st.paged_pages} page sets "
                          f"per layer" if st.paged_pages else "contiguous pages per sequence"),
            "l2": f"inputs larger than L2: {step_bytes[0] / 1e6:.0f} MB of packed KV read per "

@@ -71,7 +71,7 @@ def test_prefill_and_attention_match_contiguous(kvq_lib, bk, bv, gq):
     assert p.flags() == 0
     _same_state(a, p, lengths)
     q = synth.queries(401, cfg.batch, cfg.n_q_heads).cuda()
-    for ns in (1, 3, 11):
+    for ns in (1, 3, 11, 0):  # split plan counts, then the flat plan
         oa = kvq.kvq_decode_attn(a, q, n_splits=ns, out_dtype=torch.float32)
         op = kvq.kvq_decode_attn(p, q, n_splits=ns, out_dtype=torch.float32)
         torch.cuda.synchronize()
@@ -86,8 +86,9 @@ def test_prefill_and_attention_match_contiguous(kvq_lib, bk, bv, gq):
     assert p.flags() == 0
 
 
-@pytest.mark.parametrize("bk,bv,gq", [(1, 1, 4), (1, 1, 5), (2, 4, 4)])
-def test_decode_steps_flush_into_assigned_pages(kvq_lib, bk, bv, gq):
+@pytest.mark.parametrize("bk,bv,gq,ns", [(1, 1, 4, 4), (1, 1, 5, 4), (2, 4, 4, 4), (1, 1, 5, 0),
+                                         (2, 4, 4, 0)])
+def test_decode_steps_flush_into_assigned_pages(kvq_lib, bk, bv, gq, ns):
     # lengths that cross the flush point (L + 1 - 128 a multiple of 32)
     # within a few steps; pages for the flushed groups are assigned by the
     # caller just before the step that writes them
@@ -98,8 +99,8 @@ def test_decode_steps_flush_into_assigned_pages(kvq_lib, bk, bv, gq):
     hist = [(k.clone(), v.clone()) for k, v in kv]
     lens = list(lengths)
     g = synth.generator(411)
-    ws_a = kvq.attn_workspace(cfg, 4)
-    ws_p = kvq.attn_workspace(cfg, 4)
+    ws_a = kvq.attn_workspace(cfg, ns)  # ns = 0: the flat plan
+    ws_p = kvq.attn_workspace(cfg, ns)
     flushed = 0
     for step in range(40):
         for b, L in enumerate(lens):
@@ -110,9 +111,9 @@ def test_decode_steps_flush_into_assigned_pages(kvq_lib, bk, bv, gq):
         kn = torch.randn(cfg.batch, 2, 128, generator=g).half()
         vn = torch.randn(cfg.batch, 2, 128, generator=g).half()
         q = torch.randn(cfg.batch, cfg.n_q_heads, 128, generator=g).half()
-        oa = kvq.kvq_decode_step(a, kn.cuda(), vn.cuda(), q.cuda(), n_splits=4, workspace=ws_a,
+        oa = kvq.kvq_decode_step(a, kn.cuda(), vn.cuda(), q.cuda(), n_splits=ns, workspace=ws_a,
                                  out_dtype=torch.float32)
-        op = kvq.kvq_decode_step(p, kn.cuda(), vn.cuda(), q.cuda(), n_splits=4, workspace=ws_p,
+        op = kvq.kvq_decode_step(p, kn.cuda(), vn.cuda(), q.cuda(), n_splits=ns, workspace=ws_p,
                                  out_dtype=torch.float32)
         torch.cuda.synchronize()
         assert torch.equal(oa.view(torch.int32), op.view(torch.int32)), f"step {step}"
