@@ -61,62 +61,178 @@ __host__ __device__ inline int vmeta_index(int g, int t) {
 //   code  = clamp(rint(RN32(RN32(x - zero) / scale)), 0, levels); 0 if scale == 0
 // Codes fill B little-endian words, element i at bits [(i*B) % 32, +B) of
 // word (i*B) / 32.  Used by kvq_pack and by the decode step's flush.
+//
+// The codes come from q = RN32(d * RN32(1 / s)), d = RN32(x - zero): q and
+// RN32(d / s) both lie within 3 * 2^-24 * (d / s) <= 4.6e-5 of d / s (d / s
+// <= levels <= 255), so they round to the same integer unless q lies within
+// 4.6e-5 of a half-integer.  The rounding itself is one addition: q + 1536.5
+// lies in [1536.5, 1792.5), where float32 numbers are 2^-13 apart, so the
+// bits of y = RN32(q + 1536.5) are kCodeBias + floor(q' + 0.5) from bit 13
+// up and the fraction of q' + 0.5 below, q' being q on the 2^-13 grid.  A q
+// within 4.6e-5 (< half a grid step) of a half-integer puts y on an integer,
+// with its 13 low bits zero; so does a NaN.  A group with any such element
+// is redone by the definition's steps (the exact quotient per element);
+// every other element's code is floor(q' + 0.5) = rint(q) = rint(RN32(d / s)),
+// which lies in [0, levels] (0 <= q <= levels * (1 + 2^-23)).  A zero scale
+// takes r = 0, so q = 0 and every code is 0.
+constexpr float kCodeMagic = 1536.5f;
+constexpr uint32_t kCodeBias = 0x22600u;  // bits of 1536.5 >> 13, plus 512
+
+// Sum of kCodeBias at each code position of a word: a word accumulates
+// (y >> 13) << pos = (kCodeBias + code) << pos over its 32 / B codes.
+template <int B>
+__host__ __device__ constexpr uint32_t code_bias_word() {
+  uint32_t c = 0u;
+  for (int k = 0; k < 32 / B; ++k) c += kCodeBias << (k * B);
+  return c;
+}
+
+// Codes and scale of one group from d(i) = RN32(x_i - lo) and the group's
+// min lo and max hi.
+template <int B, typename D>
+__device__ __forceinline__ void quantize_codes(D d, float lo, float hi, uint32_t (&w)[B],
+                                               __half& scale) {
+  constexpr float kLevels = float((1 << B) - 1);
+  const __half s_h = __float2half_ru(__fdiv_ru(__fsub_ru(hi, lo), kLevels));
+  const float s = __half2float(s_h);
+  const float r = s > 0.0f ? __frcp_rn(s) : 0.0f;
+  uint32_t acc[B];
+#pragma unroll
+  for (int j = 0; j < B; ++j) acc[j] = 0u;
+  uint32_t low = 0x1fffu;  // least 13-bit fraction field seen
+#pragma unroll
+  for (int i = 0; i < kGroup; ++i) {
+    const float q = __fmul_rn(d(i), r);
+    const uint32_t y = __float_as_uint(__fadd_rn(q, kCodeMagic));
+    low = min(low, y & 0x1fffu);
+    if constexpr (B == 1) {
+      acc[0] |= ((y >> 13) & 1u) << i;  // kCodeBias is even
+    } else {
+      acc[(i * B) / 32] += (y >> 13) << ((i * B) % 32);
+    }
+  }
+  if constexpr (B > 1) {
+#pragma unroll
+    for (int j = 0; j < B; ++j) acc[j] -= code_bias_word<B>();
+  }
+  if (low == 0u) {  // near a tie (or not finite): the definition's steps
+#pragma unroll
+    for (int j = 0; j < B; ++j) acc[j] = 0u;
+#pragma unroll
+    for (int i = 0; i < kGroup; ++i) {
+      uint32_t c = 0u;
+      if (s > 0.0f) {
+        const float t = fminf(fmaxf(rintf(__fdiv_rn(d(i), s)), 0.0f), kLevels);
+        c = (uint32_t)t;
+      }
+      acc[(i * B) / 32] |= c << ((i * B) % 32);
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < B; ++j) w[j] = acc[j];
+  scale = s_h;
+}
+
 template <int B>
 __device__ __forceinline__ void quantize_group(const float (&x)[kGroup], uint32_t (&w)[B],
                                                __half& scale, __half& zero) {
-  constexpr float kLevels = float((1 << B) - 1);
   float lo = x[0], hi = x[0];
 #pragma unroll
   for (int i = 1; i < kGroup; ++i) {
     lo = fminf(lo, x[i]);
     hi = fmaxf(hi, x[i]);
   }
-  const __half s_h = __float2half_ru(__fdiv_ru(__fsub_ru(hi, lo), kLevels));
-  const float s = __half2float(s_h);
-  // The quotient d / s (d = RN32(x - zero) <= levels * s, so d / s <= 255)
-  // comes from one product with RN32(1 / s): the product and RN32(d / s) both
-  // lie within 3 * 2^-24 * (d / s) <= 4.6e-5 of d / s, so they round to the
-  // same integer unless the product is within 1/8192 of a half-integer, where
-  // the exact quotient is taken.  The codes are those of the definition.
-  const float r = s > 0.0f ? __frcp_rn(s) : 0.0f;
-#pragma unroll
-  for (int j = 0; j < B; ++j) w[j] = 0u;
-#pragma unroll
-  for (int i = 0; i < kGroup; ++i) {
-    uint32_t c = 0u;
-    if (s > 0.0f) {
-      const float dd = __fsub_rn(x[i], lo);
-      const float q = __fmul_rn(dd, r);
-      float t = rintf(q);
-      if (fabsf(fabsf(q - t) - 0.5f) < 1.0f / 8192.0f) t = rintf(__fdiv_rn(dd, s));
-      t = fminf(fmaxf(t, 0.0f), kLevels);
-      c = (uint32_t)t;
-    }
-    w[(i * B) / 32] |= c << ((i * B) % 32);
-  }
-  scale = s_h;
+  quantize_codes<B>([&](int i) { return __fsub_rn(x[i], lo); }, lo, hi, w, scale);
   zero = __float2half_rn(lo);  // lo is an fp16 value: exact
+}
+
+// Min and max of 32 fp16 numbers held as 16 pairs (exact in fp16).
+__device__ __forceinline__ void group_range(const __half2 (&x)[kGroup / 2], float& lo, float& hi) {
+  __half2 l = x[0], h = x[0];
+#pragma unroll
+  for (int p = 1; p < kGroup / 2; ++p) {
+    l = __hmin2(l, x[p]);
+    h = __hmax2(h, x[p]);
+  }
+  lo = fminf(__low2float(l), __high2float(l));
+  hi = fmaxf(__low2float(h), __high2float(h));
+}
+
+// RN32(a - c) for an fp16 a (one half of a pair) and a float32 c: one
+// mixed-precision subtraction (a is widened exactly, the difference rounded
+// once).
+template <int kHigh>
+__device__ __forceinline__ float sub_half(__half2 pair, float c) {
+  float d;
+  if constexpr (kHigh)
+    asm("{.reg .b16 l, h; mov.b32 {l, h}, %1; sub.rn.f32.f16 %0, h, %2;}"
+        : "=f"(d) : "r"(*reinterpret_cast<const uint32_t*>(&pair)), "f"(c));
+  else
+    asm("{.reg .b16 l, h; mov.b32 {l, h}, %1; sub.rn.f32.f16 %0, l, %2;}"
+        : "=f"(d) : "r"(*reinterpret_cast<const uint32_t*>(&pair)), "f"(c));
+  return d;
+}
+
+// Codes and scale of the group held as 16 pairs (element i = half i & 1 of
+// pair i >> 1); lo is the group's min (its zero).
+template <int B>
+__device__ __forceinline__ void quantize_pairs(const __half2 (&x)[kGroup / 2], uint32_t (&w)[B],
+                                               __half& scale, float& lo) {
+  float hi;
+  group_range(x, lo, hi);
+  const float z = lo;
+  quantize_codes<B>(
+      [&](int i) { return (i & 1) ? sub_half<1>(x[i >> 1], z) : sub_half<0>(x[i >> 1], z); }, lo,
+      hi, w, scale);
+}
+
+__host__ __device__ constexpr uint32_t rotl_const(uint32_t v, int p) {
+  return p == 0 ? v : (v << p) | (v >> (32 - p));
+}
+
+// One lane's word of 1-bit codes in fragment order, from the code rows
+// (bit i = element i) of eight source lanes: from source k, the nibble at
+// bit 4 gid goes to bits p_k .. p_k + 3 (mod 32).
+template <typename Src, typename Pos>
+__device__ __forceinline__ uint32_t gather_nibbles(uint32_t row, int gid, Src src, Pos pos) {
+  uint32_t word = 0u;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const uint32_t v = __shfl_sync(0xffffffffu, row, src(k));
+    const int p = pos(k) & 31;
+    word |= __funnelshift_r(v, v, (4 * gid - p) & 31) & rotl_const(0xfu, p);
+  }
+  return word;
 }
 
 // One quarter qi of a 32-token block, quantized by one warp into a page (or
 // a page image): key groups of channels 32 qi .. 32 qi + 31 (lane = channel)
 // and value group qi of the 32 tokens (lane = token).  row_k(t), row_v(t)
 // give the fp16 rows [128] of token t of the block.  The quarters write
-// disjoint words, scales and zeros (1-bit codes: words 4 l + qi, l = 0..31,
-// assembled from warp ballots in the order key1_bit / val1_bit give), so the
-// four may run in different warps.  Used by kvq_pack and by the decode
-// step's flush, which are therefore bit-identical.
+// disjoint words, scales and zeros, so the four may run in different warps.
+// Codes of b >= 2 bits: key channel c and value (group qi, token lane) both
+// take words (32 qi + lane) * b .. + b - 1 of their code areas.  1-bit
+// codes: lane l = 4 gid + tig writes word 4 l + qi, gathered with shuffles
+// in the order key1_bit / val1_bit give: keys take tokens 4 gid + j
+// (j = 0..3) of channels 16 ks1 + 4 tig + 2 h + e at bit 10 + 16 e + j -
+// 4 (2 ks1 + h); values take channels 4 gid + j of tokens 8 tig + 4 e + r
+// at bit 10 + 16 e + j - 4 r.  With equal key and value widths one code
+// body quantizes both groups in turn (half the instructions to fetch).
+// Used by kvq_pack and by the decode step's flush, which are therefore
+// bit-identical.
 template <int BK, int BV, typename RowK, typename RowV>
 __device__ __forceinline__ void quantize_quarter(RowK row_k, RowV row_v, int qi, char* image) {
   const int lane = threadIdx.x & 31;
+  const int gid = lane >> 2, tig = lane & 3;
   uint32_t* kcodes = reinterpret_cast<uint32_t*>(image);
   uint32_t* vcodes = reinterpret_cast<uint32_t*>(image + page_off_vcodes(BK));
   __half* kmeta = reinterpret_cast<__half*>(image + page_off_kmeta(BK));
   __half* vmeta = reinterpret_cast<__half*>(image + page_off_vmeta(BK, BV));
   const int c = kGroup * qi + lane;  // this lane's key channel
-  float xk[kGroup], xv[kGroup];
+  const int vm = vmeta_index(qi, lane);
+  __half2 xk[kGroup / 2], xv[kGroup / 2];  // tokens 2p, 2p + 1 / channels 2p, 2p + 1
 #pragma unroll
-  for (int t = 0; t < kGroup; ++t) xk[t] = __half2float(row_k(t)[c]);
+  for (int p = 0; p < kGroup / 2; ++p) xk[p] = __halves2half2(row_k(2 * p)[c], row_k(2 * p + 1)[c]);
   {
     const uint4* row = reinterpret_cast<const uint4*>(row_v(lane) + kGroup * qi);
 #pragma unroll
@@ -124,70 +240,60 @@ __device__ __forceinline__ void quantize_quarter(RowK row_k, RowV row_v, int qi,
       const uint4 u = row[k];
       const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&wd[e]));
-        xv[8 * k + 2 * e] = f.x;
-        xv[8 * k + 2 * e + 1] = f.y;
+      for (int e = 0; e < 4; ++e) xv[4 * k + e] = *reinterpret_cast<const __half2*>(&wd[e]);
+    }
+  }
+  uint32_t rk = 0u, rv = 0u;  // 1-bit code rows
+  if constexpr (BK == BV) {
+#pragma unroll 1
+    for (int pass = 0; pass < 2; ++pass) {  // keys from xk, then values moved there
+      uint32_t w[BK];
+      __half s;
+      float lo;
+      quantize_pairs<BK>(xk, w, s, lo);
+      __half* meta = pass ? vmeta : kmeta;
+      const int mi = pass ? vm : c;
+      meta[mi] = s;
+      meta[kHeadDim + mi] = __float2half_rn(lo);  // an fp16 value: exact
+      if constexpr (BK == 1) {
+        if (pass) rv = w[0]; else rk = w[0];
+      } else {
+        uint32_t* codes = (pass ? vcodes : kcodes) + c * BK;
+#pragma unroll
+        for (int j = 0; j < BK; ++j) codes[j] = w[j];
       }
+#pragma unroll
+      for (int p = 0; p < kGroup / 2; ++p) xk[p] = xv[p];
     }
-  }
-  uint32_t wk[BK], wv[BV];
-  __half sk, zk, sv, zv;
-  quantize_group<BK>(xk, wk, sk, zk);
-  quantize_group<BV>(xv, wv, sv, zv);
-  kmeta[c] = sk;
-  kmeta[kHeadDim + c] = zk;
-  vmeta[vmeta_index(qi, lane)] = sv;
-  vmeta[kHeadDim + vmeta_index(qi, lane)] = zv;
-  // 1-bit codes: lane l = 4 gid + tig assembles word 4 l + qi from ballots
-  // (bit positions of key1_bit / val1_bit)
-  const int gid = lane >> 2, tig = lane & 3;
-  if constexpr (BK == 1) {
-    uint32_t mine[4] = {0u, 0u, 0u, 0u};  // ballots of tokens 4 gid + j over channels
-#pragma unroll
-    for (int t = 0; t < kGroup; ++t) {
-      const uint32_t bt = __ballot_sync(0xffffffffu, (wk[0] >> t) & 1u);
-      if ((t >> 2) == gid) mine[t & 3] = bt;
-    }
-    uint32_t word = 0u;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t m = mine[j] >> (4 * tig);
-#pragma unroll
-      for (int ks1 = 0; ks1 < 2; ++ks1)
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int e = 0; e < 2; ++e)
-            word |= ((m >> (16 * ks1 + 2 * h + e)) & 1u) << ((10 + 16 * e + j - 4 * (2 * ks1 + h)) & 31);
-    }
-    kcodes[4 * lane + qi] = word;
   } else {
+    uint32_t wk[BK], wv[BV];
+    __half sk, sv;
+    float lok, lov;
+    quantize_pairs<BK>(xk, wk, sk, lok);
+    quantize_pairs<BV>(xv, wv, sv, lov);
+    kmeta[c] = sk;
+    kmeta[kHeadDim + c] = __float2half_rn(lok);
+    vmeta[vm] = sv;
+    vmeta[kHeadDim + vm] = __float2half_rn(lov);
+    if constexpr (BK == 1) rk = wk[0];
+    else {
 #pragma unroll
-    for (int j = 0; j < BK; ++j) kcodes[c * BK + j] = wk[j];
-  }
-  if constexpr (BV == 1) {
-    uint32_t mine[4] = {0u, 0u, 0u, 0u};  // ballots of channels 4 gid + j over tokens
-#pragma unroll
-    for (int ci = 0; ci < kGroup; ++ci) {
-      const uint32_t bc = __ballot_sync(0xffffffffu, (wv[0] >> ci) & 1u);
-      if ((ci >> 2) == gid) mine[ci & 3] = bc;
+      for (int j = 0; j < BK; ++j) kcodes[c * BK + j] = wk[j];
     }
-    uint32_t word = 0u;
+    if constexpr (BV == 1) rv = wv[0];
+    else {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t m = mine[j] >> (8 * tig);
-#pragma unroll
-      for (int e = 0; e < 2; ++e)
-#pragma unroll
-        for (int r = 0; r < 4; ++r)
-          word |= ((m >> (4 * e + r)) & 1u) << ((10 + 16 * e + j - 4 * r) & 31);
+      for (int j = 0; j < BV; ++j) vcodes[c * BV + j] = wv[j];
     }
-    vcodes[4 * lane + qi] = word;
-  } else {
-#pragma unroll
-    for (int j = 0; j < BV; ++j) vcodes[(qi * kGroup + lane) * BV + j] = wv[j];
   }
+  if constexpr (BK == 1)
+    kcodes[4 * lane + qi] = gather_nibbles(
+        rk, gid, [&](int k) { return 16 * (k >> 2) + 2 * ((k >> 1) & 1) + (k & 1) + 4 * tig; },
+        [](int k) { return 10 + 16 * (k & 1) - 8 * (k >> 2) - 4 * ((k >> 1) & 1); });
+  if constexpr (BV == 1)
+    vcodes[4 * lane + qi] = gather_nibbles(
+        rv, gid, [&](int k) { return 8 * tig + 4 * (k >> 2) + (k & 3); },
+        [](int k) { return 10 + 16 * (k >> 2) - 4 * (k & 3); });
 }
 
 
