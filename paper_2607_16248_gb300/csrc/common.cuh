@@ -62,19 +62,19 @@ __host__ __device__ inline int vmeta_index(int g, int t) {
 // Codes fill B little-endian words, element i at bits [(i*B) % 32, +B) of
 // word (i*B) / 32.  Used by kvq_pack and by the decode step's flush.
 //
-// The codes come from q = RN32(d * RN32(1 / s)), d = RN32(x - zero): q and
-// RN32(d / s) both lie within 3 * 2^-24 * (d / s) <= 4.6e-5 of d / s (d / s
-// <= levels <= 255), so they round to the same integer unless q lies within
-// 4.6e-5 of a half-integer.  The rounding itself is one addition: q + 1536.5
+// The codes come from one fused multiply-add, y = RN32(d * r + 1536.5) with
+// d = RN32(x - zero) and r = RN32(1 / s): the exact d * r lies within
+// 2^-24 * (d / s) of d / s, and so does RN32(d / s), so (d / s <= levels <=
+// 255) d * r is within 3.1e-5 of RN32(d / s), and both round to the same
+// integer unless d * r lies within 3.1e-5 of a half-integer.  d * r + 1536.5
 // lies in [1536.5, 1792.5), where float32 numbers are 2^-13 apart, so the
-// bits of y = RN32(q + 1536.5) are kCodeBias + floor(q' + 0.5) from bit 13
-// up and the fraction of q' + 0.5 below, q' being q on the 2^-13 grid.  A q
-// within 4.6e-5 (< half a grid step) of a half-integer puts y on an integer,
-// with its 13 low bits zero; so does a NaN.  A group with any such element
-// is redone by the definition's steps (the exact quotient per element);
-// every other element's code is floor(q' + 0.5) = rint(q) = rint(RN32(d / s)),
-// which lies in [0, levels] (0 <= q <= levels * (1 + 2^-23)).  A zero scale
-// takes r = 0, so q = 0 and every code is 0.
+// bits of y are kCodeBias + floor(q + 0.5) from bit 13 up and the fraction
+// of q + 0.5 below, q being d * r on the 2^-13 grid.  A d * r within half a
+// grid step (6.1e-5) of a half-integer puts y on an integer, with its 13 low
+// bits zero; so does a NaN.  A group with any such element is redone by the
+// definition's steps (the exact quotient per element); every other
+// element's code is floor(q + 0.5) = rint(RN32(d / s)), which lies in
+// [0, levels].  A zero scale takes r = 0, so every code is 0.
 constexpr float kCodeMagic = 1536.5f;
 constexpr uint32_t kCodeBias = 0x22600u;  // bits of 1536.5 >> 13, plus 512
 
@@ -87,13 +87,35 @@ __host__ __device__ constexpr uint32_t code_bias_word() {
   return c;
 }
 
+// RU32(x / L) for a float32 x >= 0 (or +inf) and L = levels: the product
+// with RN32(1 / L) lies within two ulps of x / L, and the sign of the exact
+// q * L - x (one fused multiply-add) moves it up, then down, to the least
+// float32 >= x / L.  L = 1 is exact.
+template <int L>
+__device__ __forceinline__ float div_ru_levels(float x) {
+  if constexpr (L == 1) {
+    return x;
+  } else {
+    float q = __fmul_rn(x, 1.0f / L);
+#pragma unroll
+    for (int k = 0; k < 2; ++k)
+      if (__fmaf_rn(q, float(L), -x) < 0.0f) q = __uint_as_float(__float_as_uint(q) + 1u);
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const float p = __uint_as_float(__float_as_uint(q) - 1u);
+      if (q > 0.0f && __fmaf_rn(p, float(L), -x) >= 0.0f) q = p;
+    }
+    return q;
+  }
+}
+
 // Codes and scale of one group from d(i) = RN32(x_i - lo) and the group's
 // min lo and max hi.
 template <int B, typename D>
 __device__ __forceinline__ void quantize_codes(D d, float lo, float hi, uint32_t (&w)[B],
                                                __half& scale) {
   constexpr float kLevels = float((1 << B) - 1);
-  const __half s_h = __float2half_ru(__fdiv_ru(__fsub_ru(hi, lo), kLevels));
+  const __half s_h = __float2half_ru(div_ru_levels<(1 << B) - 1>(__fsub_ru(hi, lo)));
   const float s = __half2float(s_h);
   const float r = s > 0.0f ? __frcp_rn(s) : 0.0f;
   uint32_t acc[B];
@@ -102,8 +124,7 @@ __device__ __forceinline__ void quantize_codes(D d, float lo, float hi, uint32_t
   uint32_t low = 0x1fffu;  // least 13-bit fraction field seen
 #pragma unroll
   for (int i = 0; i < kGroup; ++i) {
-    const float q = __fmul_rn(d(i), r);
-    const uint32_t y = __float_as_uint(__fadd_rn(q, kCodeMagic));
+    const uint32_t y = __float_as_uint(__fmaf_rn(d(i), r, kCodeMagic));
     low = min(low, y & 0x1fffu);
     if constexpr (B == 1) {
       acc[0] |= ((y >> 13) & 1u) << i;  // kCodeBias is even
