@@ -71,9 +71,9 @@ __host__ __device__ inline int vmeta_index(int g, int t) {
 // bits of y are kCodeBias + floor(q + 0.5) from bit 13 up and the fraction
 // of q + 0.5 below, q being d * r on the 2^-13 grid.  A d * r within half a
 // grid step (6.1e-5) of a half-integer puts y on an integer, with its 13 low
-// bits zero; so does a NaN.  A group with any such element is redone by the
-// definition's steps (the exact quotient per element); every other
-// element's code is floor(q + 0.5) = rint(RN32(d / s)), which lies in
+// bits zero; so does a NaN.  Such an element's code is taken by the
+// definition's steps (the exact quotient) and swapped into its word; every
+// other element's code is floor(q + 0.5) = rint(RN32(d / s)), which lies in
 // [0, levels].  A zero scale takes r = 0, so every code is 0.
 constexpr float kCodeMagic = 1536.5f;
 constexpr uint32_t kCodeBias = 0x22600u;  // bits of 1536.5 >> 13, plus 512
@@ -110,9 +110,11 @@ __device__ __forceinline__ float div_ru_levels(float x) {
 }
 
 // Codes and scale of one group from d(i) = RN32(x_i - lo) and the group's
-// min lo and max hi.
-template <int B, typename D>
-__device__ __forceinline__ void quantize_codes(D d, float lo, float hi, uint32_t (&w)[B],
+// min lo and max hi.  d2 computes the same values by other instructions, for
+// the rare elements near a tie: recomputing them there keeps the compiler
+// from holding every element's d and y in registers until then.
+template <int B, typename D, typename D2>
+__device__ __forceinline__ void quantize_codes(D d, D2 d2, float lo, float hi, uint32_t (&w)[B],
                                                __half& scale) {
   constexpr float kLevels = float((1 << B) - 1);
   const __half s_h = __float2half_ru(div_ru_levels<(1 << B) - 1>(__fsub_ru(hi, lo)));
@@ -136,17 +138,20 @@ __device__ __forceinline__ void quantize_codes(D d, float lo, float hi, uint32_t
 #pragma unroll
     for (int j = 0; j < B; ++j) acc[j] -= code_bias_word<B>();
   }
-  if (low == 0u) {  // near a tie (or not finite): the definition's steps
-#pragma unroll
-    for (int j = 0; j < B; ++j) acc[j] = 0u;
+  if (low == 0u) {  // near a tie (or not finite): those elements by the definition's steps
 #pragma unroll
     for (int i = 0; i < kGroup; ++i) {
-      uint32_t c = 0u;
-      if (s > 0.0f) {
-        const float t = fminf(fmaxf(rintf(__fdiv_rn(d(i), s)), 0.0f), kLevels);
-        c = (uint32_t)t;
+      const float di = d2(i);
+      const uint32_t y = __float_as_uint(__fmaf_rn(di, r, kCodeMagic));
+      if ((y & 0x1fffu) == 0u) {
+        uint32_t c = 0u;
+        if (s > 0.0f) c = (uint32_t)fminf(fmaxf(rintf(__fdiv_rn(di, s)), 0.0f), kLevels);
+        if constexpr (B == 1) {
+          acc[0] = (acc[0] & ~(1u << i)) | (c << i);
+        } else {  // the word is a sum of its fields: swap this one's (mod 2^32)
+          acc[(i * B) / 32] += (c + kCodeBias - (y >> 13)) << ((i * B) % 32);
+        }
       }
-      acc[(i * B) / 32] |= c << ((i * B) % 32);
     }
   }
 #pragma unroll
@@ -163,7 +168,8 @@ __device__ __forceinline__ void quantize_group(const float (&x)[kGroup], uint32_
     lo = fminf(lo, x[i]);
     hi = fmaxf(hi, x[i]);
   }
-  quantize_codes<B>([&](int i) { return __fsub_rn(x[i], lo); }, lo, hi, w, scale);
+  const auto d = [&](int i) { return __fsub_rn(x[i], lo); };
+  quantize_codes<B>(d, d, lo, hi, w, scale);
   zero = __float2half_rn(lo);  // lo is an fp16 value: exact
 }
 
@@ -203,8 +209,11 @@ __device__ __forceinline__ void quantize_pairs(const __half2 (&x)[kGroup / 2], u
   group_range(x, lo, hi);
   const float z = lo;
   quantize_codes<B>(
-      [&](int i) { return (i & 1) ? sub_half<1>(x[i >> 1], z) : sub_half<0>(x[i >> 1], z); }, lo,
-      hi, w, scale);
+      [&](int i) { return (i & 1) ? sub_half<1>(x[i >> 1], z) : sub_half<0>(x[i >> 1], z); },
+      [&](int i) {
+        return __fsub_rn((i & 1) ? __high2float(x[i >> 1]) : __low2float(x[i >> 1]), z);
+      },
+      lo, hi, w, scale);
 }
 
 __host__ __device__ constexpr uint32_t rotl_const(uint32_t v, int p) {
