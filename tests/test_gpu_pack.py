@@ -167,3 +167,63 @@ def test_tie_where_a_reciprocal_product_misrounds(kvq_lib):
     want = quant.quantize_head(k[0].numpy(), v[0].numpy(), 2, 2, 128)
     assert np.all(want["k_scale"].astype(np.float64) == 0.2216796875)
     _util.assert_head_equal(got, want)
+
+
+def _one_tie_per_group(rng, L, bits):
+    """[L, 128] fp16 keys and values whose every quantization group (keys: 32
+    tokens of a channel; values: 32 channels of a token) holds its min -1,
+    its max -1 + levels * 0.1875 (so the scale is 0.1875, not a power of two),
+    one exact tie -1 + (m + 0.5) * 0.1875 and 29 uniform values in between,
+    at random places."""
+    levels = (1 << bits) - 1
+    lo, s = -1.0, 0.1875
+
+    def groups(n):
+        g = rng.uniform(lo, lo + levels * s, (n, 32))
+        pos = np.argsort(rng.random((n, 32)), axis=1)[:, :3]
+        r = np.arange(n)
+        g[r, pos[:, 0]] = lo
+        g[r, pos[:, 1]] = lo + levels * s
+        g[r, pos[:, 2]] = lo + (rng.integers(0, levels, n) + 0.5) * s
+        return g.astype(np.float16)
+
+    nb = L // 32
+    k = groups(nb * 128).reshape(nb, 128, 32).transpose(0, 2, 1).reshape(L, 128)
+    v = groups(L * 4).reshape(L, 128)
+    return torch.from_numpy(np.ascontiguousarray(k)), torch.from_numpy(v)
+
+
+@pytest.mark.parametrize("bits", [1, 2, 4, 8])
+def test_one_tie_among_random_values_per_group(kvq_lib, bits):
+    # The tie's code comes from the exact quotient while the other 31 codes
+    # of its words come from the fused rounding: the tie's field is replaced
+    # in place, through kvq_pack and through the decode step's flush.
+    rng = np.random.default_rng(500 + bits)
+    L, L0 = 320, 150
+    cfg = kvq.CacheConfig(batch=2, n_q_heads=8, n_kv_heads=2, bits_k=bits, bits_v=bits,
+                          max_len=512)
+    kv = [[_one_tie_per_group(rng, L, bits) for _ in range(2)] for _ in range(2)]
+    k_all = [torch.stack([kv[b][h][0] for h in range(2)]) for b in range(2)]  # [Hkv, L, 128]
+    v_all = [torch.stack([kv[b][h][1] for h in range(2)]) for b in range(2)]
+    packed = kvq.QuantKVCache(cfg)
+    stepped = kvq.QuantKVCache(cfg)
+    for b in range(2):
+        kvq.kvq_pack(packed, k_all[b][None].cuda(), v_all[b][None].cuda(), batch_begin=b)
+        kvq.kvq_pack(stepped, k_all[b][None, :, :L0].cuda(), v_all[b][None, :, :L0].cuda(),
+                     batch_begin=b)
+    q = torch.zeros(2, 8, 128, dtype=torch.float16, device="cuda")
+    for t in range(L0, L):  # flushes at 160, 192, ..., 288
+        kn = torch.stack([k_all[b][:, t] for b in range(2)]).cuda()
+        vn = torch.stack([v_all[b][:, t] for b in range(2)]).cuda()
+        kvq.kvq_decode_step(stepped, kn, vn, q)
+    torch.cuda.synchronize()
+    assert packed.seq_lens().cpu().tolist() == [L, L]
+    assert stepped.seq_lens().cpu().tolist() == [L, L]
+    for b in range(2):
+        for h in range(2):
+            want = quant.quantize_head(k_all[b][h].numpy(), v_all[b][h].numpy(), bits, bits,
+                                       cfg.residual)
+            assert np.all(want["k_scale"].astype(np.float64) == 0.1875)
+            assert np.all(want["v_scale"].astype(np.float64) == 0.1875)
+            _util.assert_head_equal(_util.head_arrays(packed, b, h, L), want)
+            _util.assert_head_equal(_util.head_arrays(stepped, b, h, L), want)
