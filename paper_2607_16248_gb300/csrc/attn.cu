@@ -122,11 +122,16 @@ struct MergeGroups {
 // ---------------------------------------------------------------------------
 
 // Cost weights: a window chunk costs cw units, the first item of a pair sc
-// more (measured: a chunk takes ~4 blocks' time, a pair start ~1).  A launch
-// with too little work for every warp to hold an item under those weights
-// takes lighter ones (FlatGrid::cw, sc), down to one unit per item.
+// more (measured: a chunk takes ~4 blocks' time, a pair start ~1), and the
+// block that leaves the window in a decode step fu more (its warp quantizes
+// the block alone; Mistral-7B shape, K2V2, ragged batch of 16 where some
+// sequence flushes on most steps: 0, 4, 8 and 12 units gave 4.30, 4.24,
+// 4.19 and 4.18 ms mean and 4.70, 4.54, 4.40 and 4.37 ms p95 per 32-layer
+// step).  A launch with too little work
+// for every warp to hold an item under those weights takes lighter ones
+// (FlatGrid::k), down to one unit per item.
 struct Costs {
-  int cw, sc;
+  int cw, sc, fu;
 };
 
 struct PairShape {
@@ -139,21 +144,32 @@ __host__ __device__ inline PairShape pair_shape(int L, int residual) {
   s.nr = (L - s.Lq + kGroup - 1) / kGroup;
   return s;
 }
-__host__ __device__ inline int pair_cost(const PairShape& s, Costs k) {
-  return s.nb + s.nr > 0 ? k.sc + s.nb + k.cw * s.nr : 0;
+// Extra units f of a pair whose last packed block leaves the window in this
+// launch (a decode step that appends a token: L = L0 + 1).
+__host__ __device__ inline int flush_units(int L0, int L, int residual, Costs k) {
+  return L > L0 && packed_len(L, residual) > packed_len(L0, residual) ? k.fu : 0;
 }
-// First unit (pair-local) of item i.
-__host__ __device__ inline int item_unit(int i, int nb, Costs k) {
-  return i == 0 ? 0 : k.sc + (i < nb ? i : nb + k.cw * (i - nb));
+__host__ __device__ inline int pair_cost(const PairShape& s, Costs k, int f) {
+  return s.nb + s.nr > 0 ? k.sc + s.nb + f + k.cw * s.nr : 0;
+}
+// First unit (pair-local) of item i; the last packed block (nb - 1) costs
+// 1 + f units.
+__host__ __device__ inline int item_unit(int i, int nb, Costs k, int f) {
+  return i == 0 ? 0 : k.sc + (i < nb ? i : nb + f + k.cw * (i - nb));
+}
+// Largest cost of one item under the weights (a warp's range holds at least
+// this many units, so every warp holds an item start).
+__host__ __device__ inline int max_item_cost(Costs k) {
+  return k.cw + k.sc > 1 + k.fu + k.sc ? k.cw + k.sc : 1 + k.fu + k.sc;
 }
 // Number of items of a pair whose first unit (pair-local) is below x.
-__host__ __device__ inline int items_below(long long x, int nb, int nr, Costs k) {
+__host__ __device__ inline int items_below(long long x, int nb, int nr, Costs k, int f) {
   if (x <= 0 || nb + nr == 0) return 0;
   int c = 1;
   if (nb > 1) c += (int)min((long long)(nb - 1), max(0LL, x - k.sc - 1));
   const int lo_w = nb == 0 ? 1 : 0;
   if (nr > lo_w) {
-    const long long t = x - k.sc - nb;
+    const long long t = x - k.sc - nb - f;
     const int sh = k.cw == 4 ? 2 : k.cw == 2 ? 1 : 0;  // cw is 1, 2 or 4
     const long long n = t <= 0 ? 0 : (t + k.cw - 1) >> sh;
     c += (int)max(0LL, min(n, (long long)nr) - lo_w);
@@ -161,9 +177,10 @@ __host__ __device__ inline int items_below(long long x, int nb, int nr, Costs k)
   return c;
 }
 
-// Work totals of a launch: packed blocks, window chunks, non-empty pairs.
+// Work totals of a launch: packed blocks, window chunks, non-empty pairs,
+// pairs with a block leaving the window.
 struct WorkSums {
-  long long nb, nr, np;
+  long long nb, nr, np, nf;
 };
 
 // floor(x / d) from r = floor((2^64 - 1) / d): the high half of x * r is at
@@ -197,15 +214,15 @@ __host__ __device__ inline FlatGrid flat_grid(const WorkSums& w, int ctas) {
   const long long cap = (long long)kWarps * ctas;
   // the heaviest weights under which every one of the cap warps can still
   // hold an item start (each range >= the largest item cost)
-  const Costs pick[3] = {{4, 1}, {2, 1}, {1, 0}};
+  const Costs pick[3] = {{4, 1, 12}, {2, 1, 6}, {1, 0, 0}};
   int i = 0;
   for (; i < 2; ++i) {
-    const long long N = w.nb + pick[i].cw * w.nr + pick[i].sc * w.np;
-    if (N / (pick[i].cw + pick[i].sc) >= cap) break;
+    const long long N = w.nb + pick[i].cw * w.nr + pick[i].sc * w.np + pick[i].fu * w.nf;
+    if (N / max_item_cost(pick[i]) >= cap) break;
   }
   g.k = pick[i];
-  g.N = w.nb + g.k.cw * w.nr + g.k.sc * w.np;
-  const long long nv = g.N / (g.k.cw + g.k.sc);
+  g.N = w.nb + g.k.cw * w.nr + g.k.sc * w.np + g.k.fu * w.nf;
+  const long long nv = g.N / max_item_cost(g.k);
   g.n_v = g.N == 0 ? 0 : (int)(nv < 1 ? 1 : (nv < cap ? nv : cap));
   g.n_cta = g.n_v < ctas ? g.n_v : ctas;
   g.rN = rcp64((unsigned long long)g.N);
@@ -227,11 +244,11 @@ __host__ __device__ inline int cta_first_v(int c, const FlatGrid& g) {
 }
 // Partials of a non-empty pair (first unit U, cost C): the CTA partials of
 // CTAs [c_a, c_a + n_cta) and, if `cont`, one warp partial.
-__host__ __device__ inline int pair_partials(long long U, int C, int nb, int nr,
+__host__ __device__ inline int pair_partials(long long U, int C, int nb, int nr, int f,
                                              const FlatGrid& g, int& c_a, int& n_cta,
                                              bool& cont) {
   const int wf = unit_owner(U, g);
-  const int wl = unit_owner(U + item_unit(nb + nr - 1, nb, g.k), g);
+  const int wl = unit_owner(U + item_unit(nb + nr - 1, nb, g.k, f), g);
   cont = U + C < g.N && unit_owner(U + C, g) == wl;
   const int hv = wl - (cont ? 1 : 0);
   c_a = cta_of(wf, g);
@@ -251,18 +268,23 @@ __device__ __forceinline__ long long warp_sum_ll(long long v) {
 // Work totals of all pairs (lengths as the kernel attends them).
 __device__ WorkSums plan_sums(const int* seq_len, const Dims& d, bool append) {
   const int lane = threadIdx.x & 31;
-  long long nb = 0, nr = 0, np = 0;
+  long long nb = 0, nr = 0, np = 0, nf = 0;
+  const Costs one = {1, 0, 1};
   for (int b0 = 0; b0 < d.batch; b0 += 32) {
     const int b = b0 + lane;
-    const PairShape s = pair_shape(b < d.batch ? attended_len(read_len(seq_len + b), d, append) : 0, d.residual);
+    const int L0 = b < d.batch ? read_len(seq_len + b) : 0;
+    const int L = b < d.batch ? attended_len(L0, d, append) : 0;
+    const PairShape s = pair_shape(L, d.residual);
     nb += warp_sum_ll((long long)d.hkv * s.nb);
     nr += warp_sum_ll((long long)d.hkv * s.nr);
     np += warp_sum_ll(s.nb + s.nr > 0 ? d.hkv : 0);
+    nf += warp_sum_ll((long long)d.hkv * flush_units(L0, L, d.residual, one));
   }
   WorkSums w;
   w.nb = nb;
   w.nr = nr;
   w.np = np;
+  w.nf = nf;
   return w;
 }
 
@@ -271,13 +293,15 @@ struct Walk {
   int b, h;        // current sequence and kv-head
   long long Ub;    // first unit of sequence b
   int L0, L, pc;   // stored and attended length of b, cost of one of its pairs
+  int f;           // flush units of b's pairs
 };
 __device__ __forceinline__ void walk_load(Walk& w, const int* seq_len, const Dims& d,
                                           bool append, Costs k) {
   if (w.b < d.batch) {
     w.L0 = read_len(seq_len + w.b);
     w.L = attended_len(w.L0, d, append);
-    w.pc = pair_cost(pair_shape(w.L, d.residual), k);
+    w.f = flush_units(w.L0, w.L, d.residual, k);
+    w.pc = pair_cost(pair_shape(w.L, d.residual), k, w.f);
   }
 }
 // Position at the first pair whose units reach past a (an empty pair at or
@@ -290,7 +314,8 @@ __device__ Walk walk_start(long long a, const int* seq_len, const Dims& d, bool 
     const int b = b0 + lane;
     const int L0 = b < d.batch ? read_len(seq_len + b) : 0;
     const int L = attended_len(L0, d, append);
-    const int pc = b < d.batch ? pair_cost(pair_shape(L, d.residual), k) : 0;
+    const int f = flush_units(L0, L, d.residual, k);
+    const int pc = b < d.batch ? pair_cost(pair_shape(L, d.residual), k, f) : 0;
     const long long cst = (long long)d.hkv * pc;
     long long incl = cst;
 #pragma unroll
@@ -308,6 +333,7 @@ __device__ Walk walk_start(long long a, const int* seq_len, const Dims& d, bool 
       w.L0 = __shfl_sync(0xffffffffu, L0, l);
       w.L = __shfl_sync(0xffffffffu, L, l);
       w.pc = __shfl_sync(0xffffffffu, pc, l);
+      w.f = __shfl_sync(0xffffffffu, f, l);
       w.h = w.pc > 0 && a > w.Ub ? (int)((a - w.Ub) / w.pc) : 0;
       return w;
     }
@@ -316,7 +342,7 @@ __device__ Walk walk_start(long long a, const int* seq_len, const Dims& d, bool 
   w.b = d.batch;
   w.h = 0;
   w.Ub = base;
-  w.L0 = w.L = w.pc = 0;
+  w.L0 = w.L = w.pc = w.f = 0;
   return w;
 }
 __device__ __forceinline__ void walk_next(Walk& w, const int* seq_len, const Dims& d, bool append,
@@ -546,7 +572,7 @@ __device__ __forceinline__ long long warp_slot(int ctas, int P, int p) {
 // warp's final state.
 struct SegRec {
   long long U;      // first cost unit of the pair
-  int p, pc, nb, nr;
+  int p, pc, nb, nr, f;
 };
 
 // Row o / l of every head of a WarpState into out (a pair's only partial).
@@ -568,7 +594,7 @@ __device__ void final_merge(const SegRec& r, const FlatGrid& g, const Dims& d, c
   const int P = d.batch * d.hkv, gq = d.gq;
   int c_a, n_cta;
   bool cont;
-  const int cnt = pair_partials(r.U, r.pc, r.nb, r.nr, g, c_a, n_cta, cont);
+  const int cnt = pair_partials(r.U, r.pc, r.nb, r.nr, r.f, g, c_a, n_cta, cont);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rows = gq * kHeadDim;                  // floats of one partial's rows
   float* wv = scratch;                             // [gq][cnt] maxima, then weights
@@ -740,7 +766,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
                                long long head0) {
     int c_a, n_cta;
     bool cont;
-    const int cnt = pair_partials(r.U, r.pc, r.nb, r.nr, g, c_a, n_cta, cont);
+    const int cnt = pair_partials(r.U, r.pc, r.nb, r.nr, r.f, g, c_a, n_cta, cont);
     WarpState& s = *reinterpret_cast<WarpState*>(ring);
     if (packed_kind) tc_write_state<true, BV, kWide>(st, s, lane);
     else tc_write_state<false, BV, kWide>(st, s, lane);
@@ -801,7 +827,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         continue;
       }
       const PairShape s = pair_shape(w.L, d.residual);
-      const int k0 = items_below(a - U, s.nb, s.nr, g.k), k1 = items_below(e - U, s.nb, s.nr, g.k);
+      const int k0 = items_below(a - U, s.nb, s.nr, g.k, w.f);
+      const int k1 = items_below(e - U, s.nb, s.nr, g.k, w.f);
       if (lane == 0) X.last = U + w.pc >= e;
       __syncwarp();
       if (k1 > k0) {
@@ -834,6 +861,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
           X.seg.pc = w.pc;
           X.seg.nb = s.nb;
           X.seg.nr = s.nr;
+          X.seg.f = w.f;
           X.i0 = i0;
           X.i1 = i1;
           X.j1 = j1;
@@ -943,7 +971,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     const SegRec r = rec[mg.w0[threadIdx.x]];
     int c_a, n_cta;
     bool cont;
-    mg.cnt[threadIdx.x] = pair_partials(r.U, r.pc, r.nb, r.nr, g, c_a, n_cta, cont);
+    mg.cnt[threadIdx.x] = pair_partials(r.U, r.pc, r.nb, r.nr, r.f, g, c_a, n_cta, cont);
   }
   if (threadIdx.x < ng * gq) {  // (group, head): maximum and warp weights
     const int k = threadIdx.x / gq, gg = threadIdx.x - k * gq;
