@@ -20,6 +20,7 @@
 // (-0 folded onto +0) and then by the lower index.
 
 #include <limits.h>
+#include <stddef.h>
 
 #include "common.cuh"
 
@@ -315,14 +316,10 @@ __device__ void select_top(const uint32_t (&k)[E], const int (&x)[E], int n, Sel
 constexpr int kCandReg = 16;                // candidates of a row per thread (finalize)
 constexpr size_t kW1StageMax = 168 * 1024;  // largest staged corrector W1 (256 x 168)
 
+// The union comes last: a launch that does not stage W1 (grids of more
+// CTAs than SMs, where one ~190 KB CTA per SM would run in waves) stops the
+// shared memory after its chunk-phase part (kSmemNoW1 bytes).
 struct Smem {
-  union {
-    struct {
-      uint32_t sk[kChunk];
-      int si[kChunk];
-    } srt;                              // chunk phase: the chunk's keys
-    float w1[kW1StageMax / 4];          // finalize: corrector W1 (bulk copy)
-  } u;
   uint64_t w1_bar;
   Sel sel;
   unsigned long long sv[kSurvivors];    // select_top: candidates above the bound
@@ -339,21 +336,34 @@ struct Smem {
   float red[32];
   float f;
   int last;
+  union alignas(16) {
+    struct {
+      uint32_t sk[kChunk];
+      int si[kChunk];
+    } srt;                              // chunk phase: the chunk's keys
+    float w1[kW1StageMax / 4];          // finalize: corrector W1 (bulk copy)
+  } u;
 };
+constexpr size_t kSmemNoW1 = offsetof(Smem, u) + sizeof(static_cast<Smem*>(nullptr)->u.srt);
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-// Whether the corrector's W1 is copied to shared memory in one bulk copy.
-__device__ __forceinline__ bool stage_w1(const DgapDims& d, const dgap_params& p) {
+// Whether the corrector's W1 is copied to shared memory in one bulk copy
+// (decided by the host, passed to the kernel): when it fits and the grid
+// runs in one wave of one CTA per SM.  Otherwise the finalizing CTA reads it
+// through L1 (prefetched when the CTA learns it is last).
+inline bool stage_w1(const DgapDims& d, const dgap_params& p, int sm_count) {
   const size_t bytes = (size_t)d.hidden * (5 * d.K + 8) * sizeof(float);
   return bytes <= kW1StageMax && bytes % 16 == 0 &&
-         (reinterpret_cast<uintptr_t>(p.cor_w1) & 15) == 0;
+         (reinterpret_cast<uintptr_t>(p.cor_w1) & 15) == 0 &&
+         (long long)d.n_chunks * d.batch <= sm_count;
 }
 
 __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* logits, int row,
                              int32_t* topk_idx, float* topk_val, float* risk, uint8_t* gate,
-                             int32_t* next_token, float* features, const DWs& ws, Smem& sm) {
+                             int32_t* next_token, float* features, const DWs& ws, Smem& sm,
+                             int w1_staged) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int K = d.K, K1 = d.K + 1, nc = d.n_chunks;
   const int nin = 5 * K + 8;
@@ -361,8 +371,12 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
 
   // The corrector's first layer, fetched while the window is formed (only
   // used when the row is gated; always awaited before the CTA exits).
-  const bool w1s = stage_w1(d, p);
+  const bool w1s = w1_staged != 0;
   const uint32_t w1_bytes = (uint32_t)((size_t)d.hidden * nin * sizeof(float));
+  const bool w1v = (nin & 3) == 0 && (reinterpret_cast<uintptr_t>(p.cor_w1) & 15) == 0;
+  if (!w1s && w1v)  // every 128-byte line of W1 into L1 while the window is formed
+    for (uint32_t o = (uint32_t)tid * 128u; o < w1_bytes; o += (uint32_t)kT * 128u)
+      asm volatile("prefetch.global.L1 [%0];" ::"l"(reinterpret_cast<const char*>(p.cor_w1) + o));
   if (w1s && tid == 0) {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // chunk-phase writes first
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&sm.w1_bar)) : "memory");
@@ -574,32 +588,37 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
     if (tid < 8) sm.x[5 * K + tid] = sm.phi[tid];
     __syncthreads();
     // Hidden layer: one thread per hidden unit (W1 from shared memory when
-    // staged).
+    // staged, else through L1).
     const float* w1 = (w1s && w1_ok) ? sm.u.w1 : p.cor_w1;
-    if (w1s && w1_ok && (nin & 3) == 0) {
-      // staged rows of float4s, four accumulators.  With an even number n4
+    if (w1v && (!w1s || w1_ok)) {
+      // rows of float4s (shared memory when staged, else global memory
+      // through L1), four accumulators.  With an even number n4
       // of float4s per row, thread j starts at column j mod 8: the float4 at
       // column c of row j lies in 16-byte bank group (j n4 + c) mod 8, so the
       // eight rows a quarter-warp reads fall in groups j (n4 + 1) mod 8, all
       // different (n4 + 1 odd), and so do the eight inputs it reads.
       const float4* xv = reinterpret_cast<const float4*>(sm.x);
       const int n4 = nin / 4;
-      for (int j = tid; j < d.hidden; j += kT) {
-        const float4* wr = reinterpret_cast<const float4*>(sm.u.w1 + (size_t)j * nin);
-        float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-        int c = (n4 & 1) ? 0 : (j & 7) % n4;
+      const auto rows = [&](auto load) {
+        for (int j = tid; j < d.hidden; j += kT) {
+          const float4* wr = reinterpret_cast<const float4*>(w1 + (size_t)j * nin);
+          float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+          int c = (n4 & 1) ? 0 : (j & 7) % n4;
 #pragma unroll 6
-        for (int t = 0; t < n4; ++t) {
-          const float4 w = wr[c], xx = xv[c];
-          c = c + 1 == n4 ? 0 : c + 1;
-          a.x = fmaf(w.x, xx.x, a.x);
-          a.y = fmaf(w.y, xx.y, a.y);
-          a.z = fmaf(w.z, xx.z, a.z);
-          a.w = fmaf(w.w, xx.w, a.w);
+          for (int t = 0; t < n4; ++t) {
+            const float4 w = load(wr + c), xx = xv[c];
+            c = c + 1 == n4 ? 0 : c + 1;
+            a.x = fmaf(w.x, xx.x, a.x);
+            a.y = fmaf(w.y, xx.y, a.y);
+            a.z = fmaf(w.z, xx.z, a.z);
+            a.w = fmaf(w.w, xx.w, a.w);
+          }
+          const float b1 = j == tid ? cb1 : __ldg(p.cor_b1 + j);
+          sm.hb[j] = fmaxf((a.x + a.y) + (a.z + a.w) + b1, 0.0f);
         }
-        const float b1 = j == tid ? cb1 : __ldg(p.cor_b1 + j);
-        sm.hb[j] = fmaxf((a.x + a.y) + (a.z + a.w) + b1, 0.0f);
-      }
+      };
+      if (w1s) rows([](const float4* q) { return *q; });
+      else rows([](const float4* q) { return __ldg(q); });
     } else
     for (int j = tid; j < d.hidden; j += kT) {
       const float* wrow = w1 + (size_t)j * nin;
@@ -675,10 +694,11 @@ __device__ void finalize_row(const DgapDims& d, const dgap_params& p, float* log
   }
 }
 
-__global__ void __launch_bounds__(kT, 1)
+// Two CTAs per SM when W1 is not staged (at most 128 registers).
+__global__ void __launch_bounds__(kT, 2)
     dgap_kernel(DgapDims d, dgap_params p, float* __restrict__ logits, int32_t* topk_idx,
                 float* topk_val, float* risk, uint8_t* gate, int32_t* next_token,
-                float* features, DWs ws) {
+                float* features, DWs ws, int w1_staged) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
   // programmatic dependent launch: the logits are the previous kernel's output
@@ -744,7 +764,8 @@ __global__ void __launch_bounds__(kT, 1)
   }
   __syncthreads();
   if (!sm.last) return;
-  finalize_row(d, p, logits, row, topk_idx, topk_val, risk, gate, next_token, features, ws, sm);
+  finalize_row(d, p, logits, row, topk_idx, topk_val, risk, gate, next_token, features, ws, sm,
+               w1_staged);
 }
 
 }  // namespace
@@ -762,10 +783,18 @@ cudaError_t launch_dgap(const DgapDims& d, const dgap_params& p, float* logits, 
                         float* topk_val, float* risk, uint8_t* gate, int32_t* next_token,
                         float* features, void* workspace, cudaStream_t stream) {
   const DWs ws = carve(workspace, d.batch, d.n_chunks, d.K);
-  const size_t smem = sizeof(Smem);
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return cudaGetLastError();
+  }
+  const int w1_staged = stage_w1(d, p, sms) ? 1 : 0;
+  const size_t smem = w1_staged ? sizeof(Smem) : kSmemNoW1;
   static_assert(sizeof(Smem) <= 227 * 1024, "DGAP shared memory must fit one SM");
   cudaError_t e = cudaFuncSetAttribute(dgap_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+                                       (int)sizeof(Smem));
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(d.n_chunks, d.batch);
@@ -778,7 +807,7 @@ cudaError_t launch_dgap(const DgapDims& d, const dgap_params& p, float* logits, 
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   e = cudaLaunchKernelEx(&cfg, dgap_kernel, d, p, logits, topk_idx, topk_val, risk, gate,
-                         next_token, features, ws);
+                         next_token, features, ws, w1_staged);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
